@@ -1,0 +1,379 @@
+/*
+ * ppd_oracle.c -- slow, plain fp64 CPU reference for the verification step of
+ * Parallel Prompt Decoding (PPD).
+ *
+ * TEST INFRASTRUCTURE, NOT PRODUCT CODE.  Only the test-suite, the smoke check
+ * and the benchmark's CPU-baseline / reference arm may load this library.  It
+ * shares no source, header, table or helper with the CUDA implementation.
+ *
+ * Every function is the direct definition of one step, written with plain
+ * loops in the paper's order so that it can be checked against the paper by
+ * eye.  Floating point is fp64 throughout; inputs stored as bf16 are widened
+ * exactly, inputs stored as fp32 are first rounded to bf16 (round to nearest,
+ * ties to even) by this file's own bit routine.
+ *
+ *   oracle_round_bf16      fp32 -> bf16 rounding (IEEE 754 round-half-even)
+ *   oracle_tree_attention  tree-masked attention (Section 3 step (1); Section
+ *                          4.1: every tree token sees the cached prefix, its
+ *                          tree ancestors and itself)
+ *   oracle_node_argmax     top-1 token of every tree node's logits (the
+ *                          greedy "exact matching" check of Section 3 (2))
+ *   oracle_accept_path     longest accepted root-to-node path (Section 3
+ *                          steps (2)-(3), exact matching)
+ *   oracle_kv_compact      copy the accepted nodes' K/V into the cache
+ *                          (Section 3 step (3), "KV cache is updated")
+ *
+ * Status codes (per sequence): 0 ok, 3 malformed tree, 4 capacity / prefix
+ * length out of range.  Whole-call argument errors return 1.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+enum {
+    ORC_OK = 0,
+    ORC_ERR_INVALID_ARG = 1,
+    ORC_ERR_TREE = 3,
+    ORC_ERR_CAPACITY = 4
+};
+
+/* ------------------------------------------------------------------ bf16 */
+
+/* fp32 -> bf16 with round-to-nearest, ties-to-even on the 16 dropped bits.
+ * A carry out of the mantissa correctly bumps the exponent (and the largest
+ * finite values round to infinity).  NaN stays NaN (quiet bit forced on). */
+static uint16_t round_to_bf16(float x)
+{
+    uint32_t u;
+    memcpy(&u, &x, sizeof u);
+    if ((u & 0x7f800000u) == 0x7f800000u) {
+        if (u & 0x007fffffu)
+            return (uint16_t)((u >> 16) | 0x0040u);
+        return (uint16_t)(u >> 16);
+    }
+    uint32_t kept = u >> 16;
+    uint32_t dropped = u & 0xffffu;
+    if (dropped > 0x8000u || (dropped == 0x8000u && (kept & 1u)))
+        kept += 1u;
+    return (uint16_t)kept;
+}
+
+static double bf16_to_double(uint16_t h)
+{
+    uint32_t u = (uint32_t)h << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+void oracle_round_bf16(const float *x, uint16_t *y, int64_t n)
+{
+    for (int64_t i = 0; i < n; ++i)
+        y[i] = round_to_bf16(x[i]);
+}
+
+/* element `idx` of a tensor stored as bf16 (dtype 0) or fp32 (dtype 1),
+ * as the bf16 value it denotes, widened to double */
+static double load(const void *base, int64_t idx, int dtype)
+{
+    if (dtype == 0)
+        return bf16_to_double(((const uint16_t *)base)[idx]);
+    return bf16_to_double(round_to_bf16(((const float *)base)[idx]));
+}
+
+/* ------------------------------------------------------------------ trees */
+
+/* A tree is valid when node 0 is the root (parent -1) and every other node's
+ * parent precedes it (topological order), so each node has one path to 0. */
+static int tree_is_valid(const int32_t *parent, int T)
+{
+    if (T < 1 || parent[0] != -1)
+        return 0;
+    for (int i = 1; i < T; ++i)
+        if (parent[i] < 0 || parent[i] >= i)
+            return 0;
+    return 1;
+}
+
+/* ------------------------------------------------------------------ attention */
+
+/*
+ * Tree-masked attention, one output row per (layer, sequence, head, tree node).
+ * Query i of sequence b sees the keys of cache rows 0..P_b-1 and of the tree
+ * nodes on its own root path (its ancestors and itself).  With s_j =
+ * scale * <q_i, k_j> over those keys: o_i = sum_j exp(s_j - m) v_j /
+ * sum_j exp(s_j - m), m = max_j s_j (two passes, fp64).
+ *
+ * Layouts (row-major): q, k_tree, v_tree [L,B,H,T,D]; k_cache, v_cache
+ * [L,B,H,S_max,D]; prefix_len [B]; parent [B,T].  `units` lists which
+ * (l*B + b)*H + h slices to compute (NULL: all, in order); out is
+ * [n_units,T,D], lse and rowsum (nullable) [n_units,T].  A sequence with a
+ * malformed tree or a prefix length outside [0, S_max] gets status 3 / 4 and
+ * NaN outputs.
+ */
+int oracle_tree_attention(const void *q, const void *k_cache, const void *v_cache,
+                          const void *k_tree, const void *v_tree, int dtype,
+                          const int32_t *prefix_len, const int32_t *parent,
+                          int L, int B, int H, int T, int D, int S_max, double scale,
+                          const int64_t *units, int64_t n_units,
+                          double *out, double *lse, double *rowsum,
+                          int32_t *status, int n_threads)
+{
+    if (L < 1 || B < 1 || H < 1 || T < 1 || D < 1 || S_max < 0 || (dtype != 0 && dtype != 1))
+        return ORC_ERR_INVALID_ARG;
+    if (scale <= 0.0)
+        scale = 1.0 / sqrt((double)D);
+    int64_t total = (int64_t)L * B * H;
+    if (units == NULL)
+        n_units = total;
+
+    int32_t *st = (int32_t *)calloc((size_t)B, sizeof(int32_t));
+    for (int b = 0; b < B; ++b) {
+        if (!tree_is_valid(parent + (int64_t)b * T, T))
+            st[b] = ORC_ERR_TREE;
+        else if (prefix_len[b] < 0 || prefix_len[b] > S_max)
+            st[b] = ORC_ERR_CAPACITY;
+    }
+    if (status)
+        memcpy(status, st, (size_t)B * sizeof(int32_t));
+
+#ifdef _OPENMP
+    if (n_threads > 0)
+        omp_set_num_threads(n_threads);
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+    for (int64_t n = 0; n < n_units; ++n) {
+        int64_t u = units ? units[n] : n;
+        int b = (int)((u / H) % B);
+        double *o_unit = out + n * (int64_t)T * D;
+        if (u < 0 || u >= total || st[b] != ORC_OK) {
+            for (int64_t e = 0; e < (int64_t)T * D; ++e)
+                o_unit[e] = NAN;
+            for (int i = 0; i < T; ++i) {
+                if (lse) lse[n * T + i] = NAN;
+                if (rowsum) rowsum[n * T + i] = NAN;
+            }
+            continue;
+        }
+        const int32_t *par = parent + (int64_t)b * T;
+        int P = prefix_len[b];
+        int64_t q_base = u * (int64_t)T * D;          /* [T,D] slice of q / tree K,V */
+        int64_t c_base = u * (int64_t)S_max * D;      /* [S_max,D] slice of the cache */
+        double *s = (double *)malloc(sizeof(double) * (size_t)(P + T));
+        int *key_node = (int *)malloc(sizeof(int) * (size_t)T);
+
+        for (int i = 0; i < T; ++i) {
+            /* visible tree keys: walk from node i up to the root */
+            int n_tree = 0;
+            for (int a = i; a >= 0; a = par[a])
+                key_node[n_tree++] = a;
+
+            /* scores */
+            int n_keys = P + n_tree;
+            for (int j = 0; j < P; ++j) {
+                double dot = 0.0;
+                for (int d = 0; d < D; ++d)
+                    dot += load(q, q_base + (int64_t)i * D + d, dtype) *
+                           load(k_cache, c_base + (int64_t)j * D + d, dtype);
+                s[j] = scale * dot;
+            }
+            for (int t = 0; t < n_tree; ++t) {
+                double dot = 0.0;
+                for (int d = 0; d < D; ++d)
+                    dot += load(q, q_base + (int64_t)i * D + d, dtype) *
+                           load(k_tree, q_base + (int64_t)key_node[t] * D + d, dtype);
+                s[P + t] = scale * dot;
+            }
+
+            /* softmax: max, then normaliser */
+            double m = -INFINITY;
+            for (int j = 0; j < n_keys; ++j)
+                if (s[j] > m) m = s[j];
+            double denom = 0.0;
+            for (int j = 0; j < n_keys; ++j)
+                denom += exp(s[j] - m);
+
+            /* weighted sum of the visible value rows */
+            double *o = o_unit + (int64_t)i * D;
+            for (int d = 0; d < D; ++d)
+                o[d] = 0.0;
+            double psum = 0.0;
+            for (int j = 0; j < n_keys; ++j) {
+                double p = exp(s[j] - m) / denom;
+                psum += p;
+                for (int d = 0; d < D; ++d) {
+                    double v = (j < P) ? load(v_cache, c_base + (int64_t)j * D + d, dtype)
+                                       : load(v_tree, q_base + (int64_t)key_node[j - P] * D + d, dtype);
+                    o[d] += p * v;
+                }
+            }
+            if (lse) lse[n * T + i] = m + log(denom);
+            if (rowsum) rowsum[n * T + i] = psum;
+        }
+        free(s);
+        free(key_node);
+    }
+    free(st);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------ argmax */
+
+/*
+ * Top-1 token of each logits row [rows, V] (fp32): the lowest index holding
+ * the maximum.  NaN ranks above every number and the first NaN wins (the
+ * convention of numpy.argmax); -0 and +0 compare equal.
+ */
+void oracle_node_argmax(const float *logits, int64_t rows, int64_t V, int32_t *out)
+{
+    for (int64_t r = 0; r < rows; ++r) {
+        const float *x = logits + r * V;
+        int64_t best = 0;
+        float best_v = x[0];
+        if (!isnan(best_v)) {
+            for (int64_t v = 1; v < V; ++v) {
+                if (isnan(x[v])) {
+                    best = v;
+                    break;
+                }
+                if (x[v] > best_v) {
+                    best = v;
+                    best_v = x[v];
+                }
+            }
+        }
+        out[r] = (int32_t)best;
+    }
+}
+
+/* ------------------------------------------------------------------ accept */
+
+/*
+ * Exact-matching acceptance of one tree per sequence.
+ *
+ * Node 0 (the root, the last accepted token) is always accepted.  A node i > 0
+ * is accepted when it is a candidate token (cand[i] >= 0) equal to the top-1
+ * token predicted at its parent, argmax[parent[i]], and its parent is
+ * accepted (recursive definition along the parent pointer).  The chosen end
+ * node is the accepted node of greatest depth, the smallest index among equal
+ * depths; the path is its root path in depth order, accept_len its length
+ * (root included), next_token the top-1 token at the end node and
+ * new_prefix_len = prefix_len + accept_len.
+ *
+ * Errors (status 3: malformed tree or a token id outside [-1, V), root id
+ * outside [0, V); status 4: prefix_len outside [0, S_max] or the path does
+ * not fit in the cache) leave accept_len 0, path all -1, next_token -1 and
+ * new_prefix_len = prefix_len.
+ */
+int oracle_accept_path(const int32_t *argmax, const int32_t *cand, const int32_t *parent,
+                       const int32_t *prefix_len, int B, int T, int V, int S_max,
+                       int32_t *accept_len, int32_t *path, int32_t *next_token,
+                       int32_t *new_prefix_len, int32_t *status)
+{
+    if (B < 1 || T < 1 || V < 1)
+        return ORC_ERR_INVALID_ARG;
+    int *depth = (int *)malloc(sizeof(int) * (size_t)T);
+    int *acc = (int *)malloc(sizeof(int) * (size_t)T);
+    for (int b = 0; b < B; ++b) {
+        const int32_t *par = parent + (int64_t)b * T;
+        const int32_t *tok = cand + (int64_t)b * T;
+        const int32_t *top = argmax + (int64_t)b * T;
+        int32_t *pth = path + (int64_t)b * T;
+        int P = prefix_len[b];
+        int err = ORC_OK;
+
+        if (!tree_is_valid(par, T) || tok[0] < 0 || tok[0] >= V)
+            err = ORC_ERR_TREE;
+        for (int i = 1; i < T && err == ORC_OK; ++i)
+            if (tok[i] < -1 || tok[i] >= V)
+                err = ORC_ERR_TREE;
+        if (err == ORC_OK && (P < 0 || P > S_max))
+            err = ORC_ERR_CAPACITY;
+
+        int best = 0;
+        if (err == ORC_OK) {
+            depth[0] = 0;
+            acc[0] = 1;
+            for (int i = 1; i < T; ++i) {
+                int p = par[i];
+                depth[i] = depth[p] + 1;
+                int ok = tok[i] >= 0 && tok[i] == top[p];
+                acc[i] = ok && acc[p];
+            }
+            for (int i = 1; i < T; ++i)
+                if (acc[i] && depth[i] > depth[best])
+                    best = i;
+            if ((int64_t)P + depth[best] + 1 > S_max)
+                err = ORC_ERR_CAPACITY;
+        }
+
+        for (int i = 0; i < T; ++i)
+            pth[i] = -1;
+        if (err != ORC_OK) {
+            accept_len[b] = 0;
+            next_token[b] = -1;
+            new_prefix_len[b] = P;
+        } else {
+            int n = depth[best] + 1;
+            int k = n - 1;
+            for (int a = best; a >= 0; a = par[a])
+                pth[k--] = a;
+            accept_len[b] = n;
+            next_token[b] = top[best];
+            new_prefix_len[b] = P + n;
+        }
+        status[b] = err;
+    }
+    free(depth);
+    free(acc);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------ compaction */
+
+/*
+ * For every (layer, sequence, head): cache row prefix_len[b] + j <- tree row
+ * path[b][j] for j < accept_len[b], for K and V.  Rows are copied as raw bytes
+ * (elem_bytes per element).  Every other cache row is left untouched.
+ * Sequences whose accept_len is 0 are skipped; a path entry outside [0, T) or
+ * a destination beyond S_max makes the call return 1 without copying that row.
+ */
+int oracle_kv_compact(void *k_cache, void *v_cache, const void *k_tree, const void *v_tree,
+                      const int32_t *path, const int32_t *accept_len, const int32_t *prefix_len,
+                      int L, int B, int H, int T, int D, int S_max, int elem_bytes)
+{
+    int rc = ORC_OK;
+    size_t row = (size_t)D * (size_t)elem_bytes;
+    for (int l = 0; l < L; ++l)
+        for (int b = 0; b < B; ++b)
+            for (int h = 0; h < H; ++h) {
+                int64_t u = ((int64_t)l * B + b) * H + h;
+                int n = accept_len[b];
+                for (int j = 0; j < n; ++j) {
+                    int src = path[(int64_t)b * T + j];
+                    int64_t dst = (int64_t)prefix_len[b] + j;
+                    if (src < 0 || src >= T || dst < 0 || dst >= S_max) {
+                        rc = ORC_ERR_INVALID_ARG;
+                        continue;
+                    }
+                    memcpy((char *)k_cache + ((u * S_max + dst) * (int64_t)row),
+                           (const char *)k_tree + ((u * T + src) * (int64_t)row), row);
+                    memcpy((char *)v_cache + ((u * S_max + dst) * (int64_t)row),
+                           (const char *)v_tree + ((u * T + src) * (int64_t)row), row);
+                }
+            }
+    return rc;
+}
+
+int oracle_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
