@@ -1,0 +1,180 @@
+/*
+ * ppd.h -- C ABI of libppd, the GB300 (sm_103a) implementation of the
+ * verification step of Parallel Prompt Decoding (PPD).
+ *
+ * One PPD decode step runs a single forward pass over a token tree: the root
+ * (the last accepted token), candidate ("guess") tokens, and a chain of prompt
+ * tokens hanging below each candidate (paper Section 3; Section 4.1).  The
+ * verification part of that step, which this library implements, is:
+ *
+ *   1. tree-masked attention: every tree token attends to the KV-cache prefix,
+ *      its tree ancestors and itself (Section 3, step (1), tree attention;
+ *      Section 4.1, the attention mask over the tree-structured input);
+ *   2. node argmax: the model's top-1 token after every tree node (the greedy
+ *      "exact matching" check of Section 3, step (2));
+ *   3. acceptance: the longest root-to-node path whose every candidate equals
+ *      the top-1 token at its parent (Section 3, steps (2)-(3));
+ *   4. compaction: the accepted nodes' K/V rows enter the cache (Section 3,
+ *      step (3), "KV cache is updated accordingly").
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - All tensor pointers are DEVICE memory, row-major (last index fastest),
+ *    owned by the caller.  The library never allocates, frees or synchronises;
+ *    work is enqueued on `stream` (a cudaStream_t passed as void*; NULL = the
+ *    legacy default stream).  A PPD_OK return means the arguments passed the
+ *    host-side checks and the work was enqueued; errors found on the device
+ *    are reported per sequence in `dev_status`.
+ *  - Shapes: L layers, B sequences, H heads (K/V heads == query heads), D head
+ *    dim (64 or 128), T tree tokens (1..128), S_max cache rows per
+ *    (layer, sequence, head), V vocab size.
+ *  - Q, tree K/V and the attention output are [L,B,H,T,D]; the K/V cache is
+ *    [L,B,H,S_max,D]; rows [0, prefix_len[b]) of sequence b are the valid
+ *    prefix.  Q/K/V are bf16 (PPD_BF16) or fp32 (PPD_F32, rounded to bf16 on
+ *    load, round-to-nearest-even).  Attention accumulates in fp32.
+ *  - parent[b][0] = -1 and 0 <= parent[b][i] < i (topological order).  Trees
+ *    may differ per sequence.  cand_tokens[b][i] is the token id of node i:
+ *    in [0, V) for the root and the candidates, -1 for prompt-token nodes.
+ *  - Argmax ties break to the lowest index; NaN ranks above every number and
+ *    the first NaN wins; -0 equals +0.
+ *  - The default softmax scale (scale <= 0) is 1/sqrt(D).
+ *  - Tree buffers must not overlap the cache buffers.
+ *
+ * Per-sequence device status (dev_status[b]): PPD_OK, PPD_ERR_TREE (malformed
+ * parent array, or a token id out of range), PPD_ERR_CAPACITY (prefix_len
+ * outside [0, S_max], or prefix_len + accepted length > S_max), or
+ * PPD_ERR_TIMEOUT (an internal wait gave up; the outputs of that call are
+ * undefined).  A sequence with a non-zero status gets accept_len 0, path all
+ * -1, next_token -1, new_prefix_len = prefix_len, and no cache write.
+ */
+#ifndef PPD_H
+#define PPD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PPD_OK = 0,
+    PPD_ERR_INVALID_ARG = 1, /* host-side argument check failed; nothing enqueued */
+    PPD_ERR_UNSUPPORTED = 2, /* valid request outside what this build supports */
+    PPD_ERR_TREE = 3,        /* device: malformed tree or token id */
+    PPD_ERR_CAPACITY = 4,    /* device: prefix / accepted rows exceed S_max */
+    PPD_ERR_CUDA = 5,        /* a CUDA runtime call failed */
+    PPD_ERR_TIMEOUT = 6      /* device: a bounded internal wait expired */
+} ppd_status;
+
+typedef enum { PPD_BF16 = 0, PPD_F32 = 1 } ppd_dtype;
+
+/*
+ * Scratch bytes the entry points below need in `workspace` for these sizes
+ * (device memory, any contents, 256-byte aligned, caller-owned; it may be
+ * reused between calls that are ordered on one stream).  Covers argmax
+ * partial results and counters and, for PPD_F32, the bf16 copies of Q/K/V.
+ */
+size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt);
+
+/*
+ * Tree-masked attention (Section 3 step (1), Section 4.1).  For every layer l,
+ * sequence b, head h and tree node i:
+ *     o = sum_j softmax_j(scale * <q_i, k_j>) v_j
+ * over the keys j in {cache rows 0..prefix_len[b]-1} U {tree nodes on the
+ * path from i to the root, i included}.
+ *   q, k_tree, v_tree  [L,B,H,T,D]      k_cache, v_cache [L,B,H,S_max,D]
+ *   prefix_len int32[B]                 parent int32[B,T]
+ *   out  fp32 [L,B,H,T,D]               lse  fp32 [L,B,H,T] natural-log
+ *                                       log-sum-exp of the scaled scores, or NULL
+ *   dev_status int32[B] (required): set to 0, or to PPD_ERR_TREE /
+ *   PPD_ERR_CAPACITY / PPD_ERR_TIMEOUT; outputs of a failed sequence are
+ *   unspecified.  Cache rows at or beyond prefix_len[b] are never used and may
+ *   hold anything, NaN included.
+ * Workspace: ppd_workspace_bytes(...) bytes (only PPD_F32 uses it).
+ */
+ppd_status ppd_tree_attention(const void *q, const void *k_cache, const void *v_cache,
+                              const void *k_tree, const void *v_tree,
+                              const int32_t *prefix_len, const int32_t *parent,
+                              int L, int B, int H, int T, int D, int S_max, ppd_dtype dt,
+                              float scale, float *out, float *lse, int32_t *dev_status,
+                              void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Node argmax (Section 3 step (2), exact matching needs the top-1 token after
+ * every tree node).  logits fp32 [B,T,V] -> argmax_out int32 [B,T], lowest
+ * index on ties, first NaN wins.  Workspace: ppd_workspace_bytes(...) bytes.
+ */
+ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *argmax_out,
+                           void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Exact-matching acceptance (Section 3 steps (2)-(3)).  Node 0 is always
+ * accepted; node i > 0 is accepted when cand_tokens[b][i] >= 0 equals
+ * argmax[b][parent[b][i]] and its parent is accepted.  The end node is the
+ * deepest accepted node (smallest index among equal depths).
+ *   argmax, cand_tokens, parent int32[B,T]; prefix_len int32[B]
+ *   accept_len int32[B]   accepted tokens, root included (>= 1 on success)
+ *   path int32[B,T]       accepted node ids in depth order, then -1
+ *   next_token int32[B]   argmax at the end node (the next root token)
+ *   new_prefix_len int32[B] = prefix_len + accept_len
+ *   dev_status int32[B]   see the file header
+ */
+ppd_status ppd_accept_path(const int32_t *argmax, const int32_t *cand_tokens,
+                           const int32_t *parent, const int32_t *prefix_len,
+                           int B, int T, int V, int S_max,
+                           int32_t *accept_len, int32_t *path, int32_t *next_token,
+                           int32_t *new_prefix_len, int32_t *dev_status, void *stream);
+
+/*
+ * KV compaction (Section 3 step (3)).  For every l, b, h and j <
+ * accept_len[b]:  cache[l,b,h,prefix_len[b]+j,:] <- tree[l,b,h,path[b][j],:]
+ * for K and V, bit for bit (2 bytes per element for PPD_BF16, 4 for PPD_F32).
+ * No other cache row is written.  Rows whose source or destination index is
+ * out of range are skipped.
+ */
+ppd_status ppd_kv_compact(void *k_cache, void *v_cache, const void *k_tree, const void *v_tree,
+                          const int32_t *path, const int32_t *accept_len,
+                          const int32_t *prefix_len, int L, int B, int H, int T, int D,
+                          int S_max, ppd_dtype dt, void *stream);
+
+/*
+ * The whole verification step: node argmax and acceptance, tree-masked
+ * attention over all L layers, then compaction of the accepted rows, enqueued
+ * on `stream` with no host synchronisation.  Arguments as in the four entry
+ * points above; `out`/`lse` as in ppd_tree_attention, `argmax_out` as in
+ * ppd_node_argmax.  Attention reads only prefix rows [0, prefix_len[b]) and
+ * compaction writes only rows [prefix_len[b], new_prefix_len[b]), so the
+ * result equals running the four steps one after another.
+ */
+ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
+                           const void *k_tree, const void *v_tree,
+                           const int32_t *prefix_len, const int32_t *parent,
+                           const int32_t *cand_tokens, const float *logits,
+                           int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt,
+                           float scale, float *out, float *lse, int32_t *argmax_out,
+                           int32_t *accept_len, int32_t *path, int32_t *next_token,
+                           int32_t *new_prefix_len, int32_t *dev_status,
+                           void *workspace, size_t ws_bytes, void *stream);
+
+/* Human-readable name of a status code (static string). */
+const char *ppd_status_string(ppd_status s);
+
+/*
+ * Diagnostic (no paper counterpart): one 128 x N x 128 bf16 tensor-core product
+ * through the same shared-memory layouts the attention kernel uses, so that a
+ * test can check them against a plain matrix product.
+ *   mode 0: d[128][N] = a[128][128] * b[N][128]^T   (both operands K-major)
+ *   mode 1: d[128][N] = a[128][128]^T * b[128][N]   (a given [K][M], b given
+ *           [K][N]: both operands M/N-major; b is written by threads)
+ *   mode 2: as mode 1 with a given [K][64]; rows 64..127 of d repeat rows 0..63
+ * N in {16, 32, ..., 256}; a, b bf16 device pointers; d fp32 [128][N].
+ */
+ppd_status ppd_selftest_umma(const void *a, const void *b, float *d, int mode, int N,
+                             void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PPD_H */

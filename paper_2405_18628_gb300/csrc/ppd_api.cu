@@ -1,0 +1,398 @@
+// ppd_api.cu -- the C ABI of libppd (declared in include/ppd.h): host-side
+// argument checks, workspace layout, TMA tensor-map encoding and the launch
+// sequence of each entry point.  No entry point allocates, frees or
+// synchronises; all work is enqueued on the caller's stream.
+#include "ppd.h"
+#include "ppd_kernels.h"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+namespace {
+
+using ppd::AcceptArgs;
+using ppd::ArgmaxScratch;
+using ppd::AttnMaps;
+using ppd::AttnParams;
+
+constexpr int kMaxT = 128;
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// byte ranges [a, a+na) and [b, b+nb) intersect
+bool overlaps(const void *a, size_t na, const void *b, size_t nb)
+{
+    const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+    return x < y + nb && y < x + na;
+}
+
+int num_sms()
+{
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (cache[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+        cache[dev] = n;
+    }
+    return cache[dev];
+}
+
+// Argmax splits per row: enough blocks to cover the GPU, chunks >= 2048 logits.
+int argmax_splits(int64_t rows, int V)
+{
+    if (rows <= 0) return 1;
+    int64_t want = (1024 + rows - 1) / rows;
+    int64_t cap = V / 2048;
+    if (cap > 64) cap = 64;
+    if (cap < 1) cap = 1;
+    if (want > cap) want = cap;
+    if (want < 1) want = 1;
+    return (int)want;
+}
+
+struct WsLayout {
+    size_t part_val, part_idx, row_count, seq_count, conv, total;
+    int splits;
+};
+
+WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt)
+{
+    WsLayout w{};
+    const int64_t rows = (int64_t)B * T;
+    w.splits = argmax_splits(rows, V);
+    size_t off = 0;
+    w.part_val = off;
+    off = align_up(off + (size_t)rows * w.splits * 4);
+    w.part_idx = off;
+    off = align_up(off + (size_t)rows * w.splits * 4);
+    w.row_count = off;
+    off = align_up(off + (size_t)rows * 4);
+    w.seq_count = off;
+    off = align_up(off + (size_t)B * 4);
+    w.conv = off;
+    if (dt == PPD_F32) {
+        const size_t lbh = (size_t)L * B * H;
+        off = align_up(off + lbh * ((size_t)3 * T + 2 * (size_t)S_max) * D * 2);
+    }
+    w.total = off;
+    return w;
+}
+
+// ------------------------------------------------------------------ tensor maps
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// bf16 tensor viewed as [depth][rows][inner], box {64, box_rows, 1}, 128-byte swizzle,
+// out-of-range rows read as zero.
+bool encode_3d(CUtensorMap *m, const void *base, uint64_t inner, uint64_t rows, uint64_t depth,
+               uint32_t box_rows)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    const cuuint64_t dims[3] = {inner, rows, depth};
+    const cuuint64_t strides[2] = {inner * 2, inner * 2 * rows};
+    const cuuint32_t box[3] = {64, box_rows, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_2d(CUtensorMap *m, const void *base, uint64_t inner, uint64_t rows, uint32_t box_rows)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    const cuuint64_t dims[2] = {inner, rows};
+    const cuuint64_t strides[1] = {inner * 2};
+    const cuuint32_t box[2] = {64, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+ppd_status cuda_status(cudaError_t e) { return e == cudaSuccess ? PPD_OK : PPD_ERR_CUDA; }
+
+// ------------------------------------------------------------------ shared checks
+
+bool attn_dims_ok(int L, int B, int H, int T, int D, int S_max, ppd_dtype dt)
+{
+    if (L < 1 || B < 1 || H < 1 || T < 1 || T > kMaxT || S_max < 1) return false;
+    if (D != 64 && D != 128) return false;
+    if (dt != PPD_BF16 && dt != PPD_F32) return false;
+    const double lbh = (double)L * B * H;
+    if (lbh > 2147483647.0 || lbh * S_max * D > 9.0e15) return false;
+    return true;
+}
+
+// Enqueue the attention of all L*B*H slices (bf16 operands).
+ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, const void *kt,
+                             const void *vt, const int32_t *prefix_len, const int32_t *parent,
+                             int L, int B, int H, int T, int D, int S_max, float scale, float *out,
+                             float *lse, int32_t *dev_status, cudaStream_t stream)
+{
+    const int T_pad = (T + 31) & ~31;
+    const uint64_t lbh = (uint64_t)L * B * H;
+    AttnMaps m;
+    if (!encode_3d(&m.q, q, D, T, lbh, T_pad) || !encode_3d(&m.kc, kc, D, S_max, lbh, 128) ||
+        !encode_3d(&m.vc, vc, D, S_max, lbh, 128) || !encode_3d(&m.kt, kt, D, T, lbh, 128) ||
+        !encode_3d(&m.vt, vt, D, T, lbh, 128))
+        return PPD_ERR_CUDA;
+    AttnParams p{};
+    p.prefix_len = prefix_len;
+    p.parent = parent;
+    p.out = out;
+    p.lse = lse;
+    p.dev_status = dev_status;
+    p.L = L;
+    p.B = B;
+    p.H = H;
+    p.T = T;
+    p.T_pad = T_pad;
+    p.S_max = S_max;
+    p.n_units = (int)lbh;
+    const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
+    p.scale_log2 = sc * 1.4426950408889634f;
+    return cuda_status(ppd::launch_tree_attention(m, p, D, num_sms(), stream));
+}
+
+// fp32 operands: round to bf16 copies in the workspace first.
+ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, const void *kt,
+                                 const void *vt, const int32_t *prefix_len, const int32_t *parent,
+                                 int L, int B, int H, int T, int D, int S_max, ppd_dtype dt,
+                                 float scale, float *out, float *lse, int32_t *dev_status,
+                                 uint8_t *ws, const WsLayout &wl, cudaStream_t stream)
+{
+    if (dt == PPD_BF16)
+        return enqueue_attention(q, kc, vc, kt, vt, prefix_len, parent, L, B, H, T, D, S_max, scale,
+                                 out, lse, dev_status, stream);
+    const int64_t lbh = (int64_t)L * B * H;
+    const int64_t n_t = lbh * T * D, n_c = lbh * (int64_t)S_max * D;
+    uint16_t *bq = reinterpret_cast<uint16_t *>(ws + wl.conv);
+    uint16_t *bkt = bq + n_t;
+    uint16_t *bvt = bkt + n_t;
+    uint16_t *bkc = bvt + n_t;
+    uint16_t *bvc = bkc + n_c;
+    cudaError_t e;
+    if ((e = ppd::launch_round_bf16((const float *)q, bq, n_t, stream)) != cudaSuccess ||
+        (e = ppd::launch_round_bf16((const float *)kt, bkt, n_t, stream)) != cudaSuccess ||
+        (e = ppd::launch_round_bf16((const float *)vt, bvt, n_t, stream)) != cudaSuccess ||
+        (e = ppd::launch_round_bf16((const float *)kc, bkc, n_c, stream)) != cudaSuccess ||
+        (e = ppd::launch_round_bf16((const float *)vc, bvc, n_c, stream)) != cudaSuccess)
+        return PPD_ERR_CUDA;
+    return enqueue_attention(bq, bkc, bvc, bkt, bvt, prefix_len, parent, L, B, H, T, D, S_max,
+                             scale, out, lse, dev_status, stream);
+}
+
+ArgmaxScratch argmax_scratch(uint8_t *ws, const WsLayout &wl)
+{
+    ArgmaxScratch s;
+    s.part_val = reinterpret_cast<float *>(ws + wl.part_val);
+    s.part_idx = reinterpret_cast<int32_t *>(ws + wl.part_idx);
+    s.row_count = reinterpret_cast<int32_t *>(ws + wl.row_count);
+    s.seq_count = reinterpret_cast<int32_t *>(ws + wl.seq_count);
+    return s;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt)
+{
+    if (L < 1 || B < 1 || H < 1 || T < 1 || D < 1 || V < 1 || S_max < 0) return 0;
+    return workspace_layout(L, B, H, T, D, V, S_max, dt).total;
+}
+
+const char *ppd_status_string(ppd_status s)
+{
+    switch (s) {
+    case PPD_OK: return "ok";
+    case PPD_ERR_INVALID_ARG: return "invalid argument";
+    case PPD_ERR_UNSUPPORTED: return "unsupported configuration";
+    case PPD_ERR_TREE: return "malformed tree or token id";
+    case PPD_ERR_CAPACITY: return "cache capacity exceeded or prefix length out of range";
+    case PPD_ERR_CUDA: return "CUDA runtime error";
+    case PPD_ERR_TIMEOUT: return "device-side wait timed out";
+    }
+    return "unknown status";
+}
+
+ppd_status ppd_tree_attention(const void *q, const void *k_cache, const void *v_cache,
+                              const void *k_tree, const void *v_tree,
+                              const int32_t *prefix_len, const int32_t *parent,
+                              int L, int B, int H, int T, int D, int S_max, ppd_dtype dt,
+                              float scale, float *out, float *lse, int32_t *dev_status,
+                              void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!q || !k_cache || !v_cache || !k_tree || !v_tree || !prefix_len || !parent || !out ||
+        !dev_status)
+        return PPD_ERR_INVALID_ARG;
+    if (!attn_dims_ok(L, B, H, T, D, S_max, dt) || !std::isfinite(scale)) return PPD_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(k_tree, 16) ||
+        !aligned(v_tree, 16) || !aligned(out, 4) || !aligned(lse, 4))
+        return PPD_ERR_INVALID_ARG;
+    const WsLayout wl = workspace_layout(L, B, H, T, D, 1, S_max, dt);
+    if (dt == PPD_F32 && (!workspace || ws_bytes < wl.total || !aligned(workspace, kAlign)))
+        return PPD_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(dev_status, 0, (size_t)B * 4, s) != cudaSuccess) return PPD_ERR_CUDA;
+    return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B, H,
+                                 T, D, S_max, dt, scale, out, lse, dev_status,
+                                 static_cast<uint8_t *>(workspace), wl, s);
+}
+
+ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *argmax_out,
+                           void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!logits || !argmax_out || B < 1 || T < 1 || V < 1) return PPD_ERR_INVALID_ARG;
+    if ((double)B * T * V > 9.0e15 || (double)B * T * 64 > 2147483647.0) return PPD_ERR_INVALID_ARG;
+    const WsLayout wl = workspace_layout(1, B, 1, T, 1, V, 0, PPD_BF16);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    ArgmaxScratch scr{};
+    if (wl.splits > 1) {
+        if (!workspace || ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
+        scr = argmax_scratch(static_cast<uint8_t *>(workspace), wl);
+        if (cudaMemsetAsync(scr.row_count, 0, (size_t)B * T * 4, s) != cudaSuccess) return PPD_ERR_CUDA;
+    }
+    return cuda_status(
+        ppd::launch_node_argmax(logits, (int64_t)B * T, V, wl.splits, argmax_out, scr, nullptr, B, s));
+}
+
+ppd_status ppd_accept_path(const int32_t *argmax, const int32_t *cand_tokens,
+                           const int32_t *parent, const int32_t *prefix_len,
+                           int B, int T, int V, int S_max,
+                           int32_t *accept_len, int32_t *path, int32_t *next_token,
+                           int32_t *new_prefix_len, int32_t *dev_status, void *stream)
+{
+    if (!argmax || !cand_tokens || !parent || !prefix_len || !accept_len || !path || !next_token ||
+        !new_prefix_len || !dev_status)
+        return PPD_ERR_INVALID_ARG;
+    if (B < 1 || T < 1 || T > kMaxT || V < 1 || S_max < 0) return PPD_ERR_INVALID_ARG;
+    AcceptArgs a{cand_tokens, parent, prefix_len, accept_len, path, next_token, new_prefix_len,
+                 dev_status, T, V, S_max};
+    return cuda_status(ppd::launch_accept_path(argmax, a, B, static_cast<cudaStream_t>(stream)));
+}
+
+ppd_status ppd_kv_compact(void *k_cache, void *v_cache, const void *k_tree, const void *v_tree,
+                          const int32_t *path, const int32_t *accept_len,
+                          const int32_t *prefix_len, int L, int B, int H, int T, int D,
+                          int S_max, ppd_dtype dt, void *stream)
+{
+    if (!k_cache || !v_cache || !k_tree || !v_tree || !path || !accept_len || !prefix_len)
+        return PPD_ERR_INVALID_ARG;
+    if (L < 1 || B < 1 || H < 1 || T < 1 || T > kMaxT || D < 1 || S_max < 0) return PPD_ERR_INVALID_ARG;
+    if (dt != PPD_BF16 && dt != PPD_F32) return PPD_ERR_INVALID_ARG;
+    const int eb = dt == PPD_BF16 ? 2 : 4;
+    if ((D * eb) % 16 != 0) return PPD_ERR_UNSUPPORTED;
+    if (!aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(k_tree, 16) || !aligned(v_tree, 16))
+        return PPD_ERR_INVALID_ARG;
+    const size_t lbh = (size_t)L * B * H;
+    const size_t nc = lbh * S_max * D * eb, nt = lbh * T * D * eb;
+    if (overlaps(k_cache, nc, k_tree, nt) || overlaps(k_cache, nc, v_tree, nt) ||
+        overlaps(v_cache, nc, k_tree, nt) || overlaps(v_cache, nc, v_tree, nt) ||
+        overlaps(k_cache, nc, v_cache, nc))
+        return PPD_ERR_INVALID_ARG;
+    return cuda_status(ppd::launch_kv_compact(k_cache, v_cache, k_tree, v_tree, path, accept_len,
+                                              prefix_len, L, B, H, T, D, S_max, eb,
+                                              static_cast<cudaStream_t>(stream)));
+}
+
+ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
+                           const void *k_tree, const void *v_tree,
+                           const int32_t *prefix_len, const int32_t *parent,
+                           const int32_t *cand_tokens, const float *logits,
+                           int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt,
+                           float scale, float *out, float *lse, int32_t *argmax_out,
+                           int32_t *accept_len, int32_t *path, int32_t *next_token,
+                           int32_t *new_prefix_len, int32_t *dev_status,
+                           void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!q || !k_cache || !v_cache || !k_tree || !v_tree || !prefix_len || !parent ||
+        !cand_tokens || !logits || !out || !argmax_out || !accept_len || !path || !next_token ||
+        !new_prefix_len || !dev_status || !workspace)
+        return PPD_ERR_INVALID_ARG;
+    if (!attn_dims_ok(L, B, H, T, D, S_max, dt) || V < 1 || !std::isfinite(scale))
+        return PPD_ERR_INVALID_ARG;
+    if ((double)B * T * V > 9.0e15) return PPD_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(k_tree, 16) ||
+        !aligned(v_tree, 16) || !aligned(out, 4) || !aligned(lse, 4))
+        return PPD_ERR_INVALID_ARG;
+    const int eb = dt == PPD_BF16 ? 2 : 4;
+    const size_t lbh = (size_t)L * B * H;
+    const size_t nc = lbh * S_max * D * eb, nt = lbh * T * D * eb;
+    if (overlaps(k_cache, nc, k_tree, nt) || overlaps(k_cache, nc, v_tree, nt) ||
+        overlaps(v_cache, nc, k_tree, nt) || overlaps(v_cache, nc, v_tree, nt) ||
+        overlaps(k_cache, nc, v_cache, nc))
+        return PPD_ERR_INVALID_ARG;
+    const WsLayout wl = workspace_layout(L, B, H, T, D, V, S_max, dt);
+    if (ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+    // 1. node argmax; the block finishing a sequence's last row runs acceptance
+    const ArgmaxScratch scr = argmax_scratch(ws, wl);
+    if (cudaMemsetAsync(ws + wl.row_count, 0, wl.conv - wl.row_count, s) != cudaSuccess)
+        return PPD_ERR_CUDA;
+    AcceptArgs a{cand_tokens, parent, prefix_len, accept_len, path, next_token, new_prefix_len,
+                 dev_status, T, V, S_max};
+    if (ppd::launch_node_argmax(logits, (int64_t)B * T, V, wl.splits, argmax_out, scr, &a, B, s) !=
+        cudaSuccess)
+        return PPD_ERR_CUDA;
+    // 2. tree attention over every layer (reads cache rows [0, prefix_len) only)
+    ppd_status st = enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent,
+                                          L, B, H, T, D, S_max, dt, scale, out, lse, dev_status,
+                                          ws, wl, s);
+    if (st != PPD_OK) return st;
+    // 3. compaction (writes cache rows [prefix_len, prefix_len + accept_len) only)
+    return cuda_status(ppd::launch_kv_compact(k_cache, v_cache, k_tree, v_tree, path, accept_len,
+                                              prefix_len, L, B, H, T, D, S_max, eb, s));
+}
+
+ppd_status ppd_selftest_umma(const void *a, const void *b, float *d, int mode, int N, void *stream)
+{
+    if (!a || !b || !d || mode < 0 || mode > 2 || N < 16 || N > 256 || N % 16 != 0)
+        return PPD_ERR_INVALID_ARG;
+    if (mode != 0 && N % 8 != 0) return PPD_ERR_INVALID_ARG;
+    if (!aligned(a, 16) || !aligned(b, 16) || !aligned(d, 4)) return PPD_ERR_INVALID_ARG;
+    CUtensorMap ma, mb;
+    std::memset(&mb, 0, sizeof mb);
+    if (mode == 0) {
+        if (!encode_2d(&ma, a, 128, 128, 128) || !encode_2d(&mb, b, 128, N, N)) return PPD_ERR_CUDA;
+    } else {
+        if (!encode_2d(&ma, a, mode == 1 ? 128 : 64, 128, 128)) return PPD_ERR_CUDA;
+        mb = ma;
+    }
+    return cuda_status(ppd::launch_selftest_umma(ma, mb, b, d, mode, N, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,577 @@
+// ppd_attention.cu -- tree-masked attention of the PPD verification step on
+// sm_103a (paper Section 3 step (1): tree attention over the candidate tree;
+// Section 4.1: every tree token attends to the cached prefix, its tree
+// ancestors and itself).
+//
+// One persistent CTA per SM walks a list of (layer, sequence, head) units.  A
+// unit streams its KV prefix in tiles of 128 keys and finishes with one tile
+// holding the tree's own keys.  Per tile:
+//
+//   S^T = K_tile * Q^T     tcgen05.mma, M = 128 keys, N = T_pad queries, K = D
+//                          (keys on the M side, so a 64-token tree wastes no
+//                          tensor-core rows), accumulated in TMEM
+//   P   = exp2(S*scale*log2e - m)   by two softmax warpgroups, one key row per
+//                          thread, split into bf16 hi + lo parts (P = hi + lo to
+//                          ~2^-16) and written to shared memory
+//   O^T += V^T * [P_hi | P_lo]^T    one tcgen05.mma, M = D, N = 2*T_pad, K = 128
+//
+// Warp roles (320 threads): warps 0-7 softmax (two warpgroups, each owning
+// half of the query columns), warp 8 TMA producer, warp 9 MMA issuer and TMEM
+// owner.  The running row maximum m is updated lazily: a tile only triggers
+// a cross-lane max reduction (and a rescale of O and of the row sums) when
+// one of its scores exceeds the current m by more than 8 (log2 units), so
+// in steady state the softmax is purely per-thread.  The tree mask is an
+// ancestor bitset built from the parent array; rows beyond the prefix (which
+// may hold anything, NaN included) are masked by select and their V rows are
+// zeroed in shared memory before the PV product.
+#include "ppd_device.cuh"
+#include "ppd_kernels.h"
+
+#include <cmath>
+
+namespace ppd {
+
+template <int D_, int TPMAX_>
+struct AttnLayout {
+    static constexpr int D = D_;
+    static constexpr int TPMAX = TPMAX_;          // largest padded tree size served
+    static constexpr int KT = 128;                // keys per tile
+    static constexpr int DCH = D / 64;            // 64-column (128-byte) groups along D
+    static constexpr uint32_t GROUP_BYTES = KT * 128;   // one column group of a tile
+    static constexpr uint32_t TILE_BYTES = KT * D * 2;
+    static constexpr uint32_t Q_GROUP_BYTES = TPMAX * 128;
+    static constexpr uint32_t Q_BYTES = TPMAX * D * 2;
+    static constexpr int P_GROUPS = 2 * TPMAX / 64;      // [hi | lo] columns / 64
+    static constexpr uint32_t P_BYTES = P_GROUPS * GROUP_BYTES;
+    static constexpr int QS = (TPMAX <= 64) ? 2 : 1;     // Q buffers
+    static constexpr int KS = (TPMAX <= 64) ? 3 : 2;     // K tile ring
+    static constexpr int VS = 2;                          // V tile ring
+    static constexpr int NC_MAX = TPMAX / 2;              // query columns per warpgroup
+
+    static constexpr uint32_t OFF_Q = 0;
+    static constexpr uint32_t OFF_P = OFF_Q + QS * Q_BYTES;
+    static constexpr uint32_t OFF_K = OFF_P + P_BYTES;
+    static constexpr uint32_t OFF_V = OFF_K + KS * TILE_BYTES;
+    static constexpr uint32_t OFF_BAR = OFF_V + VS * TILE_BYTES;
+    // barrier indices
+    static constexpr int B_QFULL = 0;
+    static constexpr int B_QEMPTY = B_QFULL + QS;
+    static constexpr int B_KFULL = B_QEMPTY + QS;
+    static constexpr int B_KEMPTY = B_KFULL + KS;
+    static constexpr int B_VFULL = B_KEMPTY + KS;
+    static constexpr int B_VEMPTY = B_VFULL + VS;
+    static constexpr int B_SFULL = B_VEMPTY + VS;
+    static constexpr int B_SFREE = B_SFULL + 2;
+    static constexpr int B_PFULL = B_SFREE + 2;
+    static constexpr int B_PFREE = B_PFULL + 1;
+    static constexpr int B_DRAIN = B_PFREE + 1;
+    static constexpr int NBAR = B_DRAIN + 1;
+    static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
+    static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
+    static constexpr uint32_t OFF_M2 = (OFF_ABORT + 4 + 15) & ~15u;
+    static constexpr uint32_t OFF_UNION = OFF_M2 + TPMAX * 4;
+    // union: ancestor bitsets [128][4] u32, or reduction scratch [2][4][NC_MAX] f32
+    static constexpr uint32_t UNION_BYTES = 128 * 16;
+    static constexpr uint32_t SMEM_BYTES = OFF_UNION + UNION_BYTES;
+    static constexpr uint32_t TMEM_COLS = 4 * TPMAX;   // S0 | S1 | O (hi | lo)
+
+    static_assert(2 * 4 * NC_MAX * 4 <= (int)UNION_BYTES, "reduction scratch");
+    static_assert(SMEM_BYTES <= 232448, "shared memory budget");
+    static_assert((OFF_P | OFF_K | OFF_V) % 1024 == 0, "1024-byte aligned operand tiles");
+};
+
+struct UnitInfo {
+    int b, P, P_raw, n_pref, n_tiles;
+};
+
+PPD_DEV UnitInfo unit_info(const AttnParams &p, int u)
+{
+    UnitInfo ui;
+    ui.b = (u / p.H) % p.B;
+    ui.P_raw = __ldg(p.prefix_len + ui.b);
+    ui.P = min(max(ui.P_raw, 0), p.S_max);
+    ui.n_pref = (ui.P + 127) >> 7;
+    ui.n_tiles = ui.n_pref + 1;
+    return ui;
+}
+
+PPD_DEV void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
+{
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+                 "r"(d)
+                 : "memory");
+}
+
+// Time-bounded wait that ignores the abort flag (used only to drain copies
+// still in flight after an abort, before the CTA exits).
+PPD_DEV void mbar_wait_drain(uint64_t *bar, uint32_t parity)
+{
+    const uint32_t a = smem_addr(bar);
+    const uint64_t t0 = global_timer();
+    while (!mbar_try_wait(a, parity))
+        if (global_timer() - t0 > kWaitLimitNs) return;
+}
+
+template <int D, int TPMAX>
+__global__ void __launch_bounds__(320, 1)
+tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
+                      const __grid_constant__ CUtensorMap map_kc,
+                      const __grid_constant__ CUtensorMap map_vc,
+                      const __grid_constant__ CUtensorMap map_kt,
+                      const __grid_constant__ CUtensorMap map_vt, const AttnParams p)
+{
+    using Lay = AttnLayout<D, TPMAX>;
+    extern __shared__ __align__(1024) uint8_t smem[];
+    // The swizzled operand tiles need a 1024-byte aligned base; the check is
+    // uniform over the CTA, before any barrier.
+    if (smem_addr(smem) & 1023u) {
+        if (threadIdx.x == 0 && p.dev_status)
+            for (int b = 0; b < p.B; ++b) p.dev_status[b] = kErrUnsupported;
+        return;
+    }
+
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + Lay::OFF_BAR);
+    uint32_t *tmem_ptr = reinterpret_cast<uint32_t *>(smem + Lay::OFF_TMEMPTR);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + Lay::OFF_ABORT);
+    float *m2 = reinterpret_cast<float *>(smem + Lay::OFF_M2);
+    uint32_t *anc = reinterpret_cast<uint32_t *>(smem + Lay::OFF_UNION);   // [128][4]
+    float *red = reinterpret_cast<float *>(smem + Lay::OFF_UNION);         // [2][4][NC_MAX]
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int T = p.T;
+    const int T_pad = p.T_pad;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < Lay::NBAR; ++i) {
+            uint32_t count = 1;
+            if (i == Lay::B_SFREE || i == Lay::B_SFREE + 1 || i == Lay::B_PFULL) count = 8;
+            mbar_init(bars + i, count);
+        }
+        *abort_flag = 0;
+        mbar_fence_init();
+    }
+    for (int i = threadIdx.x; i < TPMAX; i += blockDim.x) m2[i] = -INFINITY;
+    if (warp == 9) {
+        tmem_alloc(tmem_ptr, Lay::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_ptr;
+
+    if (warp == 8) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            tma_prefetch_map(&map_q);
+            tma_prefetch_map(&map_kc);
+            tma_prefetch_map(&map_vc);
+            tma_prefetch_map(&map_kt);
+            tma_prefetch_map(&map_vt);
+            const uint64_t pol = l2_policy_evict_first();
+            const uint32_t q_tx = (uint32_t)T_pad * 128u * Lay::DCH;
+            int g = 0, k = 0;
+            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
+                const UnitInfo ui = unit_info(p, u);
+                const int qs = k % Lay::QS;
+                if (k >= Lay::QS)
+                    mbar_wait(bars + Lay::B_QEMPTY + qs, ((k / Lay::QS) - 1) & 1, abort_flag);
+                if (!*abort_flag) {
+                    mbar_arrive_expect_tx(bars + Lay::B_QFULL + qs, q_tx);
+#pragma unroll
+                    for (int c = 0; c < Lay::DCH; ++c)
+                        tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::Q_GROUP_BYTES,
+                                    &map_q, bars + Lay::B_QFULL + qs, c * 64, 0, u, pol);
+                }
+                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                    const bool tree = (j == ui.n_pref);
+                    const int row = tree ? 0 : j * Lay::KT;
+                    const int ks = g % Lay::KS;
+                    if (g >= Lay::KS)
+                        mbar_wait(bars + Lay::B_KEMPTY + ks, ((g / Lay::KS) - 1) & 1, abort_flag);
+                    if (!*abort_flag) {
+                        mbar_arrive_expect_tx(bars + Lay::B_KFULL + ks, Lay::TILE_BYTES);
+#pragma unroll
+                        for (int c = 0; c < Lay::DCH; ++c)
+                            tma_load_3d(smem + Lay::OFF_K + ks * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                        tree ? &map_kt : &map_kc, bars + Lay::B_KFULL + ks, c * 64,
+                                        row, u, pol);
+                    }
+                    const int vs = g % Lay::VS;
+                    if (g >= Lay::VS)
+                        mbar_wait(bars + Lay::B_VEMPTY + vs, ((g / Lay::VS) - 1) & 1, abort_flag);
+                    if (!*abort_flag) {
+                        mbar_arrive_expect_tx(bars + Lay::B_VFULL + vs, Lay::TILE_BYTES);
+#pragma unroll
+                        for (int c = 0; c < Lay::DCH; ++c)
+                            tma_load_3d(smem + Lay::OFF_V + vs * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                        tree ? &map_vt : &map_vc, bars + Lay::B_VFULL + vs, c * 64,
+                                        row, u, pol);
+                    }
+                }
+            }
+            if (*abort_flag) {
+                // let every copy already issued land before the CTA can exit
+                for (int i = max(0, g - Lay::KS); i < g; ++i)
+                    mbar_wait_drain(bars + Lay::B_KFULL + i % Lay::KS, (i / Lay::KS) & 1);
+                for (int i = max(0, g - Lay::VS); i < g; ++i)
+                    mbar_wait_drain(bars + Lay::B_VFULL + i % Lay::VS, (i / Lay::VS) & 1);
+                for (int i = max(0, k - Lay::QS); i < k; ++i)
+                    mbar_wait_drain(bars + Lay::B_QFULL + i % Lay::QS, (i / Lay::QS) & 1);
+            }
+        }
+    } else if (warp == 9) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc_qk = make_idesc_bf16(128, T_pad, 0, 0);
+            const uint32_t idesc_pv = make_idesc_bf16(128, 2 * T_pad, 1, 1);
+            const uint32_t sq = smem_addr(smem + Lay::OFF_Q);
+            const uint32_t sk = smem_addr(smem + Lay::OFF_K);
+            const uint32_t sv = smem_addr(smem + Lay::OFF_V);
+            const uint32_t sp = smem_addr(smem + Lay::OFF_P);
+            const uint32_t t_o = tmem_base + 2 * TPMAX;
+            // V^T as the A operand: M = D spans the tile's 64-column groups.  With
+            // D = 64 both M halves read the same group (rows 64..127 of O^T repeat
+            // rows 0..63 and are ignored).
+            const uint32_t v_lbo = (D == 128) ? Lay::GROUP_BYTES : 0u;
+
+            auto issue_pv = [&](int gp, bool first) {
+                mbar_wait(bars + Lay::B_PFULL, gp & 1, abort_flag);
+                const int vs = gp % Lay::VS;
+                mbar_wait(bars + Lay::B_VFULL + vs, (gp / Lay::VS) & 1, abort_flag);
+                tc_fence_after();
+                if (!*abort_flag) {
+#pragma unroll
+                    for (int kk = 0; kk < Lay::KT / 16; ++kk) {
+                        const uint64_t a = make_smem_desc(sv + vs * Lay::TILE_BYTES + kk * 2048,
+                                                          v_lbo, 1024);
+                        const uint64_t b = make_smem_desc(sp + kk * 2048, Lay::GROUP_BYTES, 1024);
+                        umma_bf16(t_o, a, b, idesc_pv, (first && kk == 0) ? 0u : 1u);
+                    }
+                }
+                umma_commit(bars + Lay::B_PFREE);
+                umma_commit(bars + Lay::B_VEMPTY + vs);
+            };
+
+            int g = 0, k = 0;
+            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
+                const UnitInfo ui = unit_info(p, u);
+                const int qs = k % Lay::QS;
+                mbar_wait(bars + Lay::B_QFULL + qs, (k / Lay::QS) & 1, abort_flag);
+                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                    const int ks = g % Lay::KS;
+                    const int sb = g & 1;
+                    mbar_wait(bars + Lay::B_KFULL + ks, (g / Lay::KS) & 1, abort_flag);
+                    if (g >= 2) mbar_wait(bars + Lay::B_SFREE + sb, ((g >> 1) - 1) & 1, abort_flag);
+                    tc_fence_after();
+                    if (!*abort_flag) {
+#pragma unroll
+                        for (int kk = 0; kk < D / 16; ++kk) {
+                            const uint32_t koff = (kk >> 2) * Lay::GROUP_BYTES + (kk & 3) * 32;
+                            const uint32_t qoff = (kk >> 2) * Lay::Q_GROUP_BYTES + (kk & 3) * 32;
+                            const uint64_t a = make_smem_desc(sk + ks * Lay::TILE_BYTES + koff, 16, 1024);
+                            const uint64_t b = make_smem_desc(sq + qs * Lay::Q_BYTES + qoff, 16, 1024);
+                            umma_bf16(tmem_base + sb * TPMAX, a, b, idesc_qk, kk > 0 ? 1u : 0u);
+                        }
+                    }
+                    umma_commit(bars + Lay::B_SFULL + sb);
+                    umma_commit(bars + Lay::B_KEMPTY + ks);
+                    if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
+                    if (j >= 1) issue_pv(g - 1, j == 1);
+                }
+                issue_pv(g - 1, ui.n_tiles == 1);
+            }
+            // all MMAs finished before TMEM can be released
+            umma_commit(bars + Lay::B_DRAIN);
+            mbar_wait_drain(bars + Lay::B_DRAIN, 0);
+        }
+    } else {
+        // ------------------------------------------------------------ softmax warpgroups
+        const int wg = warp >> 2;
+        const int wq = warp & 3;
+        const int t = wq * 32 + lane;           // key row of S^T, and d of O^T
+        const int NC = T_pad >> 1;              // query columns owned by this warpgroup
+        const int q0 = wg * NC;
+        const int nch = NC >> 4;
+        const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
+        const uint32_t t_o = tmem_base + lane_off + 2 * TPMAX;
+        const uint32_t sp = smem_addr(smem + Lay::OFF_P);
+        const float sl2 = p.scale_log2;
+        float *red_wg = red + wg * 4 * Lay::NC_MAX;
+
+        float lacc[Lay::NC_MAX];
+#pragma unroll
+        for (int c = 0; c < Lay::NC_MAX; ++c) lacc[c] = 0.f;
+        uint64_t dbits = 0;   // bit c: key t (tree node t) is visible to query q0 + c
+        int cur_b = -1;
+        int g = 0;
+
+        for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
+            const UnitInfo ui = unit_info(p, u);
+            if (ui.b != cur_b) {
+                // ancestor bitsets of this sequence's tree, one node per thread
+                named_bar_sync(3, 256);
+                const int i = wg * 128 + t;
+                if (i < T) {
+                    uint32_t w[4] = {0u, 0u, 0u, 0u};
+                    bool bad = false;
+                    int a = i;
+                    while (true) {
+                        w[a >> 5] |= 1u << (a & 31);
+                        const int pa = __ldg(p.parent + (size_t)ui.b * T + a);
+                        if (a == 0) {
+                            bad = (pa != -1);
+                            break;
+                        }
+                        if (pa < 0 || pa >= a) {
+                            bad = true;
+                            break;
+                        }
+                        a = pa;
+                    }
+#pragma unroll
+                    for (int x = 0; x < 4; ++x) anc[i * 4 + x] = w[x];
+                    if (bad && p.dev_status) p.dev_status[ui.b] = kErrTree;
+                }
+                if (i == 0 && p.dev_status && (ui.P_raw < 0 || ui.P_raw > p.S_max))
+                    p.dev_status[ui.b] = kErrCapacity;
+                named_bar_sync(3, 256);
+                dbits = 0;
+                for (int c = 0; c < NC; ++c) {
+                    const int q = q0 + c;
+                    if (q < T && ((anc[q * 4 + (t >> 5)] >> (t & 31)) & 1u)) dbits |= 1ull << c;
+                }
+                named_bar_sync(3, 256);
+                cur_b = ui.b;
+            }
+
+            for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                const bool tree = (j == ui.n_pref);
+                const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
+                const bool row_ok = t < n_valid;
+                const int sb = g & 1;
+                mbar_wait(bars + Lay::B_SFULL + sb, (g >> 1) & 1, abort_flag);
+                tc_fence_after();
+                const uint32_t t_s = tmem_base + lane_off + sb * TPMAX + q0;
+
+                // pass A: does any score exceed the running max by more than 2^8?
+                bool flag = false;
+#pragma unroll
+                for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                    if (ch < nch) {
+                        uint32_t r[16];
+                        tmem_ld16(t_s + ch * 16, r);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const int c = ch * 16 + e;
+                            const bool vis = tree ? ((dbits >> c) & 1ull) != 0 : row_ok;
+                            const float x = __uint_as_float(r[e]) * sl2;
+                            flag |= vis && (x > m2[q0 + c] + 8.f);
+                        }
+                    }
+                }
+                const bool any = named_bar_or(1 + wg, 128, flag);
+                if (any) {
+                    // exact tile maximum per query column, across the 128 key rows
+#pragma unroll
+                    for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                        if (ch < nch) {
+                            uint32_t r[16];
+                            float v[16];
+                            tmem_ld16(t_s + ch * 16, r);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                const int c = ch * 16 + e;
+                                const bool vis = tree ? ((dbits >> c) & 1ull) != 0 : row_ok;
+                                v[e] = vis ? __uint_as_float(r[e]) * sl2 : -INFINITY;
+                            }
+                            const float mx = warp_transpose_reduce16(v, lane, OpMax());
+                            if (!(lane & 1)) red_wg[wq * Lay::NC_MAX + ch * 16 + (lane >> 1)] = mx;
+                        }
+                    }
+                    named_bar_sync(1 + wg, 128);
+                    if (t < NC) {
+                        const float tm = fmaxf(fmaxf(red_wg[t], red_wg[Lay::NC_MAX + t]),
+                                               fmaxf(red_wg[2 * Lay::NC_MAX + t], red_wg[3 * Lay::NC_MAX + t]));
+                        const float old = m2[q0 + t];
+                        const float nw = fmaxf(old, tm);
+                        m2[q0 + t] = nw;
+                        red_wg[t] = (nw == old) ? 1.f : ex2(old - nw);   // alpha
+                    }
+                    named_bar_sync(1 + wg, 128);
+                }
+
+                // the previous tile's PV product must be done before P or O change
+                if (g > 0) mbar_wait(bars + Lay::B_PFREE, (g - 1) & 1, abort_flag);
+                tc_fence_after();
+                if (any && j > 0) {
+#pragma unroll
+                    for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                        if (ch < nch) {
+                            uint32_t rh[16], rl[16];
+                            tmem_ld16(t_o + q0 + ch * 16, rh);
+                            tmem_ld16(t_o + T_pad + q0 + ch * 16, rl);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                const float a = red_wg[ch * 16 + e];
+                                rh[e] = __float_as_uint(__uint_as_float(rh[e]) * a);
+                                rl[e] = __float_as_uint(__uint_as_float(rl[e]) * a);
+                                lacc[ch * 16 + e] *= a;
+                            }
+                            tmem_st16(t_o + q0 + ch * 16, rh);
+                            tmem_st16(t_o + T_pad + q0 + ch * 16, rl);
+                        }
+                    }
+                    tmem_wait_st();
+                }
+
+                // V rows of invisible keys in a partial prefix tile may be NaN: zero them
+                if (!tree && n_valid < Lay::KT && wg == 0) {
+                    const int vs = g % Lay::VS;
+                    mbar_wait(bars + Lay::B_VFULL + vs, (g / Lay::VS) & 1, abort_flag);
+                    if (!row_ok) {
+                        const uint32_t vrow = smem_addr(smem + Lay::OFF_V + vs * Lay::TILE_BYTES) + t * 128u;
+#pragma unroll
+                        for (int c = 0; c < Lay::DCH; ++c)
+#pragma unroll
+                            for (int x = 0; x < 8; ++x)
+                                st_shared_v4(vrow + c * Lay::GROUP_BYTES + x * 16, 0u, 0u, 0u, 0u);
+                    }
+                }
+
+                // pass B: probabilities, row sums, bf16 hi/lo split into shared memory
+#pragma unroll
+                for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                    if (ch < nch) {
+                        uint32_t r[16];
+                        tmem_ld16(t_s + ch * 16, r);
+                        tmem_wait_ld();
+                        uint32_t hw[8], lw[8];
+#pragma unroll
+                        for (int e = 0; e < 16; e += 2) {
+                            float pr[2];
+#pragma unroll
+                            for (int x = 0; x < 2; ++x) {
+                                const int c = ch * 16 + e + x;
+                                const bool vis = tree ? ((dbits >> c) & 1ull) != 0 : row_ok;
+                                const float xs = __uint_as_float(r[e + x]) * sl2 - m2[q0 + c];
+                                pr[x] = vis ? ex2(xs) : 0.f;
+                                lacc[c] += pr[x];
+                            }
+                            const uint32_t h0 = __float_as_uint(pr[0]) & 0xFFFF0000u;
+                            const uint32_t h1 = __float_as_uint(pr[1]) & 0xFFFF0000u;
+                            hw[e >> 1] = __byte_perm(h0, h1, 0x7632);
+                            const __nv_bfloat162 lo = __floats2bfloat162_rn(
+                                pr[0] - __uint_as_float(h0), pr[1] - __uint_as_float(h1));
+                            lw[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
+                        }
+#pragma unroll
+                        for (int half = 0; half < 2; ++half) {
+                            const int cc = q0 + ch * 16 + half * 8;
+                            st_shared_v4(sp + sw128_offset(t, cc, Lay::GROUP_BYTES), hw[half * 4],
+                                         hw[half * 4 + 1], hw[half * 4 + 2], hw[half * 4 + 3]);
+                            st_shared_v4(sp + sw128_offset(t, T_pad + cc, Lay::GROUP_BYTES),
+                                         lw[half * 4], lw[half * 4 + 1], lw[half * 4 + 2],
+                                         lw[half * 4 + 3]);
+                        }
+                    }
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(bars + Lay::B_PFULL);
+                    mbar_arrive(bars + Lay::B_SFREE + sb);
+                }
+
+                if (j == ui.n_tiles - 1) {
+                    // -------------------------------------------------- unit epilogue
+                    mbar_wait(bars + Lay::B_PFREE, g & 1, abort_flag);
+                    tc_fence_after();
+                    named_bar_sync(1 + wg, 128);   // every thread is done reading alpha
+#pragma unroll
+                    for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                        if (ch < nch) {
+                            float v[16];
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) v[e] = lacc[ch * 16 + e];
+                            const float s = warp_transpose_reduce16(v, lane, OpAdd());
+                            if (!(lane & 1)) red_wg[wq * Lay::NC_MAX + ch * 16 + (lane >> 1)] = s;
+                        }
+                    }
+                    named_bar_sync(1 + wg, 128);
+                    if (t < NC) {
+                        const float l = red_wg[t] + red_wg[Lay::NC_MAX + t] +
+                                        red_wg[2 * Lay::NC_MAX + t] + red_wg[3 * Lay::NC_MAX + t];
+                        const int q = q0 + t;
+                        if (p.lse && q < T)
+                            p.lse[(size_t)u * T + q] = (m2[q] + lg2(l)) * 0.69314718055994530942f;
+                        red_wg[t] = 1.f / l;
+                        m2[q] = -INFINITY;
+                    }
+                    named_bar_sync(1 + wg, 128);
+                    if (wq * 32 < D) {
+                        float *orow = p.out + (size_t)u * T * D + t;
+#pragma unroll
+                        for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                            if (ch < nch) {
+                                uint32_t rh[16], rl[16];
+                                tmem_ld16(t_o + q0 + ch * 16, rh);
+                                tmem_ld16(t_o + T_pad + q0 + ch * 16, rl);
+                                tmem_wait_ld();
+#pragma unroll
+                                for (int e = 0; e < 16; ++e) {
+                                    const int q = q0 + ch * 16 + e;
+                                    if (q < T)
+                                        orow[(size_t)q * D] = (__uint_as_float(rh[e]) + __uint_as_float(rl[e])) *
+                                                              red_wg[ch * 16 + e];
+                                }
+                            }
+                        }
+                    }
+                    tc_fence_before();
+#pragma unroll
+                    for (int c = 0; c < Lay::NC_MAX; ++c) lacc[c] = 0.f;
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (*abort_flag && threadIdx.x == 0 && p.dev_status)
+        for (int b = 0; b < p.B; ++b) p.dev_status[b] = kErrTimeout;
+    if (warp == 9) tmem_dealloc(tmem_base, Lay::TMEM_COLS);
+}
+
+template <int D, int TPMAX>
+static cudaError_t launch_tree_attention_t(const AttnMaps &m, const AttnParams &p, int num_sms,
+                                           cudaStream_t stream)
+{
+    using Lay = AttnLayout<D, TPMAX>;
+    auto kern = tree_attention_kernel<D, TPMAX>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)Lay::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    const int grid = p.n_units < num_sms ? p.n_units : num_sms;
+    kern<<<grid, 320, Lay::SMEM_BYTES, stream>>>(m.q, m.kc, m.vc, m.kt, m.vt, p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
+                                  cudaStream_t stream)
+{
+    if (D == 128) {
+        if (p.T_pad <= 64) return launch_tree_attention_t<128, 64>(m, p, num_sms, stream);
+        return launch_tree_attention_t<128, 128>(m, p, num_sms, stream);
+    }
+    if (p.T_pad <= 64) return launch_tree_attention_t<64, 64>(m, p, num_sms, stream);
+    return launch_tree_attention_t<64, 128>(m, p, num_sms, stream);
+}
+
+}  // namespace ppd

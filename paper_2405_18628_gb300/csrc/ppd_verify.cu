@@ -1,0 +1,438 @@
+// ppd_verify.cu -- node argmax, exact-matching acceptance, KV compaction,
+// fp32 -> bf16 rounding, and the tensor-core layout self-test.
+//
+// Node argmax (paper Section 3 step (2): exact matching compares every guess
+// token with the model's top-1 token at its parent) streams the fp32 logits
+// with 16-byte loads, reduces (value, index) pairs with warp shuffles, and
+// splits long rows over several blocks whose partial results are combined by
+// the last block to finish.  Acceptance (Section 3 steps (2)-(3)) runs one
+// warp per sequence: ballots build the bitset of matching nodes, each lane
+// walks its nodes' root paths, and a warp max-reduction picks the deepest
+// accepted node.  Compaction (Section 3 step (3)) copies the accepted rows
+// into the cache with 16-byte loads and stores.
+#include "ppd_device.cuh"
+#include "ppd_kernels.h"
+
+#include <climits>
+#include <cmath>
+
+namespace ppd {
+
+// ------------------------------------------------------------------ argmax
+
+// true when (av, ai) ranks before (bv, bi): NaN first (lowest index among
+// NaNs), then larger value, then lower index.  -0 == +0 compare equal.
+PPD_DEV bool ranks_before(float av, int ai, float bv, int bi)
+{
+    const bool an = av != av, bn = bv != bv;
+    if (an || bn) return an && bn ? ai < bi : an;
+    if (av != bv) return av > bv;
+    return ai < bi;
+}
+
+PPD_DEV void consider(float v, int i, float &bv, int &bi)
+{
+    if (ranks_before(v, i, bv, bi)) {
+        bv = v;
+        bi = i;
+    }
+}
+
+PPD_DEV int32_t ld_cg(const int32_t *p) { return __ldcg(p); }
+
+// One warp decides acceptance for sequence b; argmax values are read through
+// L2 because other blocks of the same grid may have written them.
+PPD_DEV void accept_sequence(int b, const int32_t *argmax_all, const AcceptArgs &a, int lane,
+                             int *s_par)
+{
+    const int T = a.T;
+    const int32_t *par = a.parent + (size_t)b * T;
+    const int32_t *tok = a.cand_tokens + (size_t)b * T;
+    const int32_t *top = argmax_all + (size_t)b * T;
+    bool bad = false;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = lane + 32 * k;
+        if (i < T) {
+            const int pa = __ldg(par + i);
+            const int tk = __ldg(tok + i);
+            s_par[i] = pa;
+            if (i == 0)
+                bad |= (pa != -1) || tk < 0 || tk >= a.V;
+            else
+                bad |= pa < 0 || pa >= i || tk < -1 || tk >= a.V;
+        }
+    }
+    __syncwarp();
+    bad = __any_sync(0xffffffffu, bad);
+    const int P = __ldg(a.prefix_len + b);
+    int err = bad ? kErrTree : ((P < 0 || P > a.S_max) ? kErrCapacity : kOk);
+
+    uint32_t okw[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = lane + 32 * k;
+        bool ok = false;
+        if (i < T && err == kOk) {
+            if (i == 0) {
+                ok = true;
+            } else {
+                const int tk = __ldg(tok + i);
+                ok = tk >= 0 && tk == ld_cg(top + s_par[i]);
+            }
+        }
+        okw[k] = __ballot_sync(0xffffffffu, ok);
+    }
+
+    int best_key = -1;   // (depth << 8) | (255 - node): deepest, then smallest index
+    if (err == kOk) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int i = lane + 32 * k;
+            if (i < T) {
+                int n = i, depth = 0;
+                bool good = true;
+                while (n > 0) {
+                    const uint32_t w = (n < 32) ? okw[0] : (n < 64) ? okw[1] : (n < 96) ? okw[2] : okw[3];
+                    good &= ((w >> (n & 31)) & 1u) != 0;
+                    n = s_par[n];
+                    ++depth;
+                }
+                if (good) best_key = max(best_key, (depth << 8) | (255 - i));
+            }
+        }
+    }
+    best_key = __reduce_max_sync(0xffffffffu, best_key);
+    const int best = 255 - (best_key & 255);
+    const int n_acc = (best_key >> 8) + 1;
+    if (err == kOk && (long long)P + n_acc > a.S_max) err = kErrCapacity;
+    const int n_out = (err == kOk) ? n_acc : 0;
+
+    int32_t *pth = a.path + (size_t)b * T;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = lane + 32 * k;
+        if (i < T && i >= n_out) pth[i] = -1;
+    }
+    if (lane == 0) {
+        if (err == kOk) {
+            int n = best;
+            for (int j = n_acc - 1; j >= 0; --j) {
+                pth[j] = n;
+                n = s_par[n];
+            }
+        }
+        a.accept_len[b] = n_out;
+        a.next_token[b] = (err == kOk) ? ld_cg(top + best) : -1;
+        a.new_prefix_len[b] = (err == kOk) ? P + n_acc : P;
+        a.dev_status[b] = err;
+    }
+}
+
+template <bool kVec>
+__global__ void __launch_bounds__(256)
+node_argmax_kernel(const float *__restrict__ logits, int64_t rows, int V, int splits, int chunk,
+                   int32_t *argmax_out, ArgmaxScratch ws, AcceptArgs acc, int has_acc)
+{
+    __shared__ float s_v[8];
+    __shared__ int s_i[8];
+    __shared__ int s_flag;
+    __shared__ int s_par[128];
+    const int64_t row = blockIdx.x / splits;
+    const int s = blockIdx.x % splits;
+    const int lo = s * chunk;
+    const int hi = min(V, lo + chunk);
+    const float *x = logits + row * (int64_t)V;
+    float bv = -INFINITY;
+    int bi = INT_MAX;
+    if (kVec) {
+        const float4 *x4 = reinterpret_cast<const float4 *>(x);
+        const int n4_lo = lo >> 2, n4_hi = hi >> 2;
+        int i = n4_lo + threadIdx.x;
+        for (; i + 3 * 256 < n4_hi; i += 4 * 256) {
+            float4 f[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) f[k] = __ldcs(x4 + i + k * 256);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int base = 4 * (i + k * 256);
+                consider(f[k].x, base, bv, bi);
+                consider(f[k].y, base + 1, bv, bi);
+                consider(f[k].z, base + 2, bv, bi);
+                consider(f[k].w, base + 3, bv, bi);
+            }
+        }
+        for (; i < n4_hi; i += 256) {
+            const float4 f = __ldcs(x4 + i);
+            consider(f.x, 4 * i, bv, bi);
+            consider(f.y, 4 * i + 1, bv, bi);
+            consider(f.z, 4 * i + 2, bv, bi);
+            consider(f.w, 4 * i + 3, bv, bi);
+        }
+    } else {
+        for (int i = lo + threadIdx.x; i < hi; i += 256) consider(__ldcs(x + i), i, bv, bi);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float ov = __shfl_down_sync(0xffffffffu, bv, off);
+        const int oi = __shfl_down_sync(0xffffffffu, bi, off);
+        consider(ov, oi, bv, bi);
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        s_v[warp] = bv;
+        s_i[warp] = bi;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < 8; ++w) consider(s_v[w], s_i[w], bv, bi);
+        int done = 0;
+        if (splits == 1) {
+            argmax_out[row] = bi;
+            done = 1;
+        } else {
+            ws.part_val[row * splits + s] = bv;
+            ws.part_idx[row * splits + s] = bi;
+            __threadfence();
+            const int prev = atomicAdd(ws.row_count + row, 1);
+            if (prev == splits - 1) {
+                __threadfence();
+                float cv = __ldcg(ws.part_val + row * splits);
+                int ci = __ldcg(ws.part_idx + row * splits);
+                for (int k = 1; k < splits; ++k)
+                    consider(__ldcg(ws.part_val + row * splits + k), __ldcg(ws.part_idx + row * splits + k),
+                             cv, ci);
+                argmax_out[row] = ci;
+                ws.row_count[row] = 0;
+                done = 1;
+            }
+        }
+        int last_of_seq = 0;
+        if (done && has_acc) {
+            __threadfence();
+            const int b = (int)(row / acc.T);
+            const int prev = atomicAdd(ws.seq_count + b, 1);
+            if (prev == acc.T - 1) {
+                __threadfence();
+                ws.seq_count[b] = 0;
+                last_of_seq = 1;
+            }
+        }
+        s_flag = last_of_seq;
+    }
+    __syncthreads();
+    if (s_flag && warp == 0) accept_sequence((int)(row / acc.T), argmax_out, acc, lane, s_par);
+}
+
+cudaError_t launch_node_argmax(const float *logits, int64_t rows, int V, int splits,
+                               int32_t *argmax_out, const ArgmaxScratch &ws,
+                               const AcceptArgs *acc, int B, cudaStream_t stream)
+{
+    (void)B;
+    const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
+    int chunk = (V + splits - 1) / splits;
+    chunk = (chunk + 3) & ~3;
+    AcceptArgs a{};
+    if (acc) a = *acc;
+    const dim3 grid((unsigned)(rows * splits));
+    if (vec)
+        node_argmax_kernel<true><<<grid, 256, 0, stream>>>(logits, rows, V, splits, chunk, argmax_out,
+                                                          ws, a, acc != nullptr);
+    else
+        node_argmax_kernel<false><<<grid, 256, 0, stream>>>(logits, rows, V, splits, chunk, argmax_out,
+                                                           ws, a, acc != nullptr);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ accept
+
+__global__ void __launch_bounds__(128)
+accept_path_kernel(const int32_t *argmax, AcceptArgs a, int B)
+{
+    __shared__ int s_par[4][128];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.x * 4 + warp;
+    if (b < B) accept_sequence(b, argmax, a, lane, s_par[warp]);
+}
+
+cudaError_t launch_accept_path(const int32_t *argmax, const AcceptArgs &a, int B,
+                               cudaStream_t stream)
+{
+    accept_path_kernel<<<(B + 3) / 4, 128, 0, stream>>>(argmax, a, B);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ compaction
+
+__global__ void __launch_bounds__(128)
+kv_compact_kernel(uint8_t *kc, uint8_t *vc, const uint8_t *__restrict__ kt,
+                  const uint8_t *__restrict__ vt, const int32_t *path, const int32_t *accept_len,
+                  const int32_t *prefix_len, int64_t n_units, int B, int H, int T, int S_max,
+                  int row_bytes)
+{
+    const int chunks = row_bytes >> 4;
+    for (int64_t u = blockIdx.x; u < n_units; u += gridDim.x) {
+        const int b = (int)((u / H) % B);
+        const int n = __ldg(accept_len + b);
+        const int P = __ldg(prefix_len + b);
+        if (n <= 0 || n > T || P < 0 || (long long)P + n > S_max) continue;
+        for (int w = threadIdx.x; w < n * chunks; w += blockDim.x) {
+            const int j = w / chunks, c = w - j * chunks;
+            const int src = __ldg(path + (size_t)b * T + j);
+            if (src < 0 || src >= T) continue;
+            const size_t so = ((size_t)u * T + src) * row_bytes + (size_t)c * 16;
+            const size_t dof = ((size_t)u * S_max + P + j) * row_bytes + (size_t)c * 16;
+            const uint4 kx = __ldg(reinterpret_cast<const uint4 *>(kt + so));
+            const uint4 vx = __ldg(reinterpret_cast<const uint4 *>(vt + so));
+            *reinterpret_cast<uint4 *>(kc + dof) = kx;
+            *reinterpret_cast<uint4 *>(vc + dof) = vx;
+        }
+    }
+}
+
+cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_tree,
+                              const void *v_tree, const int32_t *path,
+                              const int32_t *accept_len, const int32_t *prefix_len, int L,
+                              int B, int H, int T, int D, int S_max, int elem_bytes,
+                              cudaStream_t stream)
+{
+    const int64_t n_units = (int64_t)L * B * H;
+    const int grid = (int)(n_units < 4096 ? n_units : 4096);
+    kv_compact_kernel<<<grid, 128, 0, stream>>>(
+        static_cast<uint8_t *>(k_cache), static_cast<uint8_t *>(v_cache),
+        static_cast<const uint8_t *>(k_tree), static_cast<const uint8_t *>(v_tree), path,
+        accept_len, prefix_len, n_units, B, H, T, S_max, D * elem_bytes);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ fp32 -> bf16
+
+__global__ void round_bf16_kernel(const float *__restrict__ src, uint16_t *__restrict__ dst,
+                                  int64_t n)
+{
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const __nv_bfloat16 h = __float2bfloat16_rn(src[i]);
+        dst[i] = *reinterpret_cast<const uint16_t *>(&h);
+    }
+}
+
+cudaError_t launch_round_bf16(const float *src, uint16_t *dst, int64_t n, cudaStream_t stream)
+{
+    if (n <= 0) return cudaSuccess;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 8192) blocks = 8192;
+    round_bf16_kernel<<<(unsigned)blocks, 256, 0, stream>>>(src, dst, n);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ tensor-core self-test
+
+constexpr uint32_t kSelfTestSmem = 200 * 1024;   // generous: operands use < 96 KB
+
+__global__ void __launch_bounds__(128, 1)
+selftest_umma_kernel(const __grid_constant__ CUtensorMap ma, const __grid_constant__ CUtensorMap mb,
+                     const uint16_t *b_raw, float *d, int mode, int N)
+{
+    extern __shared__ __align__(1024) uint8_t smem[];
+    if (smem_addr(smem) & 1023u) return;
+    uint8_t *sa = smem;                 // 32 KB
+    uint8_t *sb = smem + 32 * 1024;     // up to 64 KB
+    uint64_t *bar = reinterpret_cast<uint64_t *>(smem + 96 * 1024);   // [0] tma, [1] mma
+    uint32_t *tmem_ptr = reinterpret_cast<uint32_t *>(smem + 96 * 1024 + 16);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + 96 * 1024 + 20);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        mbar_init(bar, 1);
+        mbar_init(bar + 1, 1);
+        *abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_ptr, 256);
+        tmem_relinquish();
+    }
+    if (mode != 0) {
+        // b given [128][N], N contiguous: thread t writes row t in the layout the
+        // attention kernel uses for its probability tile.
+        const int t = threadIdx.x;
+        for (int n = 0; n < N; n += 8) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(b_raw + (size_t)t * N + n);
+            const uint32_t addr = smem_addr(sb) + sw128_offset(t, n, 16384);
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x),
+                         "r"(v.y), "r"(v.z), "r"(v.w)
+                         : "memory");
+        }
+        fence_proxy_async_smem();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_ptr;
+
+    if (threadIdx.x == 0) {
+        uint32_t tx = 0;
+        if (mode == 0) tx = 128 * 128 * 2 + (uint32_t)N * 128 * 2;
+        else tx = (mode == 1 ? 2u : 1u) * 16384u;
+        mbar_arrive_expect_tx(bar, tx);
+        if (mode == 0) {
+            tma_load_2d(sa, &ma, bar, 0, 0);
+            tma_load_2d(sa + 16384, &ma, bar, 64, 0);
+            tma_load_2d(sb, &mb, bar, 0, 0);
+            tma_load_2d(sb + (size_t)N * 128, &mb, bar, 64, 0);
+        } else {
+            tma_load_2d(sa, &ma, bar, 0, 0);
+            if (mode == 1) tma_load_2d(sa + 16384, &ma, bar, 64, 0);
+        }
+        mbar_wait(bar, 0, abort_flag);
+        tc_fence_after();
+        if (!*abort_flag) {
+            const uint32_t a0 = smem_addr(sa), b0 = smem_addr(sb);
+            for (int kk = 0; kk < 8; ++kk) {
+                uint64_t da, db;
+                uint32_t idesc;
+                if (mode == 0) {
+                    da = make_smem_desc(a0 + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+                    db = make_smem_desc(b0 + (kk >> 2) * N * 128 + (kk & 3) * 32, 16, 1024);
+                    idesc = make_idesc_bf16(128, N, 0, 0);
+                } else {
+                    da = make_smem_desc(a0 + kk * 2048, mode == 1 ? 16384u : 0u, 1024);
+                    db = make_smem_desc(b0 + kk * 2048, 16384, 1024);
+                    idesc = make_idesc_bf16(128, N, 1, 1);
+                }
+                umma_bf16(tmem, da, db, idesc, kk > 0 ? 1u : 0u);
+            }
+        }
+        umma_commit(bar + 1);
+    }
+    __syncwarp();
+    mbar_wait(bar + 1, 0, abort_flag);
+    tc_fence_after();
+    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+    for (int ch = 0; ch < N / 16; ++ch) {
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_off + ch * 16, r);
+        tmem_wait_ld();
+        for (int e = 0; e < 16; ++e)
+            d[(size_t)(warp * 32 + lane) * N + ch * 16 + e] =
+                *abort_flag ? NAN : __uint_as_float(r[e]);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, 256);
+}
+
+cudaError_t launch_selftest_umma(const CUtensorMap &ma, const CUtensorMap &mb, const void *b_raw,
+                                 float *d, int mode, int N, cudaStream_t stream)
+{
+    cudaError_t e = cudaFuncSetAttribute(selftest_umma_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSelfTestSmem);
+    if (e != cudaSuccess) return e;
+    selftest_umma_kernel<<<1, 128, kSelfTestSmem, stream>>>(
+        ma, mb, static_cast<const uint16_t *>(b_raw), d, mode, N);
+    return cudaGetLastError();
+}
+
+}  // namespace ppd

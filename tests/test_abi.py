@@ -1,0 +1,96 @@
+"""The C-ABI library: it builds, loads, exports every entry point that
+include/ppd.h declares, and rejects bad arguments on the host before any
+device work (no GPU needed: these calls return before touching CUDA)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2405_18628_gb300 import build, ppd
+    build.build()
+    return ppd.load()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "ppd.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ppd_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("ppd_tree_attention", "ppd_node_argmax", "ppd_accept_path", "ppd_kv_compact",
+              "ppd_verify_step", "ppd_workspace_bytes", "ppd_status_string"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in _declared():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    from paper_2405_18628_gb300 import ppd
+    for s in range(7):
+        assert ppd.status_string(s) and ppd.status_string(s) != "unknown status"
+    assert ppd.status_string(99) == "unknown status"
+
+
+def test_workspace_bytes(lib):
+    from paper_2405_18628_gb300 import ppd
+    a = ppd.ppd_workspace_bytes(32, 1, 32, 64, 128, 32000, 2112)
+    assert a > 0 and a % 256 == 0
+    f = ppd.ppd_workspace_bytes(1, 1, 4, 48, 64, 1024, 176, ppd.PPD_F32)
+    assert f >= 2 * (3 * 48 + 2 * 176) * 64 * 4
+    assert ppd.ppd_workspace_bytes(0, 1, 1, 1, 64, 1, 1) == 0
+
+
+def test_host_argument_checks(lib):
+    """Invalid sizes and null pointers are rejected with PPD_ERR_INVALID_ARG
+    (or UNSUPPORTED) without launching anything."""
+    vp = ctypes.c_void_p
+    fake = vp(0x10000)            # never dereferenced: the checks fail first
+    null = None
+    s = vp(0)
+    INVALID = 1
+    # T > 128
+    assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 129, 64, 200,
+                                  0, 0.0, fake, null, fake, null, 0, s) == INVALID
+    # D not in {64, 128}
+    assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 8, 96, 200,
+                                  0, 0.0, fake, null, fake, null, 0, s) == INVALID
+    # null output
+    assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 8, 64, 200,
+                                  0, 0.0, null, null, fake, null, 0, s) == INVALID
+    # misaligned q
+    assert lib.ppd_tree_attention(vp(0x10002), fake, fake, fake, fake, fake, fake, 1, 1, 1, 8, 64,
+                                  200, 0, 0.0, fake, null, fake, null, 0, s) == INVALID
+    # fp32 without workspace
+    assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 8, 64, 200,
+                                  1, 0.0, fake, null, fake, null, 0, s) == INVALID
+    assert lib.ppd_node_argmax(fake, 0, 4, 10, fake, null, 0, s) == INVALID
+    assert lib.ppd_node_argmax(fake, 1, 64, 32000, fake, null, 0, s) == INVALID   # needs workspace
+    assert lib.ppd_accept_path(fake, fake, fake, fake, 1, 200, 10, 10, fake, fake, fake, fake,
+                               fake, s) == INVALID
+    assert lib.ppd_accept_path(fake, fake, null, fake, 1, 4, 10, 10, fake, fake, fake, fake,
+                               fake, s) == INVALID
+    # compaction: tree buffer inside the cache buffer
+    assert lib.ppd_kv_compact(vp(0x100000), vp(0x900000), vp(0x100400), vp(0xA00000), fake, fake,
+                              fake, 1, 1, 1, 4, 64, 100, 0, s) == INVALID
+    # verify step: missing workspace
+    args = [fake] * 9 + [1, 1, 1, 8, 64, 100, 200, 0, 0.0] + [fake] * 8 + [null, 0, s]
+    assert lib.ppd_verify_step(*args) == INVALID
+
+
+def test_binding_requires_library(monkeypatch, tmp_path):
+    from paper_2405_18628_gb300 import ppd
+    monkeypatch.setattr(ppd, "_lib", None)
+    monkeypatch.setattr(ppd, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        ppd.load()
