@@ -1,0 +1,422 @@
+#!/usr/bin/env python3
+"""Benchmark of the PPD verification step (tree attention over every layer,
+node argmax, acceptance, KV compaction) through libppd's C ABI.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl reference]
+
+Prints one JSON line.  The default workload is the Vicuna-7B-shaped cache
+(32 layers, 32 heads x 128, bf16 K/V, batch 1, prefix 2048, 64-token tree,
+vocab 32000).  Inputs are seeded synthetic tensors resident in HBM; L2 is
+flushed (a 256 MiB write) before every timed step, outside the step's events.
+
+Under torchrun (N > 1) each rank runs an independent replica of the workload
+on its own GPU (weak scaling: the sequences of different ranks are
+independent, no data-path collective); the step time is the maximum over
+ranks.  `--impl reference` times the fp64 CPU oracle on the host cores
+instead (rank 0 only), on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verify steps/s and achieved HBM GB/s (frac of ~8 TB/s), Vicuna-7B shapes"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_FLUSH_BYTES = 256 << 20
+
+# DRAM traffic of one tree-attention launch from an ncu capture
+# (dram__bytes_read.sum + dram__bytes_write.sum), keyed by workload, with the
+# hash of the attention source it was taken on: a stale entry reports null.
+MEASURED_TRAFFIC = {}
+
+
+def attention_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("ppd_attention.cu", "ppd_device.cuh"):
+        with open(os.path.join(ROOT, "paper_2405_18628_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peak_gbs():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ----------------------------------------------------------------------------- bytes
+
+def attention_bytes(w) -> int:
+    """Algorithmic bytes of one tree-attention launch over all L*B*H slices:
+    per slice the bf16 K/V prefix (4*P*D), tree K/V (4*T*D), Q (2*T*D) and the
+    fp32 output (4*T*D)."""
+    per_unit = 4 * w.P * w.D + 4 * w.T * w.D + 2 * w.T * w.D + 4 * w.T * w.D
+    return w.L * w.B * w.H * per_unit
+
+
+def step_bytes(w, n_acc_total: int) -> int:
+    """Algorithmic bytes of one verification step: attention, the fp32 logits,
+    the compacted K/V rows (read from the tree, written to the cache) and the
+    small integer arrays."""
+    ints = 4 * w.B * w.T * 4 + 4 * w.B * 6
+    return (attention_bytes(w) + 4 * w.B * w.T * w.V +
+            2 * 4 * w.L * w.H * w.D * n_acc_total + ints)
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            with open(self.path) as f:
+                for line in f:
+                    parts = [p.strip() for p in line.split(",")]
+                    if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                        rows.append(parts)
+        except Exception:
+            pass
+        finally:
+            if self.path and os.path.exists(self.path):
+                os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k].lower() == "active"})
+        return {"sm_mhz": statistics.median(float(r[1]) for r in rows),
+                "sm_max_mhz": max(float(r[2]) for r in rows),
+                "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())
+                if any(r[3].replace(".", "").isdigit() for r in rows) else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+
+def oracle_step_seconds(w, host, s, units, n_threads: int) -> float:
+    """One fp64 oracle verification step on a sample of the workload, scaled to
+    the whole step.  `host` holds the first few layers of Q/K/V on the host;
+    attention runs on `units` of them (None: all), compaction on all of them,
+    argmax and acceptance once, as in a full step.  Attention and compaction
+    times are scaled by the fraction of the workload the sample covers."""
+    import oracle
+    L_h = host["q"].shape[0]
+    n_sample = len(units) if units is not None else L_h * w.B * w.H
+    t0 = time.perf_counter()
+    oracle.tree_attention(host["q"], host["k_cache"], host["v_cache"], host["k_tree"],
+                          host["v_tree"], s.prefix_len, s.parent, units=units,
+                          n_threads=n_threads)
+    t_att = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    am = oracle.node_argmax(s.logits)
+    acc = oracle.accept_path(am, s.cand_tokens, s.parent, s.prefix_len, w.V, w.S_max)
+    t_acc = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    oracle.kv_compact(host["k_cache"], host["v_cache"], host["k_tree"], host["v_tree"],
+                      acc["path"], acc["accept_len"], s.prefix_len)
+    t_cmp = time.perf_counter() - t0
+    return t_att * (w.L * w.B * w.H) / n_sample + t_acc + t_cmp * w.L / L_h
+
+
+def cpu_baseline(w, t_dev, s, budget_s: float):
+    """Oracle on the first `nl` layers, `nl` chosen from a one-layer calibration
+    so the sample takes about `budget_s` seconds of host time."""
+    import oracle
+    n_threads = os.cpu_count() or 1
+    one = {k: v[:1].cpu() for k, v in t_dev.items()}
+    t0 = time.perf_counter()
+    oracle_step_seconds(w, one, s, None, n_threads)
+    t1 = time.perf_counter() - t0
+    nl = max(1, min(w.L, int(budget_s / max(t1, 1e-6))))
+    host = one if nl == 1 else {k: v[:nl].cpu() for k, v in t_dev.items()}
+    sec = oracle_step_seconds(w, host, s, None, n_threads)
+    return {"value": 1.0 / sec, "unit": "steps/s", "cores": n_threads, "kind": "oracle",
+            "sample": f"fp64 oracle verification step on the first {nl} of {w.L} layers "
+                      f"(all heads; attention and compaction time scaled by {w.L}/{nl}; "
+                      f"full argmax and acceptance)"}
+
+
+# ----------------------------------------------------------------------------- main
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--config", default="vicuna7b")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=12.0,
+                    help="seconds of oracle work in the CPU baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_reference(args, w, world, rank):
+    """The CPU oracle as the reference arm.  Each step is a bounded sample: a
+    few attention slices of layer 0 (scaled to all slices), the full argmax and
+    acceptance, and layer 0's compaction (scaled to all layers)."""
+    if rank != 0:
+        return
+    from paper_2405_18628_gb300 import workloads as W
+
+    s = W.make_step_inputs(w)
+    n_threads = os.cpu_count() or 1
+    host = W.make_tensors(W.scaled(w, L=1), device="cpu")
+    n_all = w.B * w.H
+    cal = list(range(min(n_threads, n_all)))
+    t0 = time.perf_counter()
+    oracle_step_seconds(w, host, s, cal, n_threads)
+    t_cal = time.perf_counter() - t0
+    per_step_budget = max(0.01, 150.0 / max(1, args.steps + args.warmup))
+    n_units = int(max(1, min(n_all, len(cal) * per_step_budget / max(t_cal, 1e-9))))
+    units = list(range(n_units))
+    for _ in range(args.warmup):
+        oracle_step_seconds(w, host, s, units, n_threads)
+    secs = [oracle_step_seconds(w, host, s, units, n_threads) for _ in range(args.steps)]
+    sec_per_step = statistics.mean(secs)
+    value = 1.0 / sec_per_step
+    sample = (f"{n_units} of {w.L * w.B * w.H} attention slices (layer 0) per step, scaled to all "
+              f"slices; full argmax and acceptance; layer-0 compaction scaled to {w.L} layers")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": sec_per_step * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name},
+        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": n_threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_setup()
+    from paper_2405_18628_gb300 import workloads as W
+    w = W.WORKLOADS[args.config]
+    if args.impl == "reference":
+        run_reference(args, w, world, rank)
+        return
+
+    import torch
+    from paper_2405_18628_gb300 import ppd
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    ppd.load()
+
+    # ---------------------------------------------------------------- inputs (resident in HBM)
+    s = W.make_step_inputs(w, seed=w.seed + 1000 * rank)
+    t = W.make_tensors(w, device=dev, seed=w.seed + 1000 * rank)
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
+    parent, cand, prefix = i32(s.parent), i32(s.cand_tokens), i32(s.prefix_len)
+    logits = torch.from_numpy(s.logits).to(dev)
+    bufs = ppd.StepBuffers(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
+                            parent, cand, logits, bufs.out, bufs.argmax, bufs.accept_len, bufs.path,
+                            bufs.next_token, bufs.new_prefix_len, bufs.dev_status, bufs.workspace,
+                            stream=stream)
+
+    for _ in range(max(3, args.warmup)):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    status = bufs.dev_status.cpu().numpy()
+    n_acc = int(bufs.accept_len.sum().item())
+    if (status != 0).any() or n_acc < w.B:
+        raise SystemExit(f"verification step reported device status {status.tolist()}")
+
+    # ---------------------------------------------------------------- timed region
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    with ClockSampler(local) as clocks:
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+        wall0 = time.perf_counter()
+        for k in range(K):
+            flush.zero_()
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+        if pg:
+            pg.barrier()
+        wall = time.perf_counter() - wall0
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(step_ms)
+    if pg:
+        tt = torch.tensor([total_ms], device=dev)
+        pg.all_reduce(tt, op=pg.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / K
+    value = world * K / (total_ms / 1e3)
+    clk = clocks.summary()
+
+    # ---------------------------------------------------------------- dominant kernel alone
+    K2 = min(K, 300)
+    ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(K2)]
+    st_att = torch.empty(w.B, dtype=torch.int32, device=dev)
+    for k in range(K2 + 3):
+        flush.zero_()
+        if k >= 3:
+            ev2[k - 3][0].record(stream)
+        ppd.ppd_tree_attention(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
+                               parent, bufs.out, st_att, stream=stream)
+        if k >= 3:
+            ev2[k - 3][1].record(stream)
+    torch.cuda.synchronize()
+    att_ms = statistics.mean(a.elapsed_time(b) for a, b in ev2)
+    att_bytes = attention_bytes(w)
+    peak, peak_kind = measured_peak_gbs()
+    achieved = att_bytes / (att_ms * 1e-3) / 1e9
+    tr = MEASURED_TRAFFIC.get(w.name)
+    traffic = tr["bytes_per_launch"] if tr and tr.get("src") == attention_source_hash() else None
+
+    # ---------------------------------------------------------------- end to end, host buffers
+    e2e = None
+    if not args.no_e2e:
+        K3 = min(K, 200)
+        pin = lambda x: x.cpu().pin_memory()
+        h_in = {"q": pin(t["q"]), "k_tree": pin(t["k_tree"]), "v_tree": pin(t["v_tree"]),
+                "logits": pin(logits), "parent": pin(parent), "cand": pin(cand), "prefix": pin(prefix)}
+        d_in = {k: torch.empty_like(v, device=dev) for k, v in h_in.items()}
+        outs = ["out", "argmax", "accept_len", "path", "next_token", "new_prefix_len", "dev_status"]
+        h_out = {k: torch.empty_like(getattr(bufs, k), device="cpu").pin_memory() for k in outs}
+        h2d = sum(v.numel() * v.element_size() for v in h_in.values())
+        d2h = sum(v.numel() * v.element_size() for v in h_out.values())
+
+        def e2e_step():
+            for k, v in h_in.items():
+                d_in[k].copy_(v, non_blocking=True)
+            ppd.ppd_verify_step(d_in["q"], t["k_cache"], t["v_cache"], d_in["k_tree"],
+                                d_in["v_tree"], d_in["prefix"], d_in["parent"], d_in["cand"],
+                                d_in["logits"], bufs.out, bufs.argmax, bufs.accept_len, bufs.path,
+                                bufs.next_token, bufs.new_prefix_len, bufs.dev_status,
+                                bufs.workspace, stream=stream)
+            for k in outs:
+                h_out[k].copy_(getattr(bufs, k), non_blocking=True)
+            stream.synchronize()
+
+        for _ in range(3):
+            flush.zero_()
+            e2e_step()
+        e_ms = []
+        for _ in range(K3):
+            flush.zero_()
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            e2e_step()
+            e_ms.append((time.perf_counter() - t0) * 1e3)
+        e_total = sum(e_ms)
+        if pg:
+            tt = torch.tensor([e_total], device=dev)
+            pg.all_reduce(tt, op=pg.ReduceOp.MAX)
+            e_total = float(tt.item())
+        e2e = {"value": world * K3 / (e_total / 1e3), "unit": "steps/s",
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "ms_per_step": e_total / K3,
+               "note": "KV cache resident on the device; per-step tree tensors, logits and "
+                       "index arrays copied in from pinned host memory, every output copied back"}
+
+    # ---------------------------------------------------------------- CPU baseline (oracle)
+    cpu = None
+    if world == 1 and rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, t, s, args.cpu_budget)
+
+    sb = step_bytes(w, n_acc)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "layers": w.L, "batch": w.B, "heads": w.H,
+                       "head_dim": w.D, "prefix": w.P, "tree_tokens": w.T, "vocab": w.V,
+                       "S_max": w.S_max, "l2": "flushed before every step (256 MiB write, "
+                                               "outside the step events)",
+                       "parallelism": f"replicas x{world}"},
+            "step_gbs": sb / (ms_per_step * 1e-3) / 1e9,
+            "step_frac_of_8tbs": sb / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
+            "step_bytes": sb,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": traffic,
+                         "kernel": "tree_attention_kernel", "launch_us": att_ms * 1e3,
+                         "bytes_per_launch": att_bytes, "peak_kind": peak_kind,
+                         "frac_of_8000": achieved / NOMINAL_HBM_GBS},
+            "e2e": e2e,
+            "gpu_launches": 3 * K,
+            "clocks": clk,
+            "cpu_baseline": cpu,
+            "wall_s_timed": wall,
+        }
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

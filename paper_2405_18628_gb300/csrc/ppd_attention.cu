@@ -44,13 +44,14 @@ struct AttnLayout {
     static constexpr int P_GROUPS = 2 * TPMAX / 64;      // [hi | lo] columns / 64
     static constexpr uint32_t P_BYTES = P_GROUPS * GROUP_BYTES;
     static constexpr int QS = (TPMAX <= 64) ? 2 : 1;     // Q buffers
-    static constexpr int KS = (TPMAX <= 64) ? 3 : 2;     // K tile ring
+    static constexpr int PS = (TPMAX <= 64) ? 2 : 1;     // probability tiles
+    static constexpr int KS = 2;                          // K tile ring
     static constexpr int VS = 2;                          // V tile ring
     static constexpr int NC_MAX = TPMAX / 2;              // query columns per warpgroup
 
     static constexpr uint32_t OFF_Q = 0;
     static constexpr uint32_t OFF_P = OFF_Q + QS * Q_BYTES;
-    static constexpr uint32_t OFF_K = OFF_P + P_BYTES;
+    static constexpr uint32_t OFF_K = OFF_P + PS * P_BYTES;
     static constexpr uint32_t OFF_V = OFF_K + KS * TILE_BYTES;
     static constexpr uint32_t OFF_BAR = OFF_V + VS * TILE_BYTES;
     // barrier indices
@@ -63,8 +64,8 @@ struct AttnLayout {
     static constexpr int B_SFULL = B_VEMPTY + VS;
     static constexpr int B_SFREE = B_SFULL + 2;
     static constexpr int B_PFULL = B_SFREE + 2;
-    static constexpr int B_PFREE = B_PFULL + 1;
-    static constexpr int B_DRAIN = B_PFREE + 1;
+    static constexpr int B_PFREE = B_PFULL + PS;
+    static constexpr int B_DRAIN = B_PFREE + PS;
     static constexpr int NBAR = B_DRAIN + 1;
     static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
     static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
@@ -145,7 +146,9 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
     if (threadIdx.x == 0) {
         for (int i = 0; i < Lay::NBAR; ++i) {
             uint32_t count = 1;
-            if (i == Lay::B_SFREE || i == Lay::B_SFREE + 1 || i == Lay::B_PFULL) count = 8;
+            if ((i >= Lay::B_SFREE && i < Lay::B_SFREE + 2) ||
+                (i >= Lay::B_PFULL && i < Lay::B_PFULL + Lay::PS))
+                count = 8;
             mbar_init(bars + i, count);
         }
         *abort_flag = 0;
@@ -237,7 +240,8 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             const uint32_t v_lbo = (D == 128) ? Lay::GROUP_BYTES : 0u;
 
             auto issue_pv = [&](int gp, bool first) {
-                mbar_wait(bars + Lay::B_PFULL, gp & 1, abort_flag);
+                const int ps = gp % Lay::PS;
+                mbar_wait(bars + Lay::B_PFULL + ps, (gp / Lay::PS) & 1, abort_flag);
                 const int vs = gp % Lay::VS;
                 mbar_wait(bars + Lay::B_VFULL + vs, (gp / Lay::VS) & 1, abort_flag);
                 tc_fence_after();
@@ -246,11 +250,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     for (int kk = 0; kk < Lay::KT / 16; ++kk) {
                         const uint64_t a = make_smem_desc(sv + vs * Lay::TILE_BYTES + kk * 2048,
                                                           v_lbo, 1024);
-                        const uint64_t b = make_smem_desc(sp + kk * 2048, Lay::GROUP_BYTES, 1024);
+                        const uint64_t b = make_smem_desc(sp + ps * Lay::P_BYTES + kk * 2048,
+                                                          Lay::GROUP_BYTES, 1024);
                         umma_bf16(t_o, a, b, idesc_pv, (first && kk == 0) ? 0u : 1u);
                     }
                 }
-                umma_commit(bars + Lay::B_PFREE);
+                umma_commit(bars + Lay::B_PFREE + ps);
                 umma_commit(bars + Lay::B_VEMPTY + vs);
             };
 
@@ -293,10 +298,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         const int t = wq * 32 + lane;           // key row of S^T, and d of O^T
         const int NC = T_pad >> 1;              // query columns owned by this warpgroup
         const int q0 = wg * NC;
-        const int nch = NC >> 4;
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
         const uint32_t t_o = tmem_base + lane_off + 2 * TPMAX;
-        const uint32_t sp = smem_addr(smem + Lay::OFF_P);
+        // this thread's row of the probability tile (128-byte swizzled atoms)
+        const uint32_t p_row = smem_addr(smem + Lay::OFF_P) + (uint32_t)(t >> 3) * 1024u +
+                               (uint32_t)(t & 7) * 128u;
+        const uint32_t p_swz = (uint32_t)(t & 7);
         const float sl2 = p.scale_log2;
         float *red_wg = red + wg * 4 * Lay::NC_MAX;
 
@@ -306,6 +313,58 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         uint64_t dbits = 0;   // bit c: key t (tree node t) is visible to query q0 + c
         int cur_b = -1;
         int g = 0;
+
+        // Probabilities of 16 query columns [c0, c0+16) of this thread's key row
+        // with the current running maxima, split into bf16 hi + lo and stored
+        // into probability tile `pbuf` (byte offset).  `kind`: 0 every key
+        // visible, 1 keys t < n_valid visible, 2 tree-ancestor mask.  `maxd`
+        // collects the largest exponent; the caller adds pv to the row sums.
+        auto p_chunk = [&](uint32_t t_s, int c0, int kind, bool row_ok, uint32_t pbuf,
+                           float (&pv)[16], float &maxd) {
+            uint32_t r[16];
+            tmem_ld16(t_s + c0, r);
+            const float4 *m4 = reinterpret_cast<const float4 *>(m2 + q0 + c0);
+            float m[16];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float4 v = m4[k];
+                m[4 * k] = v.x;
+                m[4 * k + 1] = v.y;
+                m[4 * k + 2] = v.z;
+                m[4 * k + 3] = v.w;
+            }
+            const uint32_t bits = (uint32_t)(dbits >> c0) & 0xFFFFu;
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                float d = fmaf(__uint_as_float(r[e]), sl2, -m[e]);
+                if (kind == 1) d = row_ok ? d : -INFINITY;
+                else if (kind == 2) d = ((bits >> e) & 1u) ? d : -INFINITY;
+                maxd = fmaxf(maxd, d);
+                pv[e] = ex2(d);
+            }
+            uint32_t hw[8], lw[8];
+#pragma unroll
+            for (int e = 0; e < 16; e += 2) {
+                const uint32_t h0 = __float_as_uint(pv[e]) & 0xFFFF0000u;
+                const uint32_t h1 = __float_as_uint(pv[e + 1]) & 0xFFFF0000u;
+                hw[e >> 1] = __byte_perm(h0, h1, 0x7632);
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(pv[e] - __uint_as_float(h0),
+                                                                pv[e + 1] - __uint_as_float(h1));
+                lw[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
+            }
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                const int ch = q0 + c0 + half * 8;            // hi column
+                const int cl = T_pad + ch;                     // lo column
+                const uint32_t ah = p_row + pbuf + (uint32_t)(ch >> 6) * Lay::GROUP_BYTES +
+                                    ((((uint32_t)(ch & 63) >> 3) ^ p_swz) << 4);
+                const uint32_t al = p_row + pbuf + (uint32_t)(cl >> 6) * Lay::GROUP_BYTES +
+                                    ((((uint32_t)(cl & 63) >> 3) ^ p_swz) << 4);
+                st_shared_v4(ah, hw[half * 4], hw[half * 4 + 1], hw[half * 4 + 2], hw[half * 4 + 3]);
+                st_shared_v4(al, lw[half * 4], lw[half * 4 + 1], lw[half * 4 + 2], lw[half * 4 + 3]);
+            }
+        };
 
         for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
             const UnitInfo ui = unit_info(p, u);
@@ -350,87 +409,115 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                 const bool tree = (j == ui.n_pref);
                 const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
                 const bool row_ok = t < n_valid;
+                const int kind = tree ? 2 : (n_valid < Lay::KT ? 1 : 0);
                 const int sb = g & 1;
                 mbar_wait(bars + Lay::B_SFULL + sb, (g >> 1) & 1, abort_flag);
                 tc_fence_after();
                 const uint32_t t_s = tmem_base + lane_off + sb * TPMAX + q0;
 
-                // pass A: does any score exceed the running max by more than 2^8?
-                bool flag = false;
+                // Column groups of up to 32 queries.  Each is done optimistically
+                // with the current running maxima; if a score exceeds its maximum
+                // by more than 2^16 (or on a unit's first tile) the group takes the
+                // exact path: cross-lane tile maximum, rescale of O and of the row
+                // sums, probabilities recomputed.
+                const int ps = g % Lay::PS;
+                const uint32_t pbuf = (uint32_t)ps * Lay::P_BYTES;
+                // probability tile ps is free once the PV product of tile g - PS is done
+                if (g >= Lay::PS)
+                    mbar_wait(bars + Lay::B_PFREE + ps, ((g / Lay::PS) - 1) & 1, abort_flag);
+                bool o_ready = (Lay::PS == 1);   // PV of tile g-1 known to be complete
 #pragma unroll
-                for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
-                    if (ch < nch) {
-                        uint32_t r[16];
-                        tmem_ld16(t_s + ch * 16, r);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            const int c = ch * 16 + e;
-                            const bool vis = tree ? ((dbits >> c) & 1ull) != 0 : row_ok;
-                            const float x = __uint_as_float(r[e]) * sl2;
-                            flag |= vis && (x > m2[q0 + c] + 8.f);
+                for (int gc0 = 0; gc0 < Lay::NC_MAX; gc0 += 32) {
+                    if (gc0 < NC) {
+                        const bool two = gc0 + 16 < NC;
+                        bool exact = (j == 0);
+                        float pv0[16], pv1[16];
+                        if (!exact) {
+                            float maxd = -INFINITY;
+                            p_chunk(t_s, gc0, kind, row_ok, pbuf, pv0, maxd);
+                            if (two) p_chunk(t_s, gc0 + 16, kind, row_ok, pbuf, pv1, maxd);
+                            exact = named_bar_or(1 + wg, 128, maxd > 16.f);
                         }
-                    }
-                }
-                const bool any = named_bar_or(1 + wg, 128, flag);
-                if (any) {
-                    // exact tile maximum per query column, across the 128 key rows
+                        if (exact) {
+                            // exact maximum per query column over the tile's 128 key rows
 #pragma unroll
-                    for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
-                        if (ch < nch) {
-                            uint32_t r[16];
-                            float v[16];
-                            tmem_ld16(t_s + ch * 16, r);
-                            tmem_wait_ld();
+                            for (int h = 0; h < 2; ++h) {
+                                if (h == 0 || two) {
+                                    const int c0 = gc0 + h * 16;
+                                    uint32_t r[16];
+                                    float v[16];
+                                    tmem_ld16(t_s + c0, r);
+                                    tmem_wait_ld();
+                                    const uint32_t bits = (uint32_t)(dbits >> c0) & 0xFFFFu;
 #pragma unroll
-                            for (int e = 0; e < 16; ++e) {
-                                const int c = ch * 16 + e;
-                                const bool vis = tree ? ((dbits >> c) & 1ull) != 0 : row_ok;
-                                v[e] = vis ? __uint_as_float(r[e]) * sl2 : -INFINITY;
+                                    for (int e = 0; e < 16; ++e) {
+                                        const bool vis = kind == 0 ? true
+                                                         : kind == 1 ? row_ok
+                                                                     : ((bits >> e) & 1u) != 0;
+                                        v[e] = vis ? __uint_as_float(r[e]) * sl2 : -INFINITY;
+                                    }
+                                    const float mx = warp_transpose_reduce16(v, lane, OpMax());
+                                    if (!(lane & 1)) red_wg[wq * Lay::NC_MAX + c0 + (lane >> 1)] = mx;
+                                }
                             }
-                            const float mx = warp_transpose_reduce16(v, lane, OpMax());
-                            if (!(lane & 1)) red_wg[wq * Lay::NC_MAX + ch * 16 + (lane >> 1)] = mx;
-                        }
-                    }
-                    named_bar_sync(1 + wg, 128);
-                    if (t < NC) {
-                        const float tm = fmaxf(fmaxf(red_wg[t], red_wg[Lay::NC_MAX + t]),
-                                               fmaxf(red_wg[2 * Lay::NC_MAX + t], red_wg[3 * Lay::NC_MAX + t]));
-                        const float old = m2[q0 + t];
-                        const float nw = fmaxf(old, tm);
-                        m2[q0 + t] = nw;
-                        red_wg[t] = (nw == old) ? 1.f : ex2(old - nw);   // alpha
-                    }
-                    named_bar_sync(1 + wg, 128);
-                }
-
-                // the previous tile's PV product must be done before P or O change
-                if (g > 0) mbar_wait(bars + Lay::B_PFREE, (g - 1) & 1, abort_flag);
-                tc_fence_after();
-                if (any && j > 0) {
-#pragma unroll
-                    for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
-                        if (ch < nch) {
-                            uint32_t rh[16], rl[16];
-                            tmem_ld16(t_o + q0 + ch * 16, rh);
-                            tmem_ld16(t_o + T_pad + q0 + ch * 16, rl);
-                            tmem_wait_ld();
-#pragma unroll
-                            for (int e = 0; e < 16; ++e) {
-                                const float a = red_wg[ch * 16 + e];
-                                rh[e] = __float_as_uint(__uint_as_float(rh[e]) * a);
-                                rl[e] = __float_as_uint(__uint_as_float(rl[e]) * a);
-                                lacc[ch * 16 + e] *= a;
+                            named_bar_sync(1 + wg, 128);
+                            const int gw = two ? 32 : 16;
+                            if (t < gw) {
+                                const int c = gc0 + t;
+                                const float tm = fmaxf(fmaxf(red_wg[c], red_wg[Lay::NC_MAX + c]),
+                                                       fmaxf(red_wg[2 * Lay::NC_MAX + c],
+                                                             red_wg[3 * Lay::NC_MAX + c]));
+                                const float old = m2[q0 + c];
+                                const float nw = fmaxf(old, tm);
+                                m2[q0 + c] = nw;
+                                red_wg[c] = (nw == old) ? 1.f : ex2(old - nw);   // alpha
                             }
-                            tmem_st16(t_o + q0 + ch * 16, rh);
-                            tmem_st16(t_o + T_pad + q0 + ch * 16, rl);
+                            named_bar_sync(1 + wg, 128);
+                            if (j > 0) {
+                                // rescale the accumulated output columns and row sums; the
+                                // PV product of the previous tile must have landed in O
+                                if (!o_ready) {
+                                    const int pp = (g - 1) % Lay::PS;
+                                    mbar_wait(bars + Lay::B_PFREE + pp, ((g - 1) / Lay::PS) & 1, abort_flag);
+                                    o_ready = true;
+                                }
+                                tc_fence_after();
+#pragma unroll
+                                for (int h = 0; h < 2; ++h) {
+                                    if (h == 0 || two) {
+                                        const int c0 = gc0 + h * 16;
+                                        uint32_t rh[16], rl[16];
+                                        tmem_ld16(t_o + q0 + c0, rh);
+                                        tmem_ld16(t_o + T_pad + q0 + c0, rl);
+                                        tmem_wait_ld();
+#pragma unroll
+                                        for (int e = 0; e < 16; ++e) {
+                                            const float a = red_wg[c0 + e];
+                                            rh[e] = __float_as_uint(__uint_as_float(rh[e]) * a);
+                                            rl[e] = __float_as_uint(__uint_as_float(rl[e]) * a);
+                                            lacc[c0 + e] *= a;
+                                        }
+                                        tmem_st16(t_o + q0 + c0, rh);
+                                        tmem_st16(t_o + T_pad + q0 + c0, rl);
+                                    }
+                                }
+                                tmem_wait_st();
+                            }
+                            float maxd = -INFINITY;
+                            p_chunk(t_s, gc0, kind, row_ok, pbuf, pv0, maxd);
+                            if (two) p_chunk(t_s, gc0 + 16, kind, row_ok, pbuf, pv1, maxd);
+                        }
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) lacc[gc0 + e] += pv0[e];
+                        if (two) {
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) lacc[gc0 + 16 + e] += pv1[e];
                         }
                     }
-                    tmem_wait_st();
                 }
 
                 // V rows of invisible keys in a partial prefix tile may be NaN: zero them
-                if (!tree && n_valid < Lay::KT && wg == 0) {
+                if (kind == 1 && wg == 0) {
                     const int vs = g % Lay::VS;
                     mbar_wait(bars + Lay::B_VFULL + vs, (g / Lay::VS) & 1, abort_flag);
                     if (!row_ok) {
@@ -442,60 +529,22 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                                 st_shared_v4(vrow + c * Lay::GROUP_BYTES + x * 16, 0u, 0u, 0u, 0u);
                     }
                 }
-
-                // pass B: probabilities, row sums, bf16 hi/lo split into shared memory
-#pragma unroll
-                for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
-                    if (ch < nch) {
-                        uint32_t r[16];
-                        tmem_ld16(t_s + ch * 16, r);
-                        tmem_wait_ld();
-                        uint32_t hw[8], lw[8];
-#pragma unroll
-                        for (int e = 0; e < 16; e += 2) {
-                            float pr[2];
-#pragma unroll
-                            for (int x = 0; x < 2; ++x) {
-                                const int c = ch * 16 + e + x;
-                                const bool vis = tree ? ((dbits >> c) & 1ull) != 0 : row_ok;
-                                const float xs = __uint_as_float(r[e + x]) * sl2 - m2[q0 + c];
-                                pr[x] = vis ? ex2(xs) : 0.f;
-                                lacc[c] += pr[x];
-                            }
-                            const uint32_t h0 = __float_as_uint(pr[0]) & 0xFFFF0000u;
-                            const uint32_t h1 = __float_as_uint(pr[1]) & 0xFFFF0000u;
-                            hw[e >> 1] = __byte_perm(h0, h1, 0x7632);
-                            const __nv_bfloat162 lo = __floats2bfloat162_rn(
-                                pr[0] - __uint_as_float(h0), pr[1] - __uint_as_float(h1));
-                            lw[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
-                        }
-#pragma unroll
-                        for (int half = 0; half < 2; ++half) {
-                            const int cc = q0 + ch * 16 + half * 8;
-                            st_shared_v4(sp + sw128_offset(t, cc, Lay::GROUP_BYTES), hw[half * 4],
-                                         hw[half * 4 + 1], hw[half * 4 + 2], hw[half * 4 + 3]);
-                            st_shared_v4(sp + sw128_offset(t, T_pad + cc, Lay::GROUP_BYTES),
-                                         lw[half * 4], lw[half * 4 + 1], lw[half * 4 + 2],
-                                         lw[half * 4 + 3]);
-                        }
-                    }
-                }
                 fence_proxy_async_smem();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
-                    mbar_arrive(bars + Lay::B_PFULL);
+                    mbar_arrive(bars + Lay::B_PFULL + ps);
                     mbar_arrive(bars + Lay::B_SFREE + sb);
                 }
 
                 if (j == ui.n_tiles - 1) {
                     // -------------------------------------------------- unit epilogue
-                    mbar_wait(bars + Lay::B_PFREE, g & 1, abort_flag);
+                    mbar_wait(bars + Lay::B_PFREE + ps, (g / Lay::PS) & 1, abort_flag);
                     tc_fence_after();
                     named_bar_sync(1 + wg, 128);   // every thread is done reading alpha
 #pragma unroll
                     for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
-                        if (ch < nch) {
+                        if (ch * 16 < NC) {
                             float v[16];
 #pragma unroll
                             for (int e = 0; e < 16; ++e) v[e] = lacc[ch * 16 + e];
@@ -518,7 +567,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         float *orow = p.out + (size_t)u * T * D + t;
 #pragma unroll
                         for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
-                            if (ch < nch) {
+                            if (ch * 16 < NC) {
                                 uint32_t rh[16], rl[16];
                                 tmem_ld16(t_o + q0 + ch * 16, rh);
                                 tmem_ld16(t_o + T_pad + q0 + ch * 16, rl);
@@ -536,6 +585,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     tc_fence_before();
 #pragma unroll
                     for (int c = 0; c < Lay::NC_MAX; ++c) lacc[c] = 0.f;
+                    named_bar_sync(1 + wg, 128);   // red_wg is free again
                 }
             }
         }
