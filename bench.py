@@ -407,7 +407,7 @@ def main():
                          "bytes_per_launch": att_bytes, "peak_kind": peak_kind,
                          "frac_of_8000": achieved / NOMINAL_HBM_GBS},
             "e2e": e2e,
-            "gpu_launches": 3 * K,
+            "gpu_launches": (2 if w.B <= 64 else 5) * K,
             "clocks": clk,
             "cpu_baseline": cpu,
             "wall_s_timed": wall,

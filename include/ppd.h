@@ -72,8 +72,8 @@ typedef enum { PPD_BF16 = 0, PPD_F32 = 1 } ppd_dtype;
 /*
  * Scratch bytes the entry points below need in `workspace` for these sizes
  * (device memory, any contents, 256-byte aligned, caller-owned; it may be
- * reused between calls that are ordered on one stream).  Covers argmax
- * partial results and counters and, for PPD_F32, the bf16 copies of Q/K/V.
+ * reused between calls that are ordered on one stream).  Covers the per-split
+ * partial maxima of the node argmax and, for PPD_F32, the bf16 copies of Q/K/V.
  */
 size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt);
 
@@ -140,8 +140,11 @@ ppd_status ppd_kv_compact(void *k_cache, void *v_cache, const void *k_tree, cons
 
 /*
  * The whole verification step: node argmax and acceptance, tree-masked
- * attention over all L layers, then compaction of the accepted rows, enqueued
- * on `stream` with no host synchronisation.  Arguments as in the four entry
+ * attention over all L layers, and compaction of the accepted rows, enqueued
+ * on `stream` with no host synchronisation.  For B <= 64 this is two grids:
+ * the argmax partial maxima, then the attention grid (allowed to start while
+ * the first still runs), whose end phase combines the argmax, decides
+ * acceptance and compacts; larger batches run the steps as separate grids.  Arguments as in the four entry
  * points above; `out`/`lse` as in ppd_tree_attention, `argmax_out` as in
  * ppd_node_argmax.  Attention reads only prefix rows [0, prefix_len[b]) and
  * compaction writes only rows [prefix_len[b], new_prefix_len[b]), so the

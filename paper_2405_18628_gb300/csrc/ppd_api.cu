@@ -16,7 +16,6 @@
 namespace {
 
 using ppd::AcceptArgs;
-using ppd::ArgmaxScratch;
 using ppd::AttnMaps;
 using ppd::AttnParams;
 
@@ -48,11 +47,11 @@ int num_sms()
     return cache[dev];
 }
 
-// Argmax splits per row: enough blocks to cover the GPU, chunks >= 2048 logits.
+// Argmax splits per row: about 512 blocks over all rows, chunks >= 2048 logits.
 int argmax_splits(int64_t rows, int V)
 {
     if (rows <= 0) return 1;
-    int64_t want = (1024 + rows - 1) / rows;
+    int64_t want = (512 + rows - 1) / rows;
     int64_t cap = V / 2048;
     if (cap > 64) cap = 64;
     if (cap < 1) cap = 1;
@@ -62,7 +61,7 @@ int argmax_splits(int64_t rows, int V)
 }
 
 struct WsLayout {
-    size_t part_val, part_idx, row_count, seq_count, conv, total;
+    size_t part_val, part_idx, side, conv, total;
     int splits;
 };
 
@@ -76,10 +75,8 @@ WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, p
     off = align_up(off + (size_t)rows * w.splits * 4);
     w.part_idx = off;
     off = align_up(off + (size_t)rows * w.splits * 4);
-    w.row_count = off;
-    off = align_up(off + (size_t)rows * 4);
-    w.seq_count = off;
-    off = align_up(off + (size_t)B * 4);
+    w.side = off;
+    off = align_up(off + (size_t)num_sms() * ppd::kSideScratchInts * 4);
     w.conv = off;
     if (dt == PPD_F32) {
         const size_t lbh = (size_t)L * B * H;
@@ -158,7 +155,8 @@ bool attn_dims_ok(int L, int B, int H, int T, int D, int S_max, ppd_dtype dt)
 ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, const void *kt,
                              const void *vt, const int32_t *prefix_len, const int32_t *parent,
                              int L, int B, int H, int T, int D, int S_max, float scale, float *out,
-                             float *lse, int32_t *dev_status, cudaStream_t stream)
+                             float *lse, int32_t *dev_status, const ppd::FusedStep *fused,
+                             bool programmatic, cudaStream_t stream)
 {
     const int T_pad = (T + 31) & ~31;
     const uint64_t lbh = (uint64_t)L * B * H;
@@ -182,7 +180,9 @@ ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, cons
     p.n_units = (int)lbh;
     const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
     p.scale_log2 = sc * 1.4426950408889634f;
-    return cuda_status(ppd::launch_tree_attention(m, p, D, num_sms(), stream));
+    p.fused = fused != nullptr;
+    if (fused) p.fs = *fused;
+    return cuda_status(ppd::launch_tree_attention(m, p, D, num_sms(), programmatic, stream));
 }
 
 // fp32 operands: round to bf16 copies in the workspace first.
@@ -190,11 +190,14 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
                                  const void *vt, const int32_t *prefix_len, const int32_t *parent,
                                  int L, int B, int H, int T, int D, int S_max, ppd_dtype dt,
                                  float scale, float *out, float *lse, int32_t *dev_status,
-                                 uint8_t *ws, const WsLayout &wl, cudaStream_t stream)
+                                 uint8_t *ws, const WsLayout &wl, const ppd::FusedStep *fused,
+                                 cudaStream_t stream)
 {
+    // With bf16 operands the attention grid only reads caller inputs before its end
+    // phase, so it may overlap the preceding (argmax) grid.
     if (dt == PPD_BF16)
         return enqueue_attention(q, kc, vc, kt, vt, prefix_len, parent, L, B, H, T, D, S_max, scale,
-                                 out, lse, dev_status, stream);
+                                 out, lse, dev_status, fused, fused != nullptr, stream);
     const int64_t lbh = (int64_t)L * B * H;
     const int64_t n_t = lbh * T * D, n_c = lbh * (int64_t)S_max * D;
     uint16_t *bq = reinterpret_cast<uint16_t *>(ws + wl.conv);
@@ -202,25 +205,14 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
     uint16_t *bvt = bkt + n_t;
     uint16_t *bkc = bvt + n_t;
     uint16_t *bvc = bkc + n_c;
-    cudaError_t e;
-    if ((e = ppd::launch_round_bf16((const float *)q, bq, n_t, stream)) != cudaSuccess ||
-        (e = ppd::launch_round_bf16((const float *)kt, bkt, n_t, stream)) != cudaSuccess ||
-        (e = ppd::launch_round_bf16((const float *)vt, bvt, n_t, stream)) != cudaSuccess ||
-        (e = ppd::launch_round_bf16((const float *)kc, bkc, n_c, stream)) != cudaSuccess ||
-        (e = ppd::launch_round_bf16((const float *)vc, bvc, n_c, stream)) != cudaSuccess)
+    if (ppd::launch_round_bf16((const float *)q, bq, n_t, stream) != cudaSuccess ||
+        ppd::launch_round_bf16((const float *)kt, bkt, n_t, stream) != cudaSuccess ||
+        ppd::launch_round_bf16((const float *)vt, bvt, n_t, stream) != cudaSuccess ||
+        ppd::launch_round_bf16((const float *)kc, bkc, n_c, stream) != cudaSuccess ||
+        ppd::launch_round_bf16((const float *)vc, bvc, n_c, stream) != cudaSuccess)
         return PPD_ERR_CUDA;
     return enqueue_attention(bq, bkc, bvc, bkt, bvt, prefix_len, parent, L, B, H, T, D, S_max,
-                             scale, out, lse, dev_status, stream);
-}
-
-ArgmaxScratch argmax_scratch(uint8_t *ws, const WsLayout &wl)
-{
-    ArgmaxScratch s;
-    s.part_val = reinterpret_cast<float *>(ws + wl.part_val);
-    s.part_idx = reinterpret_cast<int32_t *>(ws + wl.part_idx);
-    s.row_count = reinterpret_cast<int32_t *>(ws + wl.row_count);
-    s.seq_count = reinterpret_cast<int32_t *>(ws + wl.seq_count);
-    return s;
+                             scale, out, lse, dev_status, fused, false, stream);
 }
 
 }  // namespace
@@ -268,7 +260,7 @@ ppd_status ppd_tree_attention(const void *q, const void *k_cache, const void *v_
     if (cudaMemsetAsync(dev_status, 0, (size_t)B * 4, s) != cudaSuccess) return PPD_ERR_CUDA;
     return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B, H,
                                  T, D, S_max, dt, scale, out, lse, dev_status,
-                                 static_cast<uint8_t *>(workspace), wl, s);
+                                 static_cast<uint8_t *>(workspace), wl, nullptr, s);
 }
 
 ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *argmax_out,
@@ -277,15 +269,15 @@ ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *ar
     if (!logits || !argmax_out || B < 1 || T < 1 || V < 1) return PPD_ERR_INVALID_ARG;
     if ((double)B * T * V > 9.0e15 || (double)B * T * 64 > 2147483647.0) return PPD_ERR_INVALID_ARG;
     const WsLayout wl = workspace_layout(1, B, 1, T, 1, V, 0, PPD_BF16);
+    if (!workspace || ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    ArgmaxScratch scr{};
-    if (wl.splits > 1) {
-        if (!workspace || ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
-        scr = argmax_scratch(static_cast<uint8_t *>(workspace), wl);
-        if (cudaMemsetAsync(scr.row_count, 0, (size_t)B * T * 4, s) != cudaSuccess) return PPD_ERR_CUDA;
-    }
-    return cuda_status(
-        ppd::launch_node_argmax(logits, (int64_t)B * T, V, wl.splits, argmax_out, scr, nullptr, B, s));
+    float *pv = reinterpret_cast<float *>(ws + wl.part_val);
+    int32_t *pi = reinterpret_cast<int32_t *>(ws + wl.part_idx);
+    const int64_t rows = (int64_t)B * T;
+    if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, nullptr, 0, s) != cudaSuccess)
+        return PPD_ERR_CUDA;
+    return cuda_status(ppd::launch_argmax_combine(pv, pi, rows, wl.splits, argmax_out, s));
 }
 
 ppd_status ppd_accept_path(const int32_t *argmax, const int32_t *cand_tokens,
@@ -358,22 +350,50 @@ ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
     if (ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    float *pv = reinterpret_cast<float *>(ws + wl.part_val);
+    int32_t *pi = reinterpret_cast<int32_t *>(ws + wl.part_idx);
+    const int64_t rows = (int64_t)B * T;
 
-    // 1. node argmax; the block finishing a sequence's last row runs acceptance
-    const ArgmaxScratch scr = argmax_scratch(ws, wl);
-    if (cudaMemsetAsync(ws + wl.row_count, 0, wl.conv - wl.row_count, s) != cudaSuccess)
+    if (B <= ppd::kFusedMaxB) {
+        // 1. partial maxima of every node's logits (also zeroes dev_status)
+        if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, dev_status, B, s) !=
+            cudaSuccess)
+            return PPD_ERR_CUDA;
+        // 2. attention over every layer, overlapping step 1; its end phase combines
+        //    the argmax, decides acceptance and compacts the accepted rows
+        ppd::FusedStep f{};
+        f.part_val = pv;
+        f.part_idx = pi;
+        f.splits = wl.splits;
+        f.cand_tokens = cand_tokens;
+        f.argmax_out = argmax_out;
+        f.accept_len = accept_len;
+        f.path = path;
+        f.next_token = next_token;
+        f.new_prefix_len = new_prefix_len;
+        f.status = dev_status;
+        f.k_cache = static_cast<uint8_t *>(k_cache);
+        f.v_cache = static_cast<uint8_t *>(v_cache);
+        f.k_tree = static_cast<const uint8_t *>(k_tree);
+        f.v_tree = static_cast<const uint8_t *>(v_tree);
+        f.row_bytes = D * eb;
+        f.V = V;
+        f.scratch = reinterpret_cast<int *>(ws + wl.side);
+        return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B,
+                                     H, T, D, S_max, dt, scale, out, lse, nullptr, ws, wl, &f, s);
+    }
+
+    // large batches: the same steps as separate grids
+    if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, nullptr, 0, s) != cudaSuccess ||
+        ppd::launch_argmax_combine(pv, pi, rows, wl.splits, argmax_out, s) != cudaSuccess)
         return PPD_ERR_CUDA;
     AcceptArgs a{cand_tokens, parent, prefix_len, accept_len, path, next_token, new_prefix_len,
                  dev_status, T, V, S_max};
-    if (ppd::launch_node_argmax(logits, (int64_t)B * T, V, wl.splits, argmax_out, scr, &a, B, s) !=
-        cudaSuccess)
-        return PPD_ERR_CUDA;
-    // 2. tree attention over every layer (reads cache rows [0, prefix_len) only)
+    if (ppd::launch_accept_path(argmax_out, a, B, s) != cudaSuccess) return PPD_ERR_CUDA;
     ppd_status st = enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent,
                                           L, B, H, T, D, S_max, dt, scale, out, lse, dev_status,
-                                          ws, wl, s);
+                                          ws, wl, nullptr, s);
     if (st != PPD_OK) return st;
-    // 3. compaction (writes cache rows [prefix_len, prefix_len + accept_len) only)
     return cuda_status(ppd::launch_kv_compact(k_cache, v_cache, k_tree, v_tree, path, accept_len,
                                               prefix_len, L, B, H, T, D, S_max, eb, s));
 }
@@ -389,7 +409,7 @@ ppd_status ppd_selftest_umma(const void *a, const void *b, float *d, int mode, i
     if (mode == 0) {
         if (!encode_2d(&ma, a, 128, 128, 128) || !encode_2d(&mb, b, 128, N, N)) return PPD_ERR_CUDA;
     } else {
-        if (!encode_2d(&ma, a, mode == 1 ? 128 : 64, 128, 128)) return PPD_ERR_CUDA;
+        if (!encode_2d(&ma, a, mode == 2 ? 64 : 128, 128, 128)) return PPD_ERR_CUDA;
         mb = ma;
     }
     return cuda_status(ppd::launch_selftest_umma(ma, mb, b, d, mode, N, static_cast<cudaStream_t>(stream)));

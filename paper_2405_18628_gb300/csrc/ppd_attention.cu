@@ -15,19 +15,24 @@
 //                          ~2^-16) and written to shared memory
 //   O^T += V^T * [P_hi | P_lo]^T    one tcgen05.mma, M = D, N = 2*T_pad, K = 128
 //
-// Warp roles (320 threads): warps 0-7 softmax (two warpgroups, each owning
+// Warp roles (352 threads): warps 0-7 softmax (two warpgroups, each owning
 // half of the query columns), warp 8 TMA producer, warp 9 MMA issuer and TMEM
-// owner.  The running row maximum m is updated lazily: a tile only triggers
-// a cross-lane max reduction (and a rescale of O and of the row sums) when
-// one of its scores exceeds the current m by more than 8 (log2 units), so
-// in steady state the softmax is purely per-thread.  The tree mask is an
-// ancestor bitset built from the parent array; rows beyond the prefix (which
-// may hold anything, NaN included) are masked by select and their V rows are
-// zeroed in shared memory before the PV product.
+// owner, warp 10 the fused step's argmax / acceptance / compaction.  The running row maximum m is updated lazily: a tile is first done
+// with the current m, and only if a score exceeds m by more than 2^16 (or on
+// a unit's first tile) does it take the exact path -- a cross-lane maximum,
+// a rescale of O and of the row sums, and recomputed probabilities.  The
+// tree mask is an ancestor bitset built from the parent array; rows beyond
+// the prefix (which may hold anything, NaN included) are masked by select
+// and their V rows are zeroed in shared memory before the PV product.  For
+// trees of up to 64 tokens O is double-buffered in TMEM and a unit's output
+// is read back only after the next unit's first tile, so the stream of tiles
+// never waits for a unit's last PV product.
+#include "ppd_accept.cuh"
 #include "ppd_device.cuh"
 #include "ppd_kernels.h"
 
 #include <cmath>
+#include <type_traits>
 
 namespace ppd {
 
@@ -43,11 +48,13 @@ struct AttnLayout {
     static constexpr uint32_t Q_BYTES = TPMAX * D * 2;
     static constexpr int P_GROUPS = 2 * TPMAX / 64;      // [hi | lo] columns / 64
     static constexpr uint32_t P_BYTES = P_GROUPS * GROUP_BYTES;
+    static constexpr int OB = (TPMAX <= 64) ? 2 : 1;     // O accumulators in TMEM
     static constexpr int QS = (TPMAX <= 64) ? 2 : 1;     // Q buffers
     static constexpr int PS = (TPMAX <= 64) ? 2 : 1;     // probability tiles
     static constexpr int KS = 2;                          // K tile ring
     static constexpr int VS = 2;                          // V tile ring
     static constexpr int NC_MAX = TPMAX / 2;              // query columns per warpgroup
+    static constexpr int ANC_WORDS = TPMAX / 32;          // ancestor bitset words per node
 
     static constexpr uint32_t OFF_Q = 0;
     static constexpr uint32_t OFF_P = OFF_Q + QS * Q_BYTES;
@@ -70,15 +77,22 @@ struct AttnLayout {
     static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
     static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
     static constexpr uint32_t OFF_M2 = (OFF_ABORT + 4 + 15) & ~15u;
-    static constexpr uint32_t OFF_UNION = OFF_M2 + TPMAX * 4;
-    // union: ancestor bitsets [128][4] u32, or reduction scratch [2][4][NC_MAX] f32
-    static constexpr uint32_t UNION_BYTES = 128 * 16;
+    // [OB][TPMAX] reciprocal row sums; with one accumulator they share the
+    // running maxima's storage (read back before the maxima are reset)
+    static constexpr uint32_t OFF_LINV = (OB == 1) ? OFF_M2 : OFF_M2 + TPMAX * 4;
+    static constexpr uint32_t OFF_UNION = OFF_M2 + TPMAX * 4 + (OB == 1 ? 0 : OB * TPMAX * 4);
+    // union: ancestor bitsets [TPMAX][ANC_WORDS] u32, or reduction scratch [2][4][NC_MAX] f32
+    static constexpr uint32_t ANC_BYTES = TPMAX * ANC_WORDS * 4;
+    static constexpr uint32_t RED_BYTES = 2 * 4 * NC_MAX * 4;
+    static constexpr uint32_t UNION_BYTES = ANC_BYTES > RED_BYTES ? ANC_BYTES : RED_BYTES;
     static constexpr uint32_t SMEM_BYTES = OFF_UNION + UNION_BYTES;
-    static constexpr uint32_t TMEM_COLS = 4 * TPMAX;   // S0 | S1 | O (hi | lo)
+    // TMEM columns: S0 | S1 | O0 (hi | lo) [| O1 (hi | lo)]
+    static constexpr uint32_t T_S = 0, T_O = 2 * TPMAX;
+    static constexpr uint32_t TMEM_COLS = (2 + 2 * OB) * TPMAX <= 256 ? 256 : 512;
 
-    static_assert(2 * 4 * NC_MAX * 4 <= (int)UNION_BYTES, "reduction scratch");
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
     static_assert((OFF_P | OFF_K | OFF_V) % 1024 == 0, "1024-byte aligned operand tiles");
+    static_assert((2 + 2 * OB) * TPMAX <= 512, "TMEM budget");
 };
 
 struct UnitInfo {
@@ -113,8 +127,84 @@ PPD_DEV void mbar_wait_drain(uint64_t *bar, uint32_t parity)
         if (global_timer() - t0 > kWaitLimitNs) return;
 }
 
+template <int K>
+using kind_t = std::integral_constant<int, K>;
+
+// Mask kinds of a tile: every key visible (a full prefix tile), keys t < n_valid
+// visible (the last, partial prefix tile), or the tree-ancestor mask.
+enum : int { kMaskNone = 0, kMaskRows = 1, kMaskTree = 2 };
+
+// Side work of the fused verification step, done by one extra warp of every CTA
+// while the other warps stream attention.  Once the preceding argmax grid has
+// completed (griddepcontrol.wait), for every sequence b this CTA touches -- or
+// is designated to report (b mod grid) -- the warp combines the node argmax
+// from the partial maxima, decides acceptance, writes the sequence's outputs
+// if designated, and copies the accepted tree K/V rows of this CTA's own
+// (layer, sequence, head) slices into the cache.  Attention only reads cache
+// rows below each prefix, so the copies never race with it.  Scratch (parent
+// copies, top-1 tokens, path) lives in a per-CTA slice of the workspace.
+PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const FusedStep &f = p.fs;
+    const int T = p.T, B = p.B, S = f.splits;
+    int *s_par = f.scratch + (size_t)blockIdx.x * kSideScratchInts;
+    int *top = s_par + 128;
+    int *path = top + 128;
+    const int chunks = f.row_bytes >> 4;
+    for (int b = 0; b < B; ++b) {
+        const bool designated = (b % (int)gridDim.x) == (int)blockIdx.x;
+        bool has_unit = false;
+        for (int u = blockIdx.x; u < p.n_units && !has_unit; u += gridDim.x)
+            has_unit = ((u / p.H) % B) == b;
+        if (!designated && !has_unit) continue;
+        for (int r = lane; r < T; r += 32) {
+            const size_t base = ((size_t)b * T + r) * S;
+            float bv = __ldcg(f.part_val + base);
+            int bi = __ldcg(f.part_idx + base);
+#pragma unroll 8
+            for (int k = 1; k < S; ++k) consider(__ldcg(f.part_val + base + k), __ldcg(f.part_idx + base + k), bv, bi);
+            top[r] = bi;
+            if (designated) f.argmax_out[(size_t)b * T + r] = bi;
+        }
+        __syncwarp();
+        const AcceptResult res =
+            accept_warp([&](int n) { return top[n]; }, p.parent + (size_t)b * T,
+                        f.cand_tokens + (size_t)b * T, __ldg(p.prefix_len + b), T, f.V, p.S_max,
+                        lane, s_par, path);
+        if (designated) {
+            for (int i = lane; i < T; i += 32) f.path[(size_t)b * T + i] = path[i];
+            if (lane == 0) {
+                f.accept_len[b] = res.n_acc;
+                f.next_token[b] = res.next_token;
+                f.new_prefix_len[b] = res.new_prefix_len;
+                atomicMax(f.status + b, res.status);
+            }
+        }
+        if (has_unit && res.n_acc > 0) {
+            // cache rows [P_b, P_b + n_acc) <- the accepted tree rows
+            const int P = __ldg(p.prefix_len + b);
+            const int n = res.n_acc;
+            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
+                if (((u / p.H) % B) != b) continue;
+                for (int w = lane; w < n * chunks; w += 32) {
+                    const int j = w / chunks, c = w - j * chunks;
+                    const int src = path[j];
+                    const size_t so = ((size_t)u * T + src) * f.row_bytes + (size_t)c * 16;
+                    const size_t dof = ((size_t)u * p.S_max + P + j) * f.row_bytes + (size_t)c * 16;
+                    const uint4 kx = __ldg(reinterpret_cast<const uint4 *>(f.k_tree + so));
+                    const uint4 vx = __ldg(reinterpret_cast<const uint4 *>(f.v_tree + so));
+                    *reinterpret_cast<uint4 *>(f.k_cache + dof) = kx;
+                    *reinterpret_cast<uint4 *>(f.v_cache + dof) = vx;
+                }
+            }
+        }
+        __syncwarp();
+    }
+}
+
 template <int D, int TPMAX>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(352, 1)
 tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                       const __grid_constant__ CUtensorMap map_kc,
                       const __grid_constant__ CUtensorMap map_vc,
@@ -135,7 +225,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
     uint32_t *tmem_ptr = reinterpret_cast<uint32_t *>(smem + Lay::OFF_TMEMPTR);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + Lay::OFF_ABORT);
     float *m2 = reinterpret_cast<float *>(smem + Lay::OFF_M2);
-    uint32_t *anc = reinterpret_cast<uint32_t *>(smem + Lay::OFF_UNION);   // [128][4]
+    uint32_t *anc = reinterpret_cast<uint32_t *>(smem + Lay::OFF_UNION);   // [TPMAX][ANC_WORDS]
     float *red = reinterpret_cast<float *>(smem + Lay::OFF_UNION);         // [2][4][NC_MAX]
 
     const int warp = threadIdx.x >> 5;
@@ -164,7 +254,10 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
     tc_fence_after();
     const uint32_t tmem_base = *tmem_ptr;
 
-    if (warp == 8) {
+    if (warp == 10) {
+        // ------------------------------------------------------------ fused-step side work
+        if (p.fused) fused_side_warp(p, lane);
+    } else if (warp == 8) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             tma_prefetch_map(&map_q);
@@ -233,13 +326,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             const uint32_t sk = smem_addr(smem + Lay::OFF_K);
             const uint32_t sv = smem_addr(smem + Lay::OFF_V);
             const uint32_t sp = smem_addr(smem + Lay::OFF_P);
-            const uint32_t t_o = tmem_base + 2 * TPMAX;
             // V^T as the A operand: M = D spans the tile's 64-column groups.  With
             // D = 64 both M halves read the same group (rows 64..127 of O^T repeat
             // rows 0..63 and are ignored).
             const uint32_t v_lbo = (D == 128) ? Lay::GROUP_BYTES : 0u;
 
-            auto issue_pv = [&](int gp, bool first) {
+            auto issue_pv = [&](int gp, bool first, uint32_t t_o) {
                 const int ps = gp % Lay::PS;
                 mbar_wait(bars + Lay::B_PFULL + ps, (gp / Lay::PS) & 1, abort_flag);
                 const int vs = gp % Lay::VS;
@@ -263,6 +355,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
                 const UnitInfo ui = unit_info(p, u);
                 const int qs = k % Lay::QS;
+                const uint32_t t_o = tmem_base + Lay::T_O + (uint32_t)(k % Lay::OB) * 2 * TPMAX;
                 mbar_wait(bars + Lay::B_QFULL + qs, (k / Lay::QS) & 1, abort_flag);
                 for (int j = 0; j < ui.n_tiles; ++j, ++g) {
                     const int ks = g % Lay::KS;
@@ -277,15 +370,15 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                             const uint32_t qoff = (kk >> 2) * Lay::Q_GROUP_BYTES + (kk & 3) * 32;
                             const uint64_t a = make_smem_desc(sk + ks * Lay::TILE_BYTES + koff, 16, 1024);
                             const uint64_t b = make_smem_desc(sq + qs * Lay::Q_BYTES + qoff, 16, 1024);
-                            umma_bf16(tmem_base + sb * TPMAX, a, b, idesc_qk, kk > 0 ? 1u : 0u);
+                            umma_bf16(tmem_base + Lay::T_S + sb * TPMAX, a, b, idesc_qk, kk > 0 ? 1u : 0u);
                         }
                     }
                     umma_commit(bars + Lay::B_SFULL + sb);
                     umma_commit(bars + Lay::B_KEMPTY + ks);
                     if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
-                    if (j >= 1) issue_pv(g - 1, j == 1);
+                    if (j >= 1) issue_pv(g - 1, j == 1, t_o);
                 }
-                issue_pv(g - 1, ui.n_tiles == 1);
+                issue_pv(g - 1, ui.n_tiles == 1, t_o);
             }
             // all MMAs finished before TMEM can be released
             umma_commit(bars + Lay::B_DRAIN);
@@ -299,85 +392,147 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         const int NC = T_pad >> 1;              // query columns owned by this warpgroup
         const int q0 = wg * NC;
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
-        const uint32_t t_o = tmem_base + lane_off + 2 * TPMAX;
         // this thread's row of the probability tile (128-byte swizzled atoms)
         const uint32_t p_row = smem_addr(smem + Lay::OFF_P) + (uint32_t)(t >> 3) * 1024u +
                                (uint32_t)(t & 7) * 128u;
         const uint32_t p_swz = (uint32_t)(t & 7);
         const float sl2 = p.scale_log2;
         float *red_wg = red + wg * 4 * Lay::NC_MAX;
+        float *linv = reinterpret_cast<float *>(smem + Lay::OFF_LINV);   // [OB][TPMAX]
 
-        float lacc[Lay::NC_MAX];
+        constexpr int NL = Lay::NC_MAX;
+        float lacc[NL];   // this key row's share of every owned query's row sum
 #pragma unroll
-        for (int c = 0; c < Lay::NC_MAX; ++c) lacc[c] = 0.f;
+        for (int c = 0; c < NL; ++c) lacc[c] = 0.f;
         uint64_t dbits = 0;   // bit c: key t (tree node t) is visible to query q0 + c
         int cur_b = -1;
         int g = 0;
+        // a finished unit whose output still sits in TMEM
+        bool pend = false;
+        int pend_u = 0, pend_ob = 0, pend_g = 0;
 
-        // Probabilities of 16 query columns [c0, c0+16) of this thread's key row
-        // with the current running maxima, split into bf16 hi + lo and stored
-        // into probability tile `pbuf` (byte offset).  `kind`: 0 every key
-        // visible, 1 keys t < n_valid visible, 2 tree-ancestor mask.  `maxd`
-        // collects the largest exponent; the caller adds pv to the row sums.
-        auto p_chunk = [&](uint32_t t_s, int c0, int kind, bool row_ok, uint32_t pbuf,
-                           float (&pv)[16], float &maxd) {
-            uint32_t r[16];
-            tmem_ld16(t_s + c0, r);
-            const float4 *m4 = reinterpret_cast<const float4 *>(m2 + q0 + c0);
-            float m[16];
+        // Probabilities of query columns [c0, c0+16) (and [c0+16, c0+32) when `two`)
+        // of this thread's key row with the current running maxima, exponents
+        // clamped at 64 so nothing overflows before a rescale.  STORE: split into
+        // bf16 hi + lo, store into probability tile `pbuf` (byte offset) and add to
+        // lacc.  UNDO: subtract the same values from lacc again (a bit-identical
+        // recomputation).  `maxd` collects the largest unclamped exponent.
+        auto p_group = [&](auto kind_c, auto undo_c, uint32_t t_s, int c0, bool two, bool row_ok,
+                           uint32_t pbuf, float &maxd) {
+            constexpr int KIND = decltype(kind_c)::value;
+            constexpr bool UNDO = decltype(undo_c)::value != 0;
+            const uint32_t bits = (uint32_t)(dbits >> c0);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float4 v = m4[k];
-                m[4 * k] = v.x;
-                m[4 * k + 1] = v.y;
-                m[4 * k + 2] = v.z;
-                m[4 * k + 3] = v.w;
-            }
-            const uint32_t bits = (uint32_t)(dbits >> c0) & 0xFFFFu;
-            tmem_wait_ld();
+            for (int h = 0; h < 2; ++h) {
+                if (h == 0 || two) {
+                    const int cb = c0 + h * 16;
+                    uint32_t r[16];
+                    tmem_ld16(t_s + cb, r);
+                    const float4 *m4 = reinterpret_cast<const float4 *>(m2 + q0 + cb);
+                    float m[16];
 #pragma unroll
-            for (int e = 0; e < 16; ++e) {
-                float d = fmaf(__uint_as_float(r[e]), sl2, -m[e]);
-                if (kind == 1) d = row_ok ? d : -INFINITY;
-                else if (kind == 2) d = ((bits >> e) & 1u) ? d : -INFINITY;
-                maxd = fmaxf(maxd, d);
-                pv[e] = ex2(d);
-            }
-            uint32_t hw[8], lw[8];
+                    for (int k = 0; k < 4; ++k) {
+                        const float4 v = m4[k];
+                        m[4 * k] = v.x;
+                        m[4 * k + 1] = v.y;
+                        m[4 * k + 2] = v.z;
+                        m[4 * k + 3] = v.w;
+                    }
+                    float pv[16];
+                    tmem_wait_ld();
 #pragma unroll
-            for (int e = 0; e < 16; e += 2) {
-                const uint32_t h0 = __float_as_uint(pv[e]) & 0xFFFF0000u;
-                const uint32_t h1 = __float_as_uint(pv[e + 1]) & 0xFFFF0000u;
-                hw[e >> 1] = __byte_perm(h0, h1, 0x7632);
-                const __nv_bfloat162 lo = __floats2bfloat162_rn(pv[e] - __uint_as_float(h0),
-                                                                pv[e + 1] - __uint_as_float(h1));
-                lw[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
-            }
+                    for (int e = 0; e < 16; ++e) {
+                        float d = fmaf(__uint_as_float(r[e]), sl2, -m[e]);
+                        if (KIND == kMaskRows) d = row_ok ? d : -INFINITY;
+                        if (KIND == kMaskTree) d = ((bits >> (h * 16 + e)) & 1u) ? d : -INFINITY;
+                        maxd = fmaxf(maxd, d);
+                        pv[e] = ex2(fminf(d, 64.f));
+                        if (UNDO) lacc[cb + e] -= pv[e];
+                        else lacc[cb + e] += pv[e];
+                    }
+                    if (!UNDO) {
+                        uint32_t hw[8], lw[8];
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                const int ch = q0 + c0 + half * 8;            // hi column
-                const int cl = T_pad + ch;                     // lo column
-                const uint32_t ah = p_row + pbuf + (uint32_t)(ch >> 6) * Lay::GROUP_BYTES +
-                                    ((((uint32_t)(ch & 63) >> 3) ^ p_swz) << 4);
-                const uint32_t al = p_row + pbuf + (uint32_t)(cl >> 6) * Lay::GROUP_BYTES +
-                                    ((((uint32_t)(cl & 63) >> 3) ^ p_swz) << 4);
-                st_shared_v4(ah, hw[half * 4], hw[half * 4 + 1], hw[half * 4 + 2], hw[half * 4 + 3]);
-                st_shared_v4(al, lw[half * 4], lw[half * 4 + 1], lw[half * 4 + 2], lw[half * 4 + 3]);
+                        for (int e = 0; e < 16; e += 2) {
+                            const uint32_t h0 = __float_as_uint(pv[e]) & 0xFFFF0000u;
+                            const uint32_t h1 = __float_as_uint(pv[e + 1]) & 0xFFFF0000u;
+                            hw[e >> 1] = __byte_perm(h0, h1, 0x7632);
+                            const __nv_bfloat162 lo = __floats2bfloat162_rn(pv[e] - __uint_as_float(h0),
+                                                                            pv[e + 1] - __uint_as_float(h1));
+                            lw[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
+                        }
+#pragma unroll
+                        for (int half = 0; half < 2; ++half) {
+                            const int ch = q0 + cb + half * 8;   // hi column
+                            const int cl = T_pad + ch;            // lo column
+                            const uint32_t ah = p_row + pbuf + (uint32_t)(ch >> 6) * Lay::GROUP_BYTES +
+                                                ((((uint32_t)(ch & 63) >> 3) ^ p_swz) << 4);
+                            const uint32_t al = p_row + pbuf + (uint32_t)(cl >> 6) * Lay::GROUP_BYTES +
+                                                ((((uint32_t)(cl & 63) >> 3) ^ p_swz) << 4);
+                            st_shared_v4(ah, hw[half * 4], hw[half * 4 + 1], hw[half * 4 + 2], hw[half * 4 + 3]);
+                            st_shared_v4(al, lw[half * 4], lw[half * 4 + 1], lw[half * 4 + 2], lw[half * 4 + 3]);
+                        }
+                    }
+                }
             }
         };
+        auto run_group = [&](auto undo_c, int kind, uint32_t t_s, int c0, bool two, bool row_ok,
+                             uint32_t pbuf, float &maxd) {
+            if (kind == kMaskNone) p_group(kind_t<kMaskNone>{}, undo_c, t_s, c0, two, row_ok, pbuf, maxd);
+            else if (kind == kMaskRows) p_group(kind_t<kMaskRows>{}, undo_c, t_s, c0, two, row_ok, pbuf, maxd);
+            else p_group(kind_t<kMaskTree>{}, undo_c, t_s, c0, two, row_ok, pbuf, maxd);
+        };
+        using store_t = kind_t<0>;
+        using undo_t = kind_t<1>;
 
-        for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
+        // Output of a finished unit: O (hi + lo) from its TMEM accumulator times the
+        // reciprocal row sums, one head-dim element per thread, queries in order.
+        auto read_back = [&](int u_out, int ob, int g_last) {
+            mbar_wait(bars + Lay::B_PFREE + g_last % Lay::PS, (g_last / Lay::PS) & 1, abort_flag);
+            tc_fence_after();
+            if (wq * 32 < D) {
+                const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * 2 * TPMAX;
+                const float *li = linv + ob * TPMAX;
+                float *orow = p.out + (size_t)u_out * T * D + t;
+#pragma unroll
+                for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                    if (ch * 16 < NC) {
+                        uint32_t rh[16], rl[16];
+                        tmem_ld16(t_o + q0 + ch * 16, rh);
+                        tmem_ld16(t_o + T_pad + q0 + ch * 16, rl);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const int q = q0 + ch * 16 + e;
+                            if (q < T)
+                                orow[(size_t)q * D] =
+                                    (__uint_as_float(rh[e]) + __uint_as_float(rl[e])) * li[q];
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+        };
+
+        int k = 0;
+        for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
             const UnitInfo ui = unit_info(p, u);
+            const int ob = k % Lay::OB;
+            const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * 2 * TPMAX;
             if (ui.b != cur_b) {
                 // ancestor bitsets of this sequence's tree, one node per thread
                 named_bar_sync(3, 256);
                 const int i = wg * 128 + t;
                 if (i < T) {
-                    uint32_t w[4] = {0u, 0u, 0u, 0u};
+                    uint32_t w[Lay::ANC_WORDS];
+#pragma unroll
+                    for (int x = 0; x < Lay::ANC_WORDS; ++x) w[x] = 0u;
                     bool bad = false;
                     int a = i;
                     while (true) {
-                        w[a >> 5] |= 1u << (a & 31);
+#pragma unroll
+                        for (int x = 0; x < Lay::ANC_WORDS; ++x)
+                            if ((a >> 5) == x) w[x] |= 1u << (a & 31);
                         const int pa = __ldg(p.parent + (size_t)ui.b * T + a);
                         if (a == 0) {
                             bad = (pa != -1);
@@ -390,16 +545,19 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         a = pa;
                     }
 #pragma unroll
-                    for (int x = 0; x < 4; ++x) anc[i * 4 + x] = w[x];
+                    for (int x = 0; x < Lay::ANC_WORDS; ++x) anc[i * Lay::ANC_WORDS + x] = w[x];
                     if (bad && p.dev_status) p.dev_status[ui.b] = kErrTree;
                 }
                 if (i == 0 && p.dev_status && (ui.P_raw < 0 || ui.P_raw > p.S_max))
                     p.dev_status[ui.b] = kErrCapacity;
                 named_bar_sync(3, 256);
                 dbits = 0;
-                for (int c = 0; c < NC; ++c) {
-                    const int q = q0 + c;
-                    if (q < T && ((anc[q * 4 + (t >> 5)] >> (t & 31)) & 1u)) dbits |= 1ull << c;
+                if (t < T) {
+                    for (int c = 0; c < NC; ++c) {
+                        const int q = q0 + c;
+                        if (q < T && ((anc[q * Lay::ANC_WORDS + (t >> 5)] >> (t & 31)) & 1u))
+                            dbits |= 1ull << c;
+                    }
                 }
                 named_bar_sync(3, 256);
                 cur_b = ui.b;
@@ -409,37 +567,42 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                 const bool tree = (j == ui.n_pref);
                 const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
                 const bool row_ok = t < n_valid;
-                const int kind = tree ? 2 : (n_valid < Lay::KT ? 1 : 0);
+                const int kind = tree ? kMaskTree : (n_valid < Lay::KT ? kMaskRows : kMaskNone);
                 const int sb = g & 1;
                 mbar_wait(bars + Lay::B_SFULL + sb, (g >> 1) & 1, abort_flag);
                 tc_fence_after();
-                const uint32_t t_s = tmem_base + lane_off + sb * TPMAX + q0;
-
-                // Column groups of up to 32 queries.  Each is done optimistically
-                // with the current running maxima; if a score exceeds its maximum
-                // by more than 2^16 (or on a unit's first tile) the group takes the
-                // exact path: cross-lane tile maximum, rescale of O and of the row
-                // sums, probabilities recomputed.
+                const uint32_t t_s = tmem_base + lane_off + Lay::T_S + sb * TPMAX + q0;
                 const int ps = g % Lay::PS;
                 const uint32_t pbuf = (uint32_t)ps * Lay::P_BYTES;
                 // probability tile ps is free once the PV product of tile g - PS is done
                 if (g >= Lay::PS)
                     mbar_wait(bars + Lay::B_PFREE + ps, ((g / Lay::PS) - 1) & 1, abort_flag);
                 bool o_ready = (Lay::PS == 1);   // PV of tile g-1 known to be complete
+
+                // Column groups of up to 32 queries, done optimistically with the
+                // current running maxima; on a unit's first tile, or when a score
+                // exceeds its maximum by more than 2^16, the group takes the exact
+                // path: cross-lane tile maximum, rescale of O and of the row sums,
+                // probabilities recomputed.
 #pragma unroll
                 for (int gc0 = 0; gc0 < Lay::NC_MAX; gc0 += 32) {
                     if (gc0 < NC) {
                         const bool two = gc0 + 16 < NC;
-                        bool exact = (j == 0);
-                        float pv0[16], pv1[16];
-                        if (!exact) {
+                        bool exact;
+                        if (j > 0) {
                             float maxd = -INFINITY;
-                            p_chunk(t_s, gc0, kind, row_ok, pbuf, pv0, maxd);
-                            if (two) p_chunk(t_s, gc0 + 16, kind, row_ok, pbuf, pv1, maxd);
+                            run_group(store_t{}, kind, t_s, gc0, two, row_ok, pbuf, maxd);
                             exact = named_bar_or(1 + wg, 128, maxd > 16.f);
+                        } else {
+                            named_bar_sync(1 + wg, 128);   // earlier readers of red_wg are done
+                            exact = true;
                         }
                         if (exact) {
-                            // exact maximum per query column over the tile's 128 key rows
+                            if (j > 0) {
+                                // take the optimistic contributions back out of the row sums
+                                float unused = 0.f;
+                                run_group(undo_t{}, kind, t_s, gc0, two, row_ok, pbuf, unused);
+                            }
 #pragma unroll
                             for (int h = 0; h < 2; ++h) {
                                 if (h == 0 || two) {
@@ -448,12 +611,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                                     float v[16];
                                     tmem_ld16(t_s + c0, r);
                                     tmem_wait_ld();
-                                    const uint32_t bits = (uint32_t)(dbits >> c0) & 0xFFFFu;
+                                    const uint32_t bits = (uint32_t)(dbits >> c0);
 #pragma unroll
                                     for (int e = 0; e < 16; ++e) {
-                                        const bool vis = kind == 0 ? true
-                                                         : kind == 1 ? row_ok
-                                                                     : ((bits >> e) & 1u) != 0;
+                                        const bool vis = kind == kMaskNone ? true
+                                                         : kind == kMaskRows ? row_ok
+                                                                             : ((bits >> e) & 1u) != 0;
                                         v[e] = vis ? __uint_as_float(r[e]) * sl2 : -INFINITY;
                                     }
                                     const float mx = warp_transpose_reduce16(v, lane, OpMax());
@@ -475,7 +638,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                             named_bar_sync(1 + wg, 128);
                             if (j > 0) {
                                 // rescale the accumulated output columns and row sums; the
-                                // PV product of the previous tile must have landed in O
+                                // PV product of the previous tile must have landed first
                                 if (!o_ready) {
                                     const int pp = (g - 1) % Lay::PS;
                                     mbar_wait(bars + Lay::B_PFREE + pp, ((g - 1) / Lay::PS) & 1, abort_flag);
@@ -486,38 +649,34 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                                 for (int h = 0; h < 2; ++h) {
                                     if (h == 0 || two) {
                                         const int c0 = gc0 + h * 16;
-                                        uint32_t rh[16], rl[16];
-                                        tmem_ld16(t_o + q0 + c0, rh);
-                                        tmem_ld16(t_o + T_pad + q0 + c0, rl);
-                                        tmem_wait_ld();
+                                        float a[16];
 #pragma unroll
-                                        for (int e = 0; e < 16; ++e) {
-                                            const float a = red_wg[c0 + e];
-                                            rh[e] = __float_as_uint(__uint_as_float(rh[e]) * a);
-                                            rl[e] = __float_as_uint(__uint_as_float(rl[e]) * a);
-                                            lacc[c0 + e] *= a;
+                                        for (int e = 0; e < 16; ++e) a[e] = red_wg[c0 + e];
+#pragma unroll
+                                        for (int part = 0; part < 2; ++part) {
+                                            const uint32_t col = t_o + (part ? T_pad : 0) + q0 + c0;
+                                            uint32_t rr[16];
+                                            tmem_ld16(col, rr);
+                                            tmem_wait_ld();
+#pragma unroll
+                                            for (int e = 0; e < 16; ++e)
+                                                rr[e] = __float_as_uint(__uint_as_float(rr[e]) * a[e]);
+                                            tmem_st16(col, rr);
                                         }
-                                        tmem_st16(t_o + q0 + c0, rh);
-                                        tmem_st16(t_o + T_pad + q0 + c0, rl);
+#pragma unroll
+                                        for (int e = 0; e < 16; ++e) lacc[c0 + e] *= a[e];
                                     }
                                 }
                                 tmem_wait_st();
                             }
                             float maxd = -INFINITY;
-                            p_chunk(t_s, gc0, kind, row_ok, pbuf, pv0, maxd);
-                            if (two) p_chunk(t_s, gc0 + 16, kind, row_ok, pbuf, pv1, maxd);
-                        }
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) lacc[gc0 + e] += pv0[e];
-                        if (two) {
-#pragma unroll
-                            for (int e = 0; e < 16; ++e) lacc[gc0 + 16 + e] += pv1[e];
+                            run_group(store_t{}, kind, t_s, gc0, two, row_ok, pbuf, maxd);
                         }
                     }
                 }
 
                 // V rows of invisible keys in a partial prefix tile may be NaN: zero them
-                if (kind == 1 && wg == 0) {
+                if (kind == kMaskRows && wg == 0) {
                     const int vs = g % Lay::VS;
                     mbar_wait(bars + Lay::B_VFULL + vs, (g / Lay::VS) & 1, abort_flag);
                     if (!row_ok) {
@@ -537,10 +696,14 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     mbar_arrive(bars + Lay::B_SFREE + sb);
                 }
 
+                // the previous unit's output, once this unit's first tile is on its way
+                if (j == 0 && pend) {
+                    read_back(pend_u, pend_ob, pend_g);
+                    pend = false;
+                }
+
                 if (j == ui.n_tiles - 1) {
-                    // -------------------------------------------------- unit epilogue
-                    mbar_wait(bars + Lay::B_PFREE + ps, (g / Lay::PS) & 1, abort_flag);
-                    tc_fence_after();
+                    // ------------------------------------------ unit end: row sums, LSE
                     named_bar_sync(1 + wg, 128);   // every thread is done reading alpha
 #pragma unroll
                     for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
@@ -559,69 +722,76 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         const int q = q0 + t;
                         if (p.lse && q < T)
                             p.lse[(size_t)u * T + q] = (m2[q] + lg2(l)) * 0.69314718055994530942f;
-                        red_wg[t] = 1.f / l;
-                        m2[q] = -INFINITY;
+                        linv[ob * TPMAX + q] = rcp(l);
+                        if (Lay::OB > 1) m2[q] = -INFINITY;
                     }
-                    named_bar_sync(1 + wg, 128);
-                    if (wq * 32 < D) {
-                        float *orow = p.out + (size_t)u * T * D + t;
 #pragma unroll
-                        for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
-                            if (ch * 16 < NC) {
-                                uint32_t rh[16], rl[16];
-                                tmem_ld16(t_o + q0 + ch * 16, rh);
-                                tmem_ld16(t_o + T_pad + q0 + ch * 16, rl);
-                                tmem_wait_ld();
-#pragma unroll
-                                for (int e = 0; e < 16; ++e) {
-                                    const int q = q0 + ch * 16 + e;
-                                    if (q < T)
-                                        orow[(size_t)q * D] = (__uint_as_float(rh[e]) + __uint_as_float(rl[e])) *
-                                                              red_wg[ch * 16 + e];
-                                }
-                            }
-                        }
+                    for (int c = 0; c < NL; ++c) lacc[c] = 0.f;
+                    pend = true;
+                    pend_u = u;
+                    pend_ob = ob;
+                    pend_g = g;
+                    if (Lay::OB == 1) {
+                        // a single accumulator: read it back before the next unit reuses it,
+                        // then reset the running maxima that share storage with 1 / l
+                        named_bar_sync(1 + wg, 128);
+                        read_back(pend_u, pend_ob, pend_g);
+                        pend = false;
+                        named_bar_sync(1 + wg, 128);
+                        if (t < NC) m2[q0 + t] = -INFINITY;
                     }
-                    tc_fence_before();
-#pragma unroll
-                    for (int c = 0; c < Lay::NC_MAX; ++c) lacc[c] = 0.f;
-                    named_bar_sync(1 + wg, 128);   // red_wg is free again
                 }
             }
+        }
+        if (pend) {
+            named_bar_sync(1 + wg, 128);   // the reciprocal row sums are in shared memory
+            read_back(pend_u, pend_ob, pend_g);
         }
     }
 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (*abort_flag && threadIdx.x == 0 && p.dev_status)
-        for (int b = 0; b < p.B; ++b) p.dev_status[b] = kErrTimeout;
+    if (*abort_flag && threadIdx.x == 0) {
+        for (int b = 0; b < p.B; ++b) {
+            if (p.dev_status) p.dev_status[b] = kErrTimeout;
+            if (p.fused) atomicMax(p.fs.status + b, (int)kErrTimeout);
+        }
+    }
     if (warp == 9) tmem_dealloc(tmem_base, Lay::TMEM_COLS);
 }
 
 template <int D, int TPMAX>
 static cudaError_t launch_tree_attention_t(const AttnMaps &m, const AttnParams &p, int num_sms,
-                                           cudaStream_t stream)
+                                           bool programmatic, cudaStream_t stream)
 {
     using Lay = AttnLayout<D, TPMAX>;
     auto kern = tree_attention_kernel<D, TPMAX>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)Lay::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    const int grid = p.n_units < num_sms ? p.n_units : num_sms;
-    kern<<<grid, 320, Lay::SMEM_BYTES, stream>>>(m.q, m.kc, m.vc, m.kt, m.vt, p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(p.n_units < num_sms ? p.n_units : num_sms));
+    cfg.blockDim = dim3(352);
+    cfg.dynamicSmemBytes = Lay::SMEM_BYTES;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = programmatic ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, m.q, m.kc, m.vc, m.kt, m.vt, p);
 }
 
 cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
-                                  cudaStream_t stream)
+                                  bool programmatic, cudaStream_t stream)
 {
     if (D == 128) {
-        if (p.T_pad <= 64) return launch_tree_attention_t<128, 64>(m, p, num_sms, stream);
-        return launch_tree_attention_t<128, 128>(m, p, num_sms, stream);
+        if (p.T_pad <= 64) return launch_tree_attention_t<128, 64>(m, p, num_sms, programmatic, stream);
+        return launch_tree_attention_t<128, 128>(m, p, num_sms, programmatic, stream);
     }
-    if (p.T_pad <= 64) return launch_tree_attention_t<64, 64>(m, p, num_sms, stream);
-    return launch_tree_attention_t<64, 128>(m, p, num_sms, stream);
+    if (p.T_pad <= 64) return launch_tree_attention_t<64, 64>(m, p, num_sms, programmatic, stream);
+    return launch_tree_attention_t<64, 128>(m, p, num_sms, programmatic, stream);
 }
 
 }  // namespace ppd

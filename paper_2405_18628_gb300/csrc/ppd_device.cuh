@@ -302,6 +302,13 @@ PPD_DEV float lg2(float x)
     return y;
 }
 
+PPD_DEV float rcp(float x)
+{
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // Reduce 16 per-lane columns over the 32 lanes of a warp.  On return lane L
 // holds the reduction of column (L >> 1) over all lanes (lanes 2c and 2c+1
 // agree).  16 shuffles for 16 columns.

@@ -15,22 +15,55 @@ struct AttnMaps {
     CUtensorMap q, kc, vc, kt, vt;
 };
 
+// The fused verification step's side work (see ppd_attention.cu): argmax
+// partials from the preceding grid, acceptance, and compaction of the CTA's
+// own (layer, sequence, head) slices.
+struct FusedStep {
+    const float *part_val;       // [B*T*splits] partial maxima
+    const int32_t *part_idx;
+    int splits;
+    const int32_t *cand_tokens;  // [B,T]
+    int32_t *argmax_out;         // [B,T]
+    int32_t *accept_len;         // [B]
+    int32_t *path;               // [B,T]
+    int32_t *next_token;         // [B]
+    int32_t *new_prefix_len;     // [B]
+    int32_t *status;             // [B], zeroed by the argmax grid, raised with atomicMax
+    uint8_t *k_cache, *v_cache;  // raw cache storage
+    const uint8_t *k_tree, *v_tree;
+    int row_bytes;               // D * element size
+    int V;
+    int *scratch;                // [grid][kSideScratchInts] per-CTA scratch of the side warp
+};
+
+// Per-CTA scratch of the fused step's side warp: parent copy, top-1 tokens, path.
+constexpr int kSideScratchInts = 3 * 128 + 8;
+
 struct AttnParams {
     const int32_t *prefix_len;  // [B]
     const int32_t *parent;      // [B,T]
     float *out;                 // [L,B,H,T,D]
     float *lse;                 // [L,B,H,T] or null
-    int32_t *dev_status;        // [B] or null
+    int32_t *dev_status;        // [B] or null (main-loop errors; null in the fused step)
     int L, B, H, T, T_pad, S_max, n_units;
     float scale_log2;           // softmax scale * log2(e)
+    int fused;                  // run the end phase below
+    FusedStep fs;
 };
 
-cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
-                                  cudaStream_t stream);
+// Batches up to this size run the fused two-grid step.
+constexpr int kFusedMaxB = 64;
 
-// Node argmax over rows of fp32 logits, split over `splits` blocks per row
-// with a last-block combine.  When `acc` is non-null, the block that
-// finishes the last row of a sequence also runs the acceptance rule for it.
+cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
+                                  bool programmatic, cudaStream_t stream);
+
+// Node argmax in two steps: per-(row, split) partial maxima, then a combine.
+cudaError_t launch_argmax_partials(const float *logits, int64_t rows, int V, int splits,
+                                   float *part_val, int32_t *part_idx, int32_t *zero_status,
+                                   int n_zero, cudaStream_t stream);
+cudaError_t launch_argmax_combine(const float *part_val, const int32_t *part_idx, int64_t rows,
+                                  int splits, int32_t *argmax_out, cudaStream_t stream);
+
 struct AcceptArgs {
     const int32_t *cand_tokens;  // [B,T]
     const int32_t *parent;       // [B,T]
@@ -42,17 +75,6 @@ struct AcceptArgs {
     int32_t *dev_status;         // [B]
     int T, V, S_max;
 };
-
-struct ArgmaxScratch {
-    float *part_val;       // [rows * splits]
-    int32_t *part_idx;     // [rows * splits]
-    int32_t *row_count;    // [rows]   zero on entry, left zero on exit
-    int32_t *seq_count;    // [B]      zero on entry, left zero on exit
-};
-
-cudaError_t launch_node_argmax(const float *logits, int64_t rows, int V, int splits,
-                               int32_t *argmax_out, const ArgmaxScratch &ws,
-                               const AcceptArgs *acc, int B, cudaStream_t stream);
 
 cudaError_t launch_accept_path(const int32_t *argmax, const AcceptArgs &a, int B,
                                cudaStream_t stream);

@@ -10,6 +10,7 @@
 // walks its nodes' root paths, and a warp max-reduction picks the deepest
 // accepted node.  Compaction (Section 3 step (3)) copies the accepted rows
 // into the cache with 16-byte loads and stores.
+#include "ppd_accept.cuh"
 #include "ppd_device.cuh"
 #include "ppd_kernels.h"
 
@@ -20,124 +21,21 @@ namespace ppd {
 
 // ------------------------------------------------------------------ argmax
 
-// true when (av, ai) ranks before (bv, bi): NaN first (lowest index among
-// NaNs), then larger value, then lower index.  -0 == +0 compare equal.
-PPD_DEV bool ranks_before(float av, int ai, float bv, int bi)
-{
-    const bool an = av != av, bn = bv != bv;
-    if (an || bn) return an && bn ? ai < bi : an;
-    if (av != bv) return av > bv;
-    return ai < bi;
-}
-
-PPD_DEV void consider(float v, int i, float &bv, int &bi)
-{
-    if (ranks_before(v, i, bv, bi)) {
-        bv = v;
-        bi = i;
-    }
-}
-
-PPD_DEV int32_t ld_cg(const int32_t *p) { return __ldcg(p); }
-
-// One warp decides acceptance for sequence b; argmax values are read through
-// L2 because other blocks of the same grid may have written them.
-PPD_DEV void accept_sequence(int b, const int32_t *argmax_all, const AcceptArgs &a, int lane,
-                             int *s_par)
-{
-    const int T = a.T;
-    const int32_t *par = a.parent + (size_t)b * T;
-    const int32_t *tok = a.cand_tokens + (size_t)b * T;
-    const int32_t *top = argmax_all + (size_t)b * T;
-    bool bad = false;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int i = lane + 32 * k;
-        if (i < T) {
-            const int pa = __ldg(par + i);
-            const int tk = __ldg(tok + i);
-            s_par[i] = pa;
-            if (i == 0)
-                bad |= (pa != -1) || tk < 0 || tk >= a.V;
-            else
-                bad |= pa < 0 || pa >= i || tk < -1 || tk >= a.V;
-        }
-    }
-    __syncwarp();
-    bad = __any_sync(0xffffffffu, bad);
-    const int P = __ldg(a.prefix_len + b);
-    int err = bad ? kErrTree : ((P < 0 || P > a.S_max) ? kErrCapacity : kOk);
-
-    uint32_t okw[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int i = lane + 32 * k;
-        bool ok = false;
-        if (i < T && err == kOk) {
-            if (i == 0) {
-                ok = true;
-            } else {
-                const int tk = __ldg(tok + i);
-                ok = tk >= 0 && tk == ld_cg(top + s_par[i]);
-            }
-        }
-        okw[k] = __ballot_sync(0xffffffffu, ok);
-    }
-
-    int best_key = -1;   // (depth << 8) | (255 - node): deepest, then smallest index
-    if (err == kOk) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int i = lane + 32 * k;
-            if (i < T) {
-                int n = i, depth = 0;
-                bool good = true;
-                while (n > 0) {
-                    const uint32_t w = (n < 32) ? okw[0] : (n < 64) ? okw[1] : (n < 96) ? okw[2] : okw[3];
-                    good &= ((w >> (n & 31)) & 1u) != 0;
-                    n = s_par[n];
-                    ++depth;
-                }
-                if (good) best_key = max(best_key, (depth << 8) | (255 - i));
-            }
-        }
-    }
-    best_key = __reduce_max_sync(0xffffffffu, best_key);
-    const int best = 255 - (best_key & 255);
-    const int n_acc = (best_key >> 8) + 1;
-    if (err == kOk && (long long)P + n_acc > a.S_max) err = kErrCapacity;
-    const int n_out = (err == kOk) ? n_acc : 0;
-
-    int32_t *pth = a.path + (size_t)b * T;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int i = lane + 32 * k;
-        if (i < T && i >= n_out) pth[i] = -1;
-    }
-    if (lane == 0) {
-        if (err == kOk) {
-            int n = best;
-            for (int j = n_acc - 1; j >= 0; --j) {
-                pth[j] = n;
-                n = s_par[n];
-            }
-        }
-        a.accept_len[b] = n_out;
-        a.next_token[b] = (err == kOk) ? ld_cg(top + best) : -1;
-        a.new_prefix_len[b] = (err == kOk) ? P + n_acc : P;
-        a.dev_status[b] = err;
-    }
-}
-
+// Partial top-1 of rows of fp32 logits: block (row, s) scans columns
+// [s*chunk, (s+1)*chunk) with 16-byte loads and writes its (value, index) to
+// part_*[row * splits + s].  Block 0 also zeroes `zero_status` (the fused step's
+// per-sequence status, raised later with atomicMax).  A grid launched after
+// this one with programmatic stream serialization may start right away.
 template <bool kVec>
 __global__ void __launch_bounds__(256)
-node_argmax_kernel(const float *__restrict__ logits, int64_t rows, int V, int splits, int chunk,
-                   int32_t *argmax_out, ArgmaxScratch ws, AcceptArgs acc, int has_acc)
+argmax_partial_kernel(const float *__restrict__ logits, int V, int splits, int chunk,
+                      float *part_val, int32_t *part_idx, int32_t *zero_status, int n_zero)
 {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __shared__ float s_v[8];
     __shared__ int s_i[8];
-    __shared__ int s_flag;
-    __shared__ int s_par[128];
+    if (zero_status && blockIdx.x == 0)
+        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_status[i] = 0;
     const int64_t row = blockIdx.x / splits;
     const int s = blockIdx.x % splits;
     const int lo = s * chunk;
@@ -186,61 +84,40 @@ node_argmax_kernel(const float *__restrict__ logits, int64_t rows, int V, int sp
     __syncthreads();
     if (threadIdx.x == 0) {
         for (int w = 1; w < 8; ++w) consider(s_v[w], s_i[w], bv, bi);
-        int done = 0;
-        if (splits == 1) {
-            argmax_out[row] = bi;
-            done = 1;
-        } else {
-            ws.part_val[row * splits + s] = bv;
-            ws.part_idx[row * splits + s] = bi;
-            __threadfence();
-            const int prev = atomicAdd(ws.row_count + row, 1);
-            if (prev == splits - 1) {
-                __threadfence();
-                float cv = __ldcg(ws.part_val + row * splits);
-                int ci = __ldcg(ws.part_idx + row * splits);
-                for (int k = 1; k < splits; ++k)
-                    consider(__ldcg(ws.part_val + row * splits + k), __ldcg(ws.part_idx + row * splits + k),
-                             cv, ci);
-                argmax_out[row] = ci;
-                ws.row_count[row] = 0;
-                done = 1;
-            }
-        }
-        int last_of_seq = 0;
-        if (done && has_acc) {
-            __threadfence();
-            const int b = (int)(row / acc.T);
-            const int prev = atomicAdd(ws.seq_count + b, 1);
-            if (prev == acc.T - 1) {
-                __threadfence();
-                ws.seq_count[b] = 0;
-                last_of_seq = 1;
-            }
-        }
-        s_flag = last_of_seq;
+        part_val[row * splits + s] = bv;
+        part_idx[row * splits + s] = bi;
     }
-    __syncthreads();
-    if (s_flag && warp == 0) accept_sequence((int)(row / acc.T), argmax_out, acc, lane, s_par);
 }
 
-cudaError_t launch_node_argmax(const float *logits, int64_t rows, int V, int splits,
-                               int32_t *argmax_out, const ArgmaxScratch &ws,
-                               const AcceptArgs *acc, int B, cudaStream_t stream)
+__global__ void argmax_combine_kernel(const float *part_val, const int32_t *part_idx, int64_t rows,
+                                      int splits, int32_t *argmax_out)
 {
-    (void)B;
+    const int64_t row = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (row < rows) argmax_out[row] = combine_partials(part_val, part_idx, row, splits);
+}
+
+cudaError_t launch_argmax_partials(const float *logits, int64_t rows, int V, int splits,
+                                   float *part_val, int32_t *part_idx, int32_t *zero_status,
+                                   int n_zero, cudaStream_t stream)
+{
     const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
     int chunk = (V + splits - 1) / splits;
     chunk = (chunk + 3) & ~3;
-    AcceptArgs a{};
-    if (acc) a = *acc;
     const dim3 grid((unsigned)(rows * splits));
     if (vec)
-        node_argmax_kernel<true><<<grid, 256, 0, stream>>>(logits, rows, V, splits, chunk, argmax_out,
-                                                          ws, a, acc != nullptr);
+        argmax_partial_kernel<true><<<grid, 256, 0, stream>>>(logits, V, splits, chunk, part_val,
+                                                              part_idx, zero_status, n_zero);
     else
-        node_argmax_kernel<false><<<grid, 256, 0, stream>>>(logits, rows, V, splits, chunk, argmax_out,
-                                                           ws, a, acc != nullptr);
+        argmax_partial_kernel<false><<<grid, 256, 0, stream>>>(logits, V, splits, chunk, part_val,
+                                                               part_idx, zero_status, n_zero);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_argmax_combine(const float *part_val, const int32_t *part_idx, int64_t rows,
+                                  int splits, int32_t *argmax_out, cudaStream_t stream)
+{
+    argmax_combine_kernel<<<(unsigned)((rows + 127) / 128), 128, 0, stream>>>(part_val, part_idx, rows,
+                                                                              splits, argmax_out);
     return cudaGetLastError();
 }
 
@@ -252,7 +129,17 @@ accept_path_kernel(const int32_t *argmax, AcceptArgs a, int B)
     __shared__ int s_par[4][128];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.x * 4 + warp;
-    if (b < B) accept_sequence(b, argmax, a, lane, s_par[warp]);
+    if (b >= B) return;
+    const int32_t *top = argmax + (size_t)b * a.T;
+    const AcceptResult r = accept_warp([&](int n) { return __ldg(top + n); }, a.parent + (size_t)b * a.T,
+                                       a.cand_tokens + (size_t)b * a.T, __ldg(a.prefix_len + b), a.T,
+                                       a.V, a.S_max, lane, s_par[warp], a.path + (size_t)b * a.T);
+    if (lane == 0) {
+        a.accept_len[b] = r.n_acc;
+        a.next_token[b] = r.next_token;
+        a.new_prefix_len[b] = r.new_prefix_len;
+        a.dev_status[b] = r.status;
+    }
 }
 
 cudaError_t launch_accept_path(const int32_t *argmax, const AcceptArgs &a, int B,

@@ -290,3 +290,44 @@ def test_verify_step_is_repeatable(cuda_device):
     g2, b2 = _verify_step(w, s, t, cuda_device)
     assert torch.equal(out1, b2.out)
     assert torch.equal(kc1.view(torch.int16), g2["k_cache"].view(torch.int16))
+
+
+@pytest.mark.parametrize("B", [64, 65])
+def test_verify_step_batch_paths(cuda_device, B):
+    """B <= 64 runs the fused two-grid step; larger batches run separate grids."""
+    w = W.Workload("batch", L=1, B=B, H=2, D=64, P=40, T=16, V=300, n_cand=8, max_depth=3,
+                   chains="every1", match_rate=0.8, seed=B)
+    rng = np.random.default_rng(B)
+    pl = rng.integers(0, 41, size=B).astype(np.int32)
+    s = W.make_step_inputs(w, prefix_len=pl)
+    t = tensors(w, prefix_len=pl)
+    g, bufs = _verify_step(w, s, t, cuda_device)
+    ref = oracle.verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
+                             s.prefix_len, s.parent, s.cand_tokens, s.logits)
+    assert_attn_close(bufs.out.cpu().numpy().reshape(ref["out"].shape), ref["out"], f"B={B}")
+    np.testing.assert_array_equal(bufs.argmax.cpu().numpy(), ref["argmax"])
+    for k in ("accept_len", "path", "next_token", "new_prefix_len"):
+        np.testing.assert_array_equal(getattr(bufs, k).cpu().numpy(), ref[k], err_msg=k)
+    np.testing.assert_array_equal(bufs.dev_status.cpu().numpy(), ref["status"])
+    np.testing.assert_array_equal(g["k_cache"].cpu().view(torch.int16).numpy().view(np.uint16),
+                                  ref["k_cache"])
+    np.testing.assert_array_equal(g["v_cache"].cpu().view(torch.int16).numpy().view(np.uint16),
+                                  ref["v_cache"])
+
+
+def test_verify_step_reports_bad_sequences(cuda_device):
+    """Per-sequence device status in the fused step: a malformed tree and a
+    path that does not fit leave those sequences unaccepted and uncompacted."""
+    w = W.scaled(W.WORKLOADS["tiny"], B=3)
+    s = W.make_step_inputs(w)
+    s.parent[1, 7] = 9                       # parent after child
+    s.prefix_len[2] = w.S_max                # no room for even the root
+    t = tensors(w, prefix_len=s.prefix_len)
+    g, bufs = _verify_step(w, s, t, cuda_device)
+    ref = oracle.verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
+                             s.prefix_len, s.parent, s.cand_tokens, s.logits)
+    assert bufs.dev_status.cpu().tolist() == ref["status"].tolist() == [0, 3, 4]
+    for k in ("accept_len", "path", "next_token", "new_prefix_len"):
+        np.testing.assert_array_equal(getattr(bufs, k).cpu().numpy(), ref[k], err_msg=k)
+    np.testing.assert_array_equal(g["k_cache"].cpu().view(torch.int16).numpy().view(np.uint16),
+                                  ref["k_cache"])

@@ -52,3 +52,4 @@ def test_mn_major_half_width(cuda_device):
     ref = a.float().T @ b.float()
     torch.testing.assert_close(d.cpu()[:64], ref, rtol=1e-4, atol=1e-3)
     torch.testing.assert_close(d.cpu()[64:], ref, rtol=1e-4, atol=1e-3)
+
