@@ -160,6 +160,29 @@ ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
                            int32_t *new_prefix_len, int32_t *dev_status,
                            void *workspace, size_t ws_bytes, void *stream);
 
+/*
+ * Node argmax without a workspace (no paper counterpart; an interface for
+ * callers that cannot allocate device memory).  Same inputs, outputs, ranking
+ * rule and stream behaviour as ppd_node_argmax, but the per-split partial maxima
+ * live in a fixed 512 KiB array inside the library (a static __device__ object
+ * that every GPU loading the library holds until the process exits), so the
+ * call needs no scratch buffer.  It is meant for code that must not call
+ * cudaMalloc or a caching allocator at this point: a plugin given only the
+ * tensors it reads and writes, a real-time loop that forbids allocation after
+ * start-up, or memory budgets that are fixed in advance.  The function itself
+ * calls no allocating routine.
+ *   - Size limit: B*T <= 65536 node rows; larger requests return
+ *     PPD_ERR_UNSUPPORTED without enqueuing anything.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before any stream capture that contains this entry point.
+ *   - All calls share the array: calls whose kernels may overlap on the GPU
+ *     (different streams without ordering) race and give undefined results.
+ *     Nothing in the array needs to start at zero; each call rewrites what it reads.
+ */
+ppd_status ppd_node_argmax_noalloc(const float *logits, int B, int T, int V, int32_t *argmax_out,
+                                   void *stream);
+
 /* Human-readable name of a status code (static string). */
 const char *ppd_status_string(ppd_status s);
 

@@ -47,18 +47,7 @@ int num_sms()
     return cache[dev];
 }
 
-// Argmax splits per row: about 512 blocks over all rows, chunks >= 2048 logits.
-int argmax_splits(int64_t rows, int V)
-{
-    if (rows <= 0) return 1;
-    int64_t want = (512 + rows - 1) / rows;
-    int64_t cap = V / 2048;
-    if (cap > 64) cap = 64;
-    if (cap < 1) cap = 1;
-    if (want > cap) want = cap;
-    if (want < 1) want = 1;
-    return (int)want;
-}
+int argmax_splits(int64_t rows, int V) { return ppd::argmax_split_count(rows, V); }
 
 struct WsLayout {
     size_t part_val, part_idx, side, conv, total;

@@ -57,6 +57,20 @@ constexpr int kFusedMaxB = 64;
 cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
                                   bool programmatic, cudaStream_t stream);
 
+// Splits per node row of the argmax: about 512 blocks over all rows, chunks of
+// at least 2048 logits, at most 64 splits.
+inline int argmax_split_count(int64_t rows, int V)
+{
+    if (rows <= 0) return 1;
+    int64_t want = (512 + rows - 1) / rows;
+    int64_t cap = V / 2048;
+    if (cap > 64) cap = 64;
+    if (cap < 1) cap = 1;
+    if (want > cap) want = cap;
+    if (want < 1) want = 1;
+    return (int)want;
+}
+
 // Node argmax in two steps: per-(row, split) partial maxima, then a combine.
 cudaError_t launch_argmax_partials(const float *logits, int64_t rows, int V, int splits,
                                    float *part_val, int32_t *part_idx, int32_t *zero_status,

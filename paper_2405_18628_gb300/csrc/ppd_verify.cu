@@ -10,12 +10,14 @@
 // walks its nodes' root paths, and a warp max-reduction picks the deepest
 // accepted node.  Compaction (Section 3 step (3)) copies the accepted rows
 // into the cache with 16-byte loads and stores.
+#include "ppd.h"
 #include "ppd_accept.cuh"
 #include "ppd_device.cuh"
 #include "ppd_kernels.h"
 
 #include <climits>
 #include <cmath>
+#include <mutex>
 
 namespace ppd {
 
@@ -322,4 +324,63 @@ cudaError_t launch_selftest_umma(const CUtensorMap &ma, const CUtensorMap &mb, c
     return cudaGetLastError();
 }
 
+// ------------------------------------------------------------------ argmax without a workspace
+//
+// ppd_node_argmax_noalloc keeps its partial maxima in this fixed array instead of a
+// caller-provided workspace.  Every GPU that loads the library holds it until the
+// process exits.  Host code may not use the array's name as a device address: the
+// address is looked up once per device with cudaGetSymbolAddress, with that device
+// current, on the first call there.
+namespace {
+
+constexpr int64_t kNoAllocMaxPartials = 1 << 16;   // (row, split) pairs: 512 KiB in total
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocMaxPartials * 8];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+void *g_noalloc_addr[kMaxDevices] = {nullptr};
+
+// Device address of the scratch array on the current device (looked up once).
+cudaError_t noalloc_scratch(void **addr)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (g_noalloc_addr[dev] == nullptr) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        g_noalloc_addr[dev] = p;
+    }
+    *addr = g_noalloc_addr[dev];
+    return cudaSuccess;
+}
+
+}  // namespace
+
 }  // namespace ppd
+
+extern "C" ppd_status ppd_node_argmax_noalloc(const float *logits, int B, int T, int V,
+                                              int32_t *argmax_out, void *stream)
+{
+    if (!logits || !argmax_out || B < 1 || T < 1 || V < 1) return PPD_ERR_INVALID_ARG;
+    if ((double)B * T * V > 9.0e15) return PPD_ERR_INVALID_ARG;
+    const int64_t rows = (int64_t)B * T;
+    if (rows > ppd::kNoAllocMaxPartials) return PPD_ERR_UNSUPPORTED;   // B*T above the array's size
+    int splits = ppd::argmax_split_count(rows, V);
+    if (rows * splits > ppd::kNoAllocMaxPartials) splits = (int)(ppd::kNoAllocMaxPartials / rows);
+    void *scratch = nullptr;
+    if (ppd::noalloc_scratch(&scratch) != cudaSuccess) return PPD_ERR_CUDA;
+    float *pv = static_cast<float *>(scratch);
+    int32_t *pi = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(scratch) +
+                                              ppd::kNoAllocMaxPartials * 4);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (ppd::launch_argmax_partials(logits, rows, V, splits, pv, pi, nullptr, 0, s) != cudaSuccess)
+        return PPD_ERR_CUDA;
+    return ppd::launch_argmax_combine(pv, pi, rows, splits, argmax_out, s) == cudaSuccess ? PPD_OK
+                                                                                          : PPD_ERR_CUDA;
+}
+

@@ -49,6 +49,7 @@ def load() -> ctypes.CDLL:
             "ppd_kv_compact": ([vp] * 7 + [i32] * 7 + [vp], i32),
             "ppd_verify_step": ([vp] * 9 + [i32] * 8 + [f32] + [vp] * 8 + [vp, sz, vp], i32),
             "ppd_selftest_umma": ([vp, vp, vp, i32, i32, vp], i32),
+            "ppd_node_argmax_noalloc": ([vp, i32, i32, i32, vp, vp], i32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -121,6 +122,14 @@ def ppd_node_argmax(logits, argmax_out, workspace=None, stream=None):
     st = load().ppd_node_argmax(_ptr(logits), B, T, V, _ptr(argmax_out), _ptr(workspace), ws_n,
                                 _stream(stream))
     _check(st, "ppd_node_argmax")
+
+
+def ppd_node_argmax_noalloc(logits, argmax_out, stream=None):
+    """Node argmax without a workspace: logits fp32 [B,T,V] -> argmax_out int32
+    [B,T], partial maxima kept in the library's fixed device array."""
+    B, T, V = logits.shape
+    st = load().ppd_node_argmax_noalloc(_ptr(logits), B, T, V, _ptr(argmax_out), _stream(stream))
+    _check(st, "ppd_node_argmax_noalloc")
 
 
 def ppd_accept_path(argmax, cand_tokens, parent, prefix_len, V, S_max, accept_len, path,
