@@ -198,11 +198,28 @@ def parse():
     return ap.parse_args()
 
 
-def dist_setup():
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+def dist_setup(env=None):
+    """(world size, rank, local rank) from the torchrun environment."""
+    env = os.environ if env is None else env
+    world = int(env.get("WORLD_SIZE", "1"))
+    rank = int(env.get("RANK", "0"))
+    local = int(env.get("LOCAL_RANK", "0"))
     return world, rank, local
+
+
+def max_over_ranks(value: float, dist=None, device="cpu") -> float:
+    """The largest `value` over all ranks (the slowest rank's time)."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_rate(steps_per_rank: int, world: int, slowest_ms: float) -> float:
+    """Whole-job steps/s: every rank's steps over the slowest rank's time."""
+    return world * steps_per_rank / (slowest_ms / 1e3)
 
 
 def run_reference(args, w, world, rank):
@@ -309,13 +326,9 @@ def main():
             pg.barrier()
         wall = time.perf_counter() - wall0
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    total_ms = sum(step_ms)
-    if pg:
-        tt = torch.tensor([total_ms], device=dev)
-        pg.all_reduce(tt, op=pg.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(sum(step_ms), pg, dev)
     ms_per_step = total_ms / K
-    value = world * K / (total_ms / 1e3)
+    value = aggregate_rate(K, world, total_ms)
     clk = clocks.summary()
 
     # ---------------------------------------------------------------- dominant kernel alone
@@ -374,12 +387,8 @@ def main():
             t0 = time.perf_counter()
             e2e_step()
             e_ms.append((time.perf_counter() - t0) * 1e3)
-        e_total = sum(e_ms)
-        if pg:
-            tt = torch.tensor([e_total], device=dev)
-            pg.all_reduce(tt, op=pg.ReduceOp.MAX)
-            e_total = float(tt.item())
-        e2e = {"value": world * K3 / (e_total / 1e3), "unit": "steps/s",
+        e_total = max_over_ranks(sum(e_ms), pg, dev)
+        e2e = {"value": aggregate_rate(K3, world, e_total), "unit": "steps/s",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "ms_per_step": e_total / K3,
                "note": "KV cache resident on the device; per-step tree tensors, logits and "

@@ -252,9 +252,13 @@ def make_tensors(w: Workload, device="cpu", seed: Optional[int] = None,
     dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
 
     def draw(*shape):
-        x = torch.empty(shape, dtype=torch.float32, device=device)
-        x.normal_(generator=g)
-        return x.to(dt)
+        # drawn one layer at a time so the fp32 temporary stays small
+        out = torch.empty(shape, dtype=dt, device=device)
+        for l in range(shape[0]):
+            x = torch.empty(shape[1:], dtype=torch.float32, device=device)
+            x.normal_(generator=g)
+            out[l].copy_(x)
+        return out
 
     q = draw(w.L, w.B, w.H, w.T, w.D)
     k_cache = draw(w.L, w.B, w.H, S, w.D)

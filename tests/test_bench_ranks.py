@@ -1,0 +1,58 @@
+"""Host logic of bench.py's multi-rank runs (one replica per GPU, timing is
+the slowest rank's): checked with two gloo ranks on the CPU."""
+import os
+import socket
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out):
+    sys.path.insert(0, ROOT)
+    import torch.distributed as dist
+    import bench
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank,
+                            world_size=world)
+    try:
+        ms = 100.0 + 50.0 * rank                       # rank 1 is slower
+        slowest = bench.max_over_ranks(ms, dist, "cpu")
+        out[rank] = (slowest, bench.aggregate_rate(20, world, slowest))
+        dist.barrier()
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_take_the_slowest_time():
+    world, port = 2, _free_port()
+    ctx = mp.get_context("spawn")
+    with ctx.Manager() as m:
+        out = m.dict()
+        procs = [ctx.Process(target=_rank_main, args=(r, world, port, out)) for r in range(world)]
+        for p in procs:
+            p.start()
+        for p in procs:
+            p.join(120)
+            assert p.exitcode == 0
+        res = dict(out)
+    for r in range(world):
+        slowest, rate = res[r]
+        assert slowest == 150.0
+        assert rate == pytest.approx(2 * 20 / 0.150)
+
+
+def test_single_process_defaults():
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.dist_setup({}) == (1, 0, 0)
+    assert bench.dist_setup({"WORLD_SIZE": "4", "RANK": "2", "LOCAL_RANK": "2"}) == (4, 2, 2)
+    assert bench.max_over_ranks(3.5) == 3.5
+    assert bench.aggregate_rate(10, 1, 1000.0) == pytest.approx(10.0)

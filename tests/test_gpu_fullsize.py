@@ -1,0 +1,86 @@
+"""The fused verification step at the full workload sizes, in the launch
+configuration the benchmark times.  Inputs are drawn on the device; the oracle
+checks every index output in full and the attention outputs of sampled
+(layer, sequence, head) slices, including the first and last layer; compaction
+is checked row by row on the device against the tree rows the path names."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2405_18628_gb300 import ppd
+from paper_2405_18628_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+ATOL, RTOL_L2 = 5e-3, 1e-3
+
+
+def _row_checksums(x):
+    """Per (l,b,h,row) int64 sums of the raw bit patterns, one layer at a time."""
+    return torch.stack([x[l].view(torch.int16).to(torch.int64).sum(dim=-1)
+                        for l in range(x.shape[0])])
+
+
+@pytest.mark.parametrize("name", ["mobilellama", "vicuna7b", "vicuna13b",
+                                  "sweep_t16", "sweep_t32", "sweep_t64", "sweep_t128"])
+def test_full_size_step(cuda_device, name):
+    w = W.WORKLOADS[name]
+    need = 2 * w.L * w.B * w.H * (w.S_max + 2 * w.T) * w.D * 2
+    torch.cuda.empty_cache()                    # earlier cases' blocks back to the device
+    free, _ = torch.cuda.mem_get_info()
+    if need * 1.3 > free:
+        pytest.skip(f"{name} needs {need / 2**30:.0f} GiB")
+    s = W.make_step_inputs(w)
+    t = W.make_tensors(w, device=cuda_device)
+    before = {k: _row_checksums(t[k]) for k in ("k_cache", "v_cache")}
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(cuda_device)
+    bufs = ppd.StepBuffers(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max, device=cuda_device)
+    ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
+                        i32(s.prefix_len), i32(s.parent), i32(s.cand_tokens),
+                        torch.from_numpy(s.logits).to(cuda_device), bufs.out, bufs.argmax,
+                        bufs.accept_len, bufs.path, bufs.next_token, bufs.new_prefix_len,
+                        bufs.dev_status, bufs.workspace)
+    torch.cuda.synchronize()
+
+    # indices: in full
+    am = oracle.node_argmax(s.logits)
+    np.testing.assert_array_equal(bufs.argmax.cpu().numpy(), am)
+    np.testing.assert_array_equal(am, s.top)                   # the planted maxima
+    acc = oracle.accept_path(am, s.cand_tokens, s.parent, s.prefix_len, w.V, w.S_max)
+    for k in ("accept_len", "path", "next_token", "new_prefix_len"):
+        np.testing.assert_array_equal(getattr(bufs, k).cpu().numpy(), acc[k], err_msg=k)
+    assert (bufs.dev_status.cpu().numpy() == 0).all() and (acc["status"] == 0).all()
+
+    # compaction: accepted rows hold the named tree rows; every other row unchanged
+    for b in range(w.B):
+        n, P = int(acc["accept_len"][b]), int(s.prefix_len[b])
+        src = torch.from_numpy(acc["path"][b, :n].astype(np.int64)).to(cuda_device)
+        for k, kt in (("k_cache", "k_tree"), ("v_cache", "v_tree")):
+            got = t[k][:, b, :, P:P + n].view(torch.int16)
+            want = t[kt][:, b, :, :][:, :, src].view(torch.int16)
+            assert torch.equal(got, want), (k, b)
+    for k in ("k_cache", "v_cache"):
+        after = _row_checksums(t[k])
+        mask = torch.ones_like(after, dtype=torch.bool)
+        for b in range(w.B):
+            n, P = int(acc["accept_len"][b]), int(s.prefix_len[b])
+            mask[:, b, :, P:P + n] = False
+        assert torch.equal(after[mask], before[k][mask]), k
+
+    # attention: sampled slices, first and last layer included
+    rng = np.random.default_rng(w.seed)
+    picks = {(0, 0, 0), (w.L - 1, w.B - 1, w.H - 1)}
+    while len(picks) < 6:
+        picks.add((int(rng.integers(w.L)), int(rng.integers(w.B)), int(rng.integers(w.H))))
+    for (l, b, h) in sorted(picks):
+        sl = lambda x: x[l:l + 1, b:b + 1, h:h + 1].cpu()
+        P = int(s.prefix_len[b])
+        kc, vc = sl(t["k_cache"]), sl(t["v_cache"])
+        ref, _, _, st = oracle.tree_attention(sl(t["q"]), kc, vc, sl(t["k_tree"]), sl(t["v_tree"]),
+                                              s.prefix_len[b:b + 1], s.parent[b:b + 1])
+        got = bufs.out[l, b, h].double().cpu().numpy()
+        assert np.isfinite(got).all()
+        err = np.abs(got - ref[0]).max()
+        rel = np.linalg.norm(got - ref[0]) / np.linalg.norm(ref[0])
+        assert err <= ATOL and rel <= RTOL_L2, ((l, b, h), err, rel)
