@@ -50,9 +50,14 @@ struct AttnLayout {
     static constexpr uint32_t P_BYTES = P_GROUPS * GROUP_BYTES;
     static constexpr int OB = (TPMAX <= 64) ? 2 : 1;     // O accumulators in TMEM
     static constexpr int QS = (TPMAX <= 64) ? 2 : 1;     // Q buffers
-    static constexpr int PS = (TPMAX <= 64) ? 2 : 1;     // probability tiles
-    static constexpr int KS = 2;                          // K tile ring
-    static constexpr int VS = 2;                          // V tile ring
+    // With D = 128 and trees of <= 64 tokens a tile's probabilities fit exactly in
+    // its own K slot, free once S^T = K Q^T is done: no dedicated probability
+    // tiles, and the freed shared memory buys a third K and V stage.
+    static constexpr bool P_IN_K = (D == 128) && (TPMAX <= 64);
+    static constexpr int PS = P_IN_K ? 0 : ((TPMAX <= 64) ? 2 : 1);   // dedicated P tiles
+    static constexpr int PB = P_IN_K ? 2 : PS;            // P full/free barrier pairs
+    static constexpr int KS = P_IN_K ? 3 : 2;             // K tile ring
+    static constexpr int VS = P_IN_K ? 3 : 2;             // V tile ring
     static constexpr int NC_MAX = TPMAX / 2;              // query columns per warpgroup
     static constexpr int ANC_WORDS = TPMAX / 32;          // ancestor bitset words per node
 
@@ -71,8 +76,8 @@ struct AttnLayout {
     static constexpr int B_SFULL = B_VEMPTY + VS;
     static constexpr int B_SFREE = B_SFULL + 2;
     static constexpr int B_PFULL = B_SFREE + 2;
-    static constexpr int B_PFREE = B_PFULL + PS;
-    static constexpr int B_DRAIN = B_PFREE + PS;
+    static constexpr int B_PFREE = B_PFULL + PB;
+    static constexpr int B_DRAIN = B_PFREE + PB;
     static constexpr int NBAR = B_DRAIN + 1;
     static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
     static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
@@ -91,9 +96,18 @@ struct AttnLayout {
     static constexpr uint32_t TMEM_COLS = (2 + 2 * OB) * TPMAX <= 256 ? 256 : 512;
 
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
+    static_assert(!P_IN_K || P_BYTES <= TILE_BYTES, "probability tile fits in a K slot");
     static_assert((OFF_P | OFF_K | OFF_V) % 1024 == 0, "1024-byte aligned operand tiles");
     static_assert((2 + 2 * OB) * TPMAX <= 512, "TMEM budget");
 };
+
+// Byte offset (from the shared-memory base) of tile g's probability tile.
+template <class Lay>
+PPD_DEV uint32_t p_offset(int g)
+{
+    if (Lay::P_IN_K) return Lay::OFF_K + (uint32_t)(g % Lay::KS) * Lay::TILE_BYTES;
+    return Lay::OFF_P + (uint32_t)(g % (Lay::PS > 0 ? Lay::PS : 1)) * Lay::P_BYTES;
+}
 
 struct UnitInfo {
     int b, P, P_raw, n_pref, n_tiles;
@@ -237,7 +251,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         for (int i = 0; i < Lay::NBAR; ++i) {
             uint32_t count = 1;
             if ((i >= Lay::B_SFREE && i < Lay::B_SFREE + 2) ||
-                (i >= Lay::B_PFULL && i < Lay::B_PFULL + Lay::PS))
+                (i >= Lay::B_PFULL && i < Lay::B_PFULL + Lay::PB))
                 count = 8;
             mbar_init(bars + i, count);
         }
@@ -325,15 +339,15 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             const uint32_t sq = smem_addr(smem + Lay::OFF_Q);
             const uint32_t sk = smem_addr(smem + Lay::OFF_K);
             const uint32_t sv = smem_addr(smem + Lay::OFF_V);
-            const uint32_t sp = smem_addr(smem + Lay::OFF_P);
+            const uint32_t s0 = smem_addr(smem);
             // V^T as the A operand: M = D spans the tile's 64-column groups.  With
             // D = 64 both M halves read the same group (rows 64..127 of O^T repeat
             // rows 0..63 and are ignored).
             const uint32_t v_lbo = (D == 128) ? Lay::GROUP_BYTES : 0u;
 
             auto issue_pv = [&](int gp, bool first, uint32_t t_o) {
-                const int ps = gp % Lay::PS;
-                mbar_wait(bars + Lay::B_PFULL + ps, (gp / Lay::PS) & 1, abort_flag);
+                const int ps = gp % Lay::PB;
+                mbar_wait(bars + Lay::B_PFULL + ps, (gp / Lay::PB) & 1, abort_flag);
                 const int vs = gp % Lay::VS;
                 mbar_wait(bars + Lay::B_VFULL + vs, (gp / Lay::VS) & 1, abort_flag);
                 tc_fence_after();
@@ -342,13 +356,14 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     for (int kk = 0; kk < Lay::KT / 16; ++kk) {
                         const uint64_t a = make_smem_desc(sv + vs * Lay::TILE_BYTES + kk * 2048,
                                                           v_lbo, 1024);
-                        const uint64_t b = make_smem_desc(sp + ps * Lay::P_BYTES + kk * 2048,
+                        const uint64_t b = make_smem_desc(s0 + p_offset<Lay>(gp) + kk * 2048,
                                                           Lay::GROUP_BYTES, 1024);
                         umma_bf16(t_o, a, b, idesc_pv, (first && kk == 0) ? 0u : 1u);
                     }
                 }
                 umma_commit(bars + Lay::B_PFREE + ps);
                 umma_commit(bars + Lay::B_VEMPTY + vs);
+                if (Lay::P_IN_K) umma_commit(bars + Lay::B_KEMPTY + gp % Lay::KS);
             };
 
             int g = 0, k = 0;
@@ -374,7 +389,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         }
                     }
                     umma_commit(bars + Lay::B_SFULL + sb);
-                    umma_commit(bars + Lay::B_KEMPTY + ks);
+                    if (!Lay::P_IN_K) umma_commit(bars + Lay::B_KEMPTY + ks);
                     if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
                     if (j >= 1) issue_pv(g - 1, j == 1, t_o);
                 }
@@ -393,7 +408,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         const int q0 = wg * NC;
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
         // this thread's row of the probability tile (128-byte swizzled atoms)
-        const uint32_t p_row = smem_addr(smem + Lay::OFF_P) + (uint32_t)(t >> 3) * 1024u +
+        const uint32_t p_row = smem_addr(smem) + (uint32_t)(t >> 3) * 1024u +
                                (uint32_t)(t & 7) * 128u;
         const uint32_t p_swz = (uint32_t)(t & 7);
         const float sl2 = p.scale_log2;
@@ -407,88 +422,175 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         uint64_t dbits = 0;   // bit c: key t (tree node t) is visible to query q0 + c
         int cur_b = -1;
         int g = 0;
+        int cur_k = 0;        // this CTA's unit counter (selects the O accumulator)
         // a finished unit whose output still sits in TMEM
         bool pend = false;
         int pend_u = 0, pend_ob = 0, pend_g = 0;
 
-        // Probabilities of query columns [c0, c0+16) (and [c0+16, c0+32) when `two`)
-        // of this thread's key row with the current running maxima, exponents
+        // Probabilities of the 16 query columns [cb, cb+16) of this thread's key row
+        // from its raw scores r, against the current running maxima, exponents
         // clamped at 64 so nothing overflows before a rescale.  STORE: split into
         // bf16 hi + lo, store into probability tile `pbuf` (byte offset) and add to
-        // lacc.  UNDO: subtract the same values from lacc again (a bit-identical
-        // recomputation).  `maxd` collects the largest unclamped exponent.
-        auto p_group = [&](auto kind_c, auto undo_c, uint32_t t_s, int c0, bool two, bool row_ok,
-                           uint32_t pbuf, float &maxd) {
+        // lacc.  UNDO: subtract the same values from lacc again (bit-identical to
+        // an earlier STORE with the same maxima).  `maxd` collects the largest
+        // unclamped exponent.  WAIT: r is the target of a TMEM load still in flight.
+        auto emit_half = [&](auto kind_c, auto undo_c, auto wait_c, const uint32_t (&r)[16], int cb,
+                             uint32_t bits16, bool row_ok, uint32_t pbuf, float &maxd) {
             constexpr int KIND = decltype(kind_c)::value;
             constexpr bool UNDO = decltype(undo_c)::value != 0;
+            const float4 *m4 = reinterpret_cast<const float4 *>(m2 + q0 + cb);
+            float m[16];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float4 v = m4[k];
+                m[4 * k] = v.x;
+                m[4 * k + 1] = v.y;
+                m[4 * k + 2] = v.z;
+                m[4 * k + 3] = v.w;
+            }
+            if (decltype(wait_c)::value) tmem_wait_ld();
+            float pv[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                float d = fmaf(__uint_as_float(r[e]), sl2, -m[e]);
+                if (KIND == kMaskRows) d = row_ok ? d : -INFINITY;
+                if (KIND == kMaskTree) d = ((bits16 >> e) & 1u) ? d : -INFINITY;
+                maxd = fmaxf(maxd, d);
+                pv[e] = ex2(fminf(d, 64.f));
+                if (UNDO) lacc[cb + e] -= pv[e];
+                else lacc[cb + e] += pv[e];
+            }
+            if (!UNDO) {
+                uint32_t hw[8], lw[8];
+#pragma unroll
+                for (int e = 0; e < 16; e += 2) {
+                    const uint32_t h0 = __float_as_uint(pv[e]) & 0xFFFF0000u;
+                    const uint32_t h1 = __float_as_uint(pv[e + 1]) & 0xFFFF0000u;
+                    hw[e >> 1] = __byte_perm(h0, h1, 0x7632);
+                    const __nv_bfloat162 lo = __floats2bfloat162_rn(pv[e] - __uint_as_float(h0),
+                                                                    pv[e + 1] - __uint_as_float(h1));
+                    lw[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
+                }
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    const int ch = q0 + cb + half * 8;   // hi column
+                    const int cl = T_pad + ch;            // lo column
+                    const uint32_t ah = p_row + pbuf + (uint32_t)(ch >> 6) * Lay::GROUP_BYTES +
+                                        ((((uint32_t)(ch & 63) >> 3) ^ p_swz) << 4);
+                    const uint32_t al = p_row + pbuf + (uint32_t)(cl >> 6) * Lay::GROUP_BYTES +
+                                        ((((uint32_t)(cl & 63) >> 3) ^ p_swz) << 4);
+                    st_shared_v4(ah, hw[half * 4], hw[half * 4 + 1], hw[half * 4 + 2], hw[half * 4 + 3]);
+                    st_shared_v4(al, lw[half * 4], lw[half * 4 + 1], lw[half * 4 + 2], lw[half * 4 + 3]);
+                }
+            }
+        };
+        using store_t = kind_t<0>;
+        using undo_t = kind_t<1>;
+        using wait_t = kind_t<1>;
+        using nowait_t = kind_t<0>;
+
+        // Optimistic pass over query columns [c0, c0+16) (and [c0+16, c0+32) when
+        // `two`): scores straight from TMEM against the current maxima.
+        auto p_group = [&](auto kind_c, uint32_t t_s, int c0, bool two, bool row_ok, uint32_t pbuf,
+                           float &maxd) {
             const uint32_t bits = (uint32_t)(dbits >> c0);
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 if (h == 0 || two) {
-                    const int cb = c0 + h * 16;
                     uint32_t r[16];
-                    tmem_ld16(t_s + cb, r);
-                    const float4 *m4 = reinterpret_cast<const float4 *>(m2 + q0 + cb);
-                    float m[16];
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const float4 v = m4[k];
-                        m[4 * k] = v.x;
-                        m[4 * k + 1] = v.y;
-                        m[4 * k + 2] = v.z;
-                        m[4 * k + 3] = v.w;
-                    }
-                    float pv[16];
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        float d = fmaf(__uint_as_float(r[e]), sl2, -m[e]);
-                        if (KIND == kMaskRows) d = row_ok ? d : -INFINITY;
-                        if (KIND == kMaskTree) d = ((bits >> (h * 16 + e)) & 1u) ? d : -INFINITY;
-                        maxd = fmaxf(maxd, d);
-                        pv[e] = ex2(fminf(d, 64.f));
-                        if (UNDO) lacc[cb + e] -= pv[e];
-                        else lacc[cb + e] += pv[e];
-                    }
-                    if (!UNDO) {
-                        uint32_t hw[8], lw[8];
-#pragma unroll
-                        for (int e = 0; e < 16; e += 2) {
-                            const uint32_t h0 = __float_as_uint(pv[e]) & 0xFFFF0000u;
-                            const uint32_t h1 = __float_as_uint(pv[e + 1]) & 0xFFFF0000u;
-                            hw[e >> 1] = __byte_perm(h0, h1, 0x7632);
-                            const __nv_bfloat162 lo = __floats2bfloat162_rn(pv[e] - __uint_as_float(h0),
-                                                                            pv[e + 1] - __uint_as_float(h1));
-                            lw[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
-                        }
-#pragma unroll
-                        for (int half = 0; half < 2; ++half) {
-                            const int ch = q0 + cb + half * 8;   // hi column
-                            const int cl = T_pad + ch;            // lo column
-                            const uint32_t ah = p_row + pbuf + (uint32_t)(ch >> 6) * Lay::GROUP_BYTES +
-                                                ((((uint32_t)(ch & 63) >> 3) ^ p_swz) << 4);
-                            const uint32_t al = p_row + pbuf + (uint32_t)(cl >> 6) * Lay::GROUP_BYTES +
-                                                ((((uint32_t)(cl & 63) >> 3) ^ p_swz) << 4);
-                            st_shared_v4(ah, hw[half * 4], hw[half * 4 + 1], hw[half * 4 + 2], hw[half * 4 + 3]);
-                            st_shared_v4(al, lw[half * 4], lw[half * 4 + 1], lw[half * 4 + 2], lw[half * 4 + 3]);
-                        }
-                    }
+                    tmem_ld16(t_s + c0 + h * 16, r);
+                    emit_half(kind_c, store_t{}, wait_t{}, r, c0 + h * 16, bits >> (h * 16), row_ok,
+                              pbuf, maxd);
                 }
             }
         };
-        auto run_group = [&](auto undo_c, int kind, uint32_t t_s, int c0, bool two, bool row_ok,
-                             uint32_t pbuf, float &maxd) {
-            if (kind == kMaskNone) p_group(kind_t<kMaskNone>{}, undo_c, t_s, c0, two, row_ok, pbuf, maxd);
-            else if (kind == kMaskRows) p_group(kind_t<kMaskRows>{}, undo_c, t_s, c0, two, row_ok, pbuf, maxd);
-            else p_group(kind_t<kMaskTree>{}, undo_c, t_s, c0, two, row_ok, pbuf, maxd);
+
+        // Exact pass over the same columns, on a unit's first tile or after a score
+        // jumped past its maximum: the scores are loaded once and kept in registers;
+        // the optimistic contributions are taken back out of the row sums (later
+        // tiles); every column's maximum over the 128 key rows is a warp max
+        // (redux) combined across the four warps; O and the row sums are rescaled
+        // (later tiles); the probabilities are recomputed.
+        auto exact_group = [&](auto kind_c, uint32_t t_s, int c0, bool two, bool row_ok,
+                               uint32_t pbuf, bool later, bool &o_ready) {
+            constexpr int KIND = decltype(kind_c)::value;
+            uint32_t r0[16], r1[16];
+            tmem_ld16(t_s + c0, r0);
+            if (two) tmem_ld16(t_s + c0 + 16, r1);
+            tmem_wait_ld();
+            const uint32_t bits = (uint32_t)(dbits >> c0);
+            if (later) {
+                float unused = 0.f;
+                emit_half(kind_c, undo_t{}, nowait_t{}, r0, c0, bits, row_ok, pbuf, unused);
+                if (two) emit_half(kind_c, undo_t{}, nowait_t{}, r1, c0 + 16, bits >> 16, row_ok, pbuf, unused);
+            }
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                if (e < 16 || two) {
+                    const float sv = __uint_as_float(e < 16 ? r0[e] : r1[e - 16]);
+                    const bool vis = KIND == kMaskNone ? true
+                                     : KIND == kMaskRows ? row_ok
+                                                         : ((bits >> e) & 1u) != 0;
+                    const float mx = warp_max(vis ? sv * sl2 : -INFINITY);
+                    if (lane == e) red_wg[wq * Lay::NC_MAX + c0 + e] = mx;
+                }
+            }
+            named_bar_sync(1 + wg, 128);
+            const int gw = two ? 32 : 16;
+            if (t < gw) {
+                const int c = c0 + t;
+                const float tm = fmaxf(fmaxf(red_wg[c], red_wg[Lay::NC_MAX + c]),
+                                       fmaxf(red_wg[2 * Lay::NC_MAX + c], red_wg[3 * Lay::NC_MAX + c]));
+                const float old = m2[q0 + c];
+                const float nw = fmaxf(old, tm);
+                m2[q0 + c] = nw;
+                red_wg[c] = (nw == old) ? 1.f : ex2(old - nw);   // alpha
+            }
+            named_bar_sync(1 + wg, 128);
+            if (later) {
+                // rescale the accumulated output columns and row sums; the PV product
+                // of the previous tile must have landed first
+                if (!o_ready) {
+                    const int pp = (g - 1) % Lay::PB;
+                    mbar_wait(bars + Lay::B_PFREE + pp, ((g - 1) / Lay::PB) & 1, abort_flag);
+                    o_ready = true;
+                }
+                tc_fence_after();
+                const uint32_t t_o = tmem_base + lane_off + Lay::T_O +
+                                     (uint32_t)(cur_k % Lay::OB) * 2 * TPMAX;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    if (h == 0 || two) {
+                        const int cb = c0 + h * 16;
+                        float a[16];
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) a[e] = red_wg[cb + e];
+#pragma unroll
+                        for (int part = 0; part < 2; ++part) {
+                            const uint32_t col = t_o + (part ? T_pad : 0) + q0 + cb;
+                            uint32_t rr[16];
+                            tmem_ld16(col, rr);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int e = 0; e < 16; ++e)
+                                rr[e] = __float_as_uint(__uint_as_float(rr[e]) * a[e]);
+                            tmem_st16(col, rr);
+                        }
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) lacc[cb + e] *= a[e];
+                    }
+                }
+                tmem_wait_st();
+            }
+            float maxd = -INFINITY;
+            emit_half(kind_c, store_t{}, nowait_t{}, r0, c0, bits, row_ok, pbuf, maxd);
+            if (two) emit_half(kind_c, store_t{}, nowait_t{}, r1, c0 + 16, bits >> 16, row_ok, pbuf, maxd);
         };
-        using store_t = kind_t<0>;
-        using undo_t = kind_t<1>;
 
         // Output of a finished unit: O (hi + lo) from its TMEM accumulator times the
         // reciprocal row sums, one head-dim element per thread, queries in order.
         auto read_back = [&](int u_out, int ob, int g_last) {
-            mbar_wait(bars + Lay::B_PFREE + g_last % Lay::PS, (g_last / Lay::PS) & 1, abort_flag);
+            mbar_wait(bars + Lay::B_PFREE + g_last % Lay::PB, (g_last / Lay::PB) & 1, abort_flag);
             tc_fence_after();
             if (wq * 32 < D) {
                 const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * 2 * TPMAX;
@@ -517,6 +619,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         int k = 0;
         for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
             const UnitInfo ui = unit_info(p, u);
+            cur_k = k;
             const int ob = k % Lay::OB;
             const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * 2 * TPMAX;
             if (ui.b != cur_b) {
@@ -572,12 +675,15 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                 mbar_wait(bars + Lay::B_SFULL + sb, (g >> 1) & 1, abort_flag);
                 tc_fence_after();
                 const uint32_t t_s = tmem_base + lane_off + Lay::T_S + sb * TPMAX + q0;
-                const int ps = g % Lay::PS;
-                const uint32_t pbuf = (uint32_t)ps * Lay::P_BYTES;
-                // probability tile ps is free once the PV product of tile g - PS is done
-                if (g >= Lay::PS)
-                    mbar_wait(bars + Lay::B_PFREE + ps, ((g / Lay::PS) - 1) & 1, abort_flag);
-                bool o_ready = (Lay::PS == 1);   // PV of tile g-1 known to be complete
+                const int ps = g % Lay::PB;
+                const uint32_t pbuf = p_offset<Lay>(g);
+                // a dedicated probability tile is free once the PV product of tile
+                // g - PS is done; a K slot is free as soon as S(g) is (waited above)
+                if constexpr (!Lay::P_IN_K) {
+                    if (g >= Lay::PS)
+                        mbar_wait(bars + Lay::B_PFREE + ps, ((g / Lay::PS) - 1) & 1, abort_flag);
+                }
+                bool o_ready = (Lay::PB == 1);   // PV of tile g-1 known to be complete
 
                 // Column groups of up to 32 queries, done optimistically with the
                 // current running maxima; on a unit's first tile, or when a score
@@ -591,86 +697,19 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         bool exact;
                         if (j > 0) {
                             float maxd = -INFINITY;
-                            run_group(store_t{}, kind, t_s, gc0, two, row_ok, pbuf, maxd);
+                            if (kind == kMaskNone) p_group(kind_t<kMaskNone>{}, t_s, gc0, two, row_ok, pbuf, maxd);
+                            else if (kind == kMaskRows) p_group(kind_t<kMaskRows>{}, t_s, gc0, two, row_ok, pbuf, maxd);
+                            else p_group(kind_t<kMaskTree>{}, t_s, gc0, two, row_ok, pbuf, maxd);
                             exact = named_bar_or(1 + wg, 128, maxd > 16.f);
                         } else {
                             named_bar_sync(1 + wg, 128);   // earlier readers of red_wg are done
                             exact = true;
                         }
                         if (exact) {
-                            if (j > 0) {
-                                // take the optimistic contributions back out of the row sums
-                                float unused = 0.f;
-                                run_group(undo_t{}, kind, t_s, gc0, two, row_ok, pbuf, unused);
-                            }
-#pragma unroll
-                            for (int h = 0; h < 2; ++h) {
-                                if (h == 0 || two) {
-                                    const int c0 = gc0 + h * 16;
-                                    uint32_t r[16];
-                                    float v[16];
-                                    tmem_ld16(t_s + c0, r);
-                                    tmem_wait_ld();
-                                    const uint32_t bits = (uint32_t)(dbits >> c0);
-#pragma unroll
-                                    for (int e = 0; e < 16; ++e) {
-                                        const bool vis = kind == kMaskNone ? true
-                                                         : kind == kMaskRows ? row_ok
-                                                                             : ((bits >> e) & 1u) != 0;
-                                        v[e] = vis ? __uint_as_float(r[e]) * sl2 : -INFINITY;
-                                    }
-                                    const float mx = warp_transpose_reduce16(v, lane, OpMax());
-                                    if (!(lane & 1)) red_wg[wq * Lay::NC_MAX + c0 + (lane >> 1)] = mx;
-                                }
-                            }
-                            named_bar_sync(1 + wg, 128);
-                            const int gw = two ? 32 : 16;
-                            if (t < gw) {
-                                const int c = gc0 + t;
-                                const float tm = fmaxf(fmaxf(red_wg[c], red_wg[Lay::NC_MAX + c]),
-                                                       fmaxf(red_wg[2 * Lay::NC_MAX + c],
-                                                             red_wg[3 * Lay::NC_MAX + c]));
-                                const float old = m2[q0 + c];
-                                const float nw = fmaxf(old, tm);
-                                m2[q0 + c] = nw;
-                                red_wg[c] = (nw == old) ? 1.f : ex2(old - nw);   // alpha
-                            }
-                            named_bar_sync(1 + wg, 128);
-                            if (j > 0) {
-                                // rescale the accumulated output columns and row sums; the
-                                // PV product of the previous tile must have landed first
-                                if (!o_ready) {
-                                    const int pp = (g - 1) % Lay::PS;
-                                    mbar_wait(bars + Lay::B_PFREE + pp, ((g - 1) / Lay::PS) & 1, abort_flag);
-                                    o_ready = true;
-                                }
-                                tc_fence_after();
-#pragma unroll
-                                for (int h = 0; h < 2; ++h) {
-                                    if (h == 0 || two) {
-                                        const int c0 = gc0 + h * 16;
-                                        float a[16];
-#pragma unroll
-                                        for (int e = 0; e < 16; ++e) a[e] = red_wg[c0 + e];
-#pragma unroll
-                                        for (int part = 0; part < 2; ++part) {
-                                            const uint32_t col = t_o + (part ? T_pad : 0) + q0 + c0;
-                                            uint32_t rr[16];
-                                            tmem_ld16(col, rr);
-                                            tmem_wait_ld();
-#pragma unroll
-                                            for (int e = 0; e < 16; ++e)
-                                                rr[e] = __float_as_uint(__uint_as_float(rr[e]) * a[e]);
-                                            tmem_st16(col, rr);
-                                        }
-#pragma unroll
-                                        for (int e = 0; e < 16; ++e) lacc[c0 + e] *= a[e];
-                                    }
-                                }
-                                tmem_wait_st();
-                            }
-                            float maxd = -INFINITY;
-                            run_group(store_t{}, kind, t_s, gc0, two, row_ok, pbuf, maxd);
+                            const bool later = j > 0;
+                            if (kind == kMaskNone) exact_group(kind_t<kMaskNone>{}, t_s, gc0, two, row_ok, pbuf, later, o_ready);
+                            else if (kind == kMaskRows) exact_group(kind_t<kMaskRows>{}, t_s, gc0, two, row_ok, pbuf, later, o_ready);
+                            else exact_group(kind_t<kMaskTree>{}, t_s, gc0, two, row_ok, pbuf, later, o_ready);
                         }
                     }
                 }

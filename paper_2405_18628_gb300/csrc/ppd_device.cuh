@@ -309,6 +309,14 @@ PPD_DEV float rcp(float x)
     return y;
 }
 
+// Maximum of v over the 32 lanes of a warp (every lane gets it).
+PPD_DEV float warp_max(float v)
+{
+    float r;
+    asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+    return r;
+}
+
 // Reduce 16 per-lane columns over the 32 lanes of a warp.  On return lane L
 // holds the reduction of column (L >> 1) over all lanes (lanes 2c and 2c+1
 // agree).  16 shuffles for 16 columns.
