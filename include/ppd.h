@@ -194,6 +194,10 @@ const char *ppd_status_string(ppd_status s);
  *   mode 1: d[128][N] = a[128][128]^T * b[128][N]   (a given [K][M], b given
  *           [K][N]: both operands M/N-major; b is written by threads)
  *   mode 2: as mode 1 with a given [K][64]; rows 64..127 of d repeat rows 0..63
+ *   mode 3: d[128][N] = (a_hi + a_lo)[128][128] * b[128][N], a given [128][256]
+ *           (columns 0..127 a_hi, 128..255 a_lo), held in tensor memory in the
+ *           layout of the probability tile of the 65..128-token attention
+ *           kernel and multiplied as two products; N <= 128
  * N in {16, 32, ..., 256}; a, b bf16 device pointers; d fp32 [128][N].
  */
 ppd_status ppd_selftest_umma(const void *a, const void *b, float *d, int mode, int N,

@@ -149,8 +149,11 @@ ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, cons
 {
     const int T_pad = (T + 31) & ~31;
     const uint64_t lbh = (uint64_t)L * B * H;
+    // trees of more than 64 tokens run the row-layout kernel, which reads Q in
+    // boxes of 128 rows (rows past T arrive as zeros)
+    const uint32_t q_box = T_pad > 64 ? 128u : (uint32_t)T_pad;
     AttnMaps m;
-    if (!encode_3d(&m.q, q, D, T, lbh, T_pad) || !encode_3d(&m.kc, kc, D, S_max, lbh, 128) ||
+    if (!encode_3d(&m.q, q, D, T, lbh, q_box) || !encode_3d(&m.kc, kc, D, S_max, lbh, 128) ||
         !encode_3d(&m.vc, vc, D, S_max, lbh, 128) || !encode_3d(&m.kt, kt, D, T, lbh, 128) ||
         !encode_3d(&m.vt, vt, D, T, lbh, 128))
         return PPD_ERR_CUDA;
@@ -389,19 +392,23 @@ ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
 
 ppd_status ppd_selftest_umma(const void *a, const void *b, float *d, int mode, int N, void *stream)
 {
-    if (!a || !b || !d || mode < 0 || mode > 2 || N < 16 || N > 256 || N % 16 != 0)
+    if (!a || !b || !d || mode < 0 || mode > 3 || N < 16 || N > 256 || N % 16 != 0)
         return PPD_ERR_INVALID_ARG;
+    if (mode == 3 && N > 128) return PPD_ERR_INVALID_ARG;
     if (mode != 0 && N % 8 != 0) return PPD_ERR_INVALID_ARG;
     if (!aligned(a, 16) || !aligned(b, 16) || !aligned(d, 4)) return PPD_ERR_INVALID_ARG;
     CUtensorMap ma, mb;
+    std::memset(&ma, 0, sizeof ma);
     std::memset(&mb, 0, sizeof mb);
-    if (mode == 0) {
+    if (mode == 3) {
+        // A is written to TMEM by threads, B to shared memory: no tensor maps
+    } else if (mode == 0) {
         if (!encode_2d(&ma, a, 128, 128, 128) || !encode_2d(&mb, b, 128, N, N)) return PPD_ERR_CUDA;
     } else {
         if (!encode_2d(&ma, a, mode == 2 ? 64 : 128, 128, 128)) return PPD_ERR_CUDA;
         mb = ma;
     }
-    return cuda_status(ppd::launch_selftest_umma(ma, mb, b, d, mode, N, static_cast<cudaStream_t>(stream)));
+    return cuda_status(ppd::launch_selftest_umma(ma, mb, a, b, d, mode, N, static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"

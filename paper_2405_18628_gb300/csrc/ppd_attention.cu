@@ -27,9 +27,7 @@
 // trees of up to 64 tokens O is double-buffered in TMEM and a unit's output
 // is read back only after the next unit's first tile, so the stream of tiles
 // never waits for a unit's last PV product.
-#include "ppd_accept.cuh"
-#include "ppd_device.cuh"
-#include "ppd_kernels.h"
+#include "ppd_attention_common.cuh"
 
 #include <cmath>
 #include <type_traits>
@@ -109,113 +107,6 @@ PPD_DEV uint32_t p_offset(int g)
     return Lay::OFF_P + (uint32_t)(g % (Lay::PS > 0 ? Lay::PS : 1)) * Lay::P_BYTES;
 }
 
-struct UnitInfo {
-    int b, P, P_raw, n_pref, n_tiles;
-};
-
-PPD_DEV UnitInfo unit_info(const AttnParams &p, int u)
-{
-    UnitInfo ui;
-    ui.b = (u / p.H) % p.B;
-    ui.P_raw = __ldg(p.prefix_len + ui.b);
-    ui.P = min(max(ui.P_raw, 0), p.S_max);
-    ui.n_pref = (ui.P + 127) >> 7;
-    ui.n_tiles = ui.n_pref + 1;
-    return ui;
-}
-
-PPD_DEV void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
-{
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
-                 "r"(d)
-                 : "memory");
-}
-
-// Time-bounded wait that ignores the abort flag (used only to drain copies
-// still in flight after an abort, before the CTA exits).
-PPD_DEV void mbar_wait_drain(uint64_t *bar, uint32_t parity)
-{
-    const uint32_t a = smem_addr(bar);
-    const uint64_t t0 = global_timer();
-    while (!mbar_try_wait(a, parity))
-        if (global_timer() - t0 > kWaitLimitNs) return;
-}
-
-template <int K>
-using kind_t = std::integral_constant<int, K>;
-
-// Mask kinds of a tile: every key visible (a full prefix tile), keys t < n_valid
-// visible (the last, partial prefix tile), or the tree-ancestor mask.
-enum : int { kMaskNone = 0, kMaskRows = 1, kMaskTree = 2 };
-
-// Side work of the fused verification step, done by one extra warp of every CTA
-// while the other warps stream attention.  Once the preceding argmax grid has
-// completed (griddepcontrol.wait), for every sequence b this CTA touches -- or
-// is designated to report (b mod grid) -- the warp combines the node argmax
-// from the partial maxima, decides acceptance, writes the sequence's outputs
-// if designated, and copies the accepted tree K/V rows of this CTA's own
-// (layer, sequence, head) slices into the cache.  Attention only reads cache
-// rows below each prefix, so the copies never race with it.  Scratch (parent
-// copies, top-1 tokens, path) lives in a per-CTA slice of the workspace.
-PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
-{
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    const FusedStep &f = p.fs;
-    const int T = p.T, B = p.B, S = f.splits;
-    int *s_par = f.scratch + (size_t)blockIdx.x * kSideScratchInts;
-    int *top = s_par + 128;
-    int *path = top + 128;
-    const int chunks = f.row_bytes >> 4;
-    for (int b = 0; b < B; ++b) {
-        const bool designated = (b % (int)gridDim.x) == (int)blockIdx.x;
-        bool has_unit = false;
-        for (int u = blockIdx.x; u < p.n_units && !has_unit; u += gridDim.x)
-            has_unit = ((u / p.H) % B) == b;
-        if (!designated && !has_unit) continue;
-        for (int r = lane; r < T; r += 32) {
-            const size_t base = ((size_t)b * T + r) * S;
-            float bv = __ldcg(f.part_val + base);
-            int bi = __ldcg(f.part_idx + base);
-#pragma unroll 8
-            for (int k = 1; k < S; ++k) consider(__ldcg(f.part_val + base + k), __ldcg(f.part_idx + base + k), bv, bi);
-            top[r] = bi;
-            if (designated) f.argmax_out[(size_t)b * T + r] = bi;
-        }
-        __syncwarp();
-        const AcceptResult res =
-            accept_warp([&](int n) { return top[n]; }, p.parent + (size_t)b * T,
-                        f.cand_tokens + (size_t)b * T, __ldg(p.prefix_len + b), T, f.V, p.S_max,
-                        lane, s_par, path);
-        if (designated) {
-            for (int i = lane; i < T; i += 32) f.path[(size_t)b * T + i] = path[i];
-            if (lane == 0) {
-                f.accept_len[b] = res.n_acc;
-                f.next_token[b] = res.next_token;
-                f.new_prefix_len[b] = res.new_prefix_len;
-                atomicMax(f.status + b, res.status);
-            }
-        }
-        if (has_unit && res.n_acc > 0) {
-            // cache rows [P_b, P_b + n_acc) <- the accepted tree rows
-            const int P = __ldg(p.prefix_len + b);
-            const int n = res.n_acc;
-            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
-                if (((u / p.H) % B) != b) continue;
-                for (int w = lane; w < n * chunks; w += 32) {
-                    const int j = w / chunks, c = w - j * chunks;
-                    const int src = path[j];
-                    const size_t so = ((size_t)u * T + src) * f.row_bytes + (size_t)c * 16;
-                    const size_t dof = ((size_t)u * p.S_max + P + j) * f.row_bytes + (size_t)c * 16;
-                    const uint4 kx = __ldg(reinterpret_cast<const uint4 *>(f.k_tree + so));
-                    const uint4 vx = __ldg(reinterpret_cast<const uint4 *>(f.v_tree + so));
-                    *reinterpret_cast<uint4 *>(f.k_cache + dof) = kx;
-                    *reinterpret_cast<uint4 *>(f.v_cache + dof) = vx;
-                }
-            }
-        }
-        __syncwarp();
-    }
-}
 
 template <int D, int TPMAX>
 __global__ void __launch_bounds__(352, 1)
@@ -825,12 +716,9 @@ static cudaError_t launch_tree_attention_t(const AttnMaps &m, const AttnParams &
 cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
                                   bool programmatic, cudaStream_t stream)
 {
-    if (D == 128) {
-        if (p.T_pad <= 64) return launch_tree_attention_t<128, 64>(m, p, num_sms, programmatic, stream);
-        return launch_tree_attention_t<128, 128>(m, p, num_sms, programmatic, stream);
-    }
-    if (p.T_pad <= 64) return launch_tree_attention_t<64, 64>(m, p, num_sms, programmatic, stream);
-    return launch_tree_attention_t<64, 128>(m, p, num_sms, programmatic, stream);
+    if (p.T_pad > 64) return launch_tree_attention_rows(m, p, D, num_sms, programmatic, stream);
+    if (D == 128) return launch_tree_attention_t<128, 64>(m, p, num_sms, programmatic, stream);
+    return launch_tree_attention_t<64, 64>(m, p, num_sms, programmatic, stream);
 }
 
 }  // namespace ppd

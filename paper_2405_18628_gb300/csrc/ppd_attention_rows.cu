@@ -1,0 +1,528 @@
+// ppd_attention_rows.cu -- tree-masked attention of the PPD verification step
+// for trees of 65..128 tokens on sm_103a (paper Section 3 step (1): tree
+// attention over the candidate tree; Section 4.1: every tree token attends to
+// the cached prefix, its tree ancestors and itself).
+//
+// With more than 64 tree tokens the queries fill the tensor core's M side, so
+// this kernel keeps one query per TMEM lane (queries zero-padded to 128):
+//
+//   S  = Q * K_tile^T          tcgen05.mma, M = 128 queries, N = 128 keys, K = D
+//   P  = exp2(S*scale*log2e - m)   two softmax warps per 32 query rows, each
+//                              thread owning one query row and 64 of the 128
+//                              keys; P is split into bf16 hi + lo and written
+//                              back to TMEM over the scores it came from
+//   O += P_hi * V + P_lo * V   tcgen05.mma with A read from TMEM, M = 128
+//                              queries, N = D, two products per 16 keys
+//
+// A row's running maximum and row sum are registers of its two threads; they
+// exchange partial maxima through shared memory only on the exact path (a
+// unit's first tile, or a score more than 2^16 above the running maximum --
+// decided per tile by a vote over the softmax warps) and partial sums at the
+// end of a unit.  The tree mask is a 64-bit ancestor bitset per thread, built
+// from the parent array in registers.  Warp roles, the unit walk, the
+// double-buffered O with deferred readback and the fused step's side warp are
+// those of the kernel for trees of up to 64 tokens (ppd_attention.cu).
+#include "ppd_attention_common.cuh"
+
+#include <cmath>
+
+namespace ppd {
+
+template <int D_>
+struct RowsLayout {
+    static constexpr int D = D_;
+    static constexpr int KT = 128;                         // keys per tile
+    static constexpr int M = 128;                          // query rows per unit (zero-padded)
+    static constexpr int DCH = D / 64;                     // 64-column groups along D
+    static constexpr uint32_t GROUP_BYTES = 128 * 128;     // 128 rows of 64 bf16
+    static constexpr uint32_t TILE_BYTES = KT * D * 2;
+    static constexpr uint32_t Q_BYTES = M * D * 2;
+    static constexpr int QS = 2;                           // Q buffers
+    static constexpr int KS = (D == 64) ? 4 : 2;           // K tile ring
+    static constexpr int VS = (D == 64) ? 4 : 3;           // V tile ring
+
+    static constexpr uint32_t OFF_Q = 0;
+    static constexpr uint32_t OFF_K = OFF_Q + QS * Q_BYTES;
+    static constexpr uint32_t OFF_V = OFF_K + KS * TILE_BYTES;
+    static constexpr uint32_t OFF_BAR = OFF_V + VS * TILE_BYTES;
+    static constexpr int B_QFULL = 0;
+    static constexpr int B_QEMPTY = B_QFULL + QS;
+    static constexpr int B_KFULL = B_QEMPTY + QS;
+    static constexpr int B_KEMPTY = B_KFULL + KS;
+    static constexpr int B_VFULL = B_KEMPTY + KS;
+    static constexpr int B_VEMPTY = B_VFULL + VS;
+    static constexpr int B_SFULL = B_VEMPTY + VS;   // [2] scores of tile g in TMEM
+    static constexpr int B_PFULL = B_SFULL + 2;     // [2] probabilities of tile g in TMEM (8 warps)
+    static constexpr int B_PDONE = B_PFULL + 2;     // [2] PV product of tile g complete
+    static constexpr int B_DRAIN = B_PDONE + 2;
+    static constexpr int NBAR = B_DRAIN + 1;
+    static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
+    static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
+    static constexpr uint32_t OFF_XM = (OFF_ABORT + 4 + 15) & ~15u;   // [2][M] partial row maxima
+    static constexpr uint32_t OFF_XL = OFF_XM + 2 * M * 4;            // [2][M] partial row sums
+    static constexpr uint32_t SMEM_BYTES = OFF_XL + 2 * M * 4;
+    // TMEM columns: S0 | S1 (128 each; P is written over S) | O0 | O1 (D each)
+    static constexpr uint32_t T_S = 0, T_O = 256, O_STRIDE = 128, TMEM_COLS = 512;
+
+    static_assert(SMEM_BYTES <= 232448, "shared memory budget");
+    static_assert((OFF_K | OFF_V | Q_BYTES) % 1024 == 0, "1024-byte aligned operand tiles");
+};
+
+template <int D>
+__global__ void __launch_bounds__(352, 1)
+tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
+                           const __grid_constant__ CUtensorMap map_kc,
+                           const __grid_constant__ CUtensorMap map_vc,
+                           const __grid_constant__ CUtensorMap map_kt,
+                           const __grid_constant__ CUtensorMap map_vt, const AttnParams p)
+{
+    using Lay = RowsLayout<D>;
+    extern __shared__ __align__(1024) uint8_t smem[];
+    if (smem_addr(smem) & 1023u) {
+        if (threadIdx.x == 0 && p.dev_status)
+            for (int b = 0; b < p.B; ++b) p.dev_status[b] = kErrUnsupported;
+        return;
+    }
+
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + Lay::OFF_BAR);
+    uint32_t *tmem_ptr = reinterpret_cast<uint32_t *>(smem + Lay::OFF_TMEMPTR);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + Lay::OFF_ABORT);
+    float *xm = reinterpret_cast<float *>(smem + Lay::OFF_XM);
+    float *xl = reinterpret_cast<float *>(smem + Lay::OFF_XL);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int T = p.T;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < Lay::NBAR; ++i)
+            mbar_init(bars + i, (i >= Lay::B_PFULL && i < Lay::B_PFULL + 2) ? 8u : 1u);
+        *abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == 9) {
+        tmem_alloc(tmem_ptr, Lay::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_ptr;
+
+    if (warp == 10) {
+        // ------------------------------------------------------------ fused-step side work
+        if (p.fused) fused_side_warp(p, lane);
+    } else if (warp == 8) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            tma_prefetch_map(&map_q);
+            tma_prefetch_map(&map_kc);
+            tma_prefetch_map(&map_vc);
+            tma_prefetch_map(&map_kt);
+            tma_prefetch_map(&map_vt);
+            const uint64_t pol = l2_policy_evict_first();
+            int g = 0, k = 0;
+            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
+                const UnitInfo ui = unit_info(p, u);
+                const int qs = k % Lay::QS;
+                if (k >= Lay::QS)
+                    mbar_wait(bars + Lay::B_QEMPTY + qs, ((k / Lay::QS) - 1) & 1, abort_flag);
+                if (!*abort_flag) {
+                    // rows T..127 of the box lie beyond the tensor and arrive as zeros
+                    mbar_arrive_expect_tx(bars + Lay::B_QFULL + qs, Lay::Q_BYTES);
+#pragma unroll
+                    for (int c = 0; c < Lay::DCH; ++c)
+                        tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::GROUP_BYTES,
+                                    &map_q, bars + Lay::B_QFULL + qs, c * 64, 0, u, pol);
+                }
+                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                    const bool tree = (j == ui.n_pref);
+                    const int row = tree ? 0 : j * Lay::KT;
+                    const int ks = g % Lay::KS;
+                    if (g >= Lay::KS)
+                        mbar_wait(bars + Lay::B_KEMPTY + ks, ((g / Lay::KS) - 1) & 1, abort_flag);
+                    if (!*abort_flag) {
+                        mbar_arrive_expect_tx(bars + Lay::B_KFULL + ks, Lay::TILE_BYTES);
+#pragma unroll
+                        for (int c = 0; c < Lay::DCH; ++c)
+                            tma_load_3d(smem + Lay::OFF_K + ks * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                        tree ? &map_kt : &map_kc, bars + Lay::B_KFULL + ks, c * 64,
+                                        row, u, pol);
+                    }
+                    const int vs = g % Lay::VS;
+                    if (g >= Lay::VS)
+                        mbar_wait(bars + Lay::B_VEMPTY + vs, ((g / Lay::VS) - 1) & 1, abort_flag);
+                    if (!*abort_flag) {
+                        mbar_arrive_expect_tx(bars + Lay::B_VFULL + vs, Lay::TILE_BYTES);
+#pragma unroll
+                        for (int c = 0; c < Lay::DCH; ++c)
+                            tma_load_3d(smem + Lay::OFF_V + vs * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                        tree ? &map_vt : &map_vc, bars + Lay::B_VFULL + vs, c * 64,
+                                        row, u, pol);
+                    }
+                }
+            }
+            if (*abort_flag) {
+                for (int i = max(0, g - Lay::KS); i < g; ++i)
+                    mbar_wait_drain(bars + Lay::B_KFULL + i % Lay::KS, (i / Lay::KS) & 1);
+                for (int i = max(0, g - Lay::VS); i < g; ++i)
+                    mbar_wait_drain(bars + Lay::B_VFULL + i % Lay::VS, (i / Lay::VS) & 1);
+                for (int i = max(0, k - Lay::QS); i < k; ++i)
+                    mbar_wait_drain(bars + Lay::B_QFULL + i % Lay::QS, (i / Lay::QS) & 1);
+            }
+        }
+    } else if (warp == 9) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc_qk = make_idesc_bf16(128, 128, 0, 0);
+            const uint32_t idesc_pv = make_idesc_bf16(128, D, 0, 1);
+            const uint32_t sq = smem_addr(smem + Lay::OFF_Q);
+            const uint32_t sk = smem_addr(smem + Lay::OFF_K);
+            const uint32_t sv = smem_addr(smem + Lay::OFF_V);
+
+            // O += P_hi V + P_lo V for tile gp.  Per 32 keys the probability columns
+            // hold 8 columns of hi pairs for keys 0..15, 8 for keys 16..31, then the
+            // lo pairs in the same order.
+            auto issue_pv = [&](int gp, bool first, uint32_t t_o) {
+                const int pb = gp & 1;
+                mbar_wait(bars + Lay::B_PFULL + pb, (gp >> 1) & 1, abort_flag);
+                const int vs = gp % Lay::VS;
+                mbar_wait(bars + Lay::B_VFULL + vs, (gp / Lay::VS) & 1, abort_flag);
+                tc_fence_after();
+                if (!*abort_flag) {
+                    const uint32_t a0 = tmem_base + Lay::T_S + (uint32_t)pb * 128u;
+#pragma unroll
+                    for (int kk = 0; kk < Lay::KT / 16; ++kk) {
+                        const uint64_t b = make_smem_desc(sv + vs * Lay::TILE_BYTES + kk * 2048,
+                                                          Lay::GROUP_BYTES, 1024);
+                        const uint32_t a_hi = a0 + 32u * (kk >> 1) + 8u * (kk & 1);
+                        umma_bf16_ta(t_o, a_hi, b, idesc_pv, (first && kk == 0) ? 0u : 1u);
+                        umma_bf16_ta(t_o, a_hi + 16u, b, idesc_pv, 1u);
+                    }
+                }
+                umma_commit(bars + Lay::B_PDONE + pb);
+                umma_commit(bars + Lay::B_VEMPTY + vs);
+            };
+
+            // Tiles are issued as S(g), PV(g-1) across unit boundaries, so the next
+            // unit's first scores are under way before this unit's last PV product.
+            int g = 0, k = 0;
+            int prev_g = -1;
+            bool prev_first = false;
+            uint32_t prev_to = 0;
+            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
+                const UnitInfo ui = unit_info(p, u);
+                const int qs = k % Lay::QS;
+                const uint32_t t_o = tmem_base + Lay::T_O + (uint32_t)(k & 1) * Lay::O_STRIDE;
+                mbar_wait(bars + Lay::B_QFULL + qs, (k / Lay::QS) & 1, abort_flag);
+                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                    const int ks = g % Lay::KS;
+                    const int sb = g & 1;
+                    mbar_wait(bars + Lay::B_KFULL + ks, (g / Lay::KS) & 1, abort_flag);
+                    // P(g-2) lives in this S buffer until its PV product is done
+                    if (g >= 2) mbar_wait(bars + Lay::B_PDONE + sb, ((g - 2) >> 1) & 1, abort_flag);
+                    tc_fence_after();
+                    if (!*abort_flag) {
+#pragma unroll
+                        for (int kk = 0; kk < D / 16; ++kk) {
+                            const uint32_t off = (kk >> 2) * Lay::GROUP_BYTES + (kk & 3) * 32;
+                            const uint64_t a = make_smem_desc(sq + qs * Lay::Q_BYTES + off, 16, 1024);
+                            const uint64_t b = make_smem_desc(sk + ks * Lay::TILE_BYTES + off, 16, 1024);
+                            umma_bf16(tmem_base + Lay::T_S + sb * 128u, a, b, idesc_qk, kk > 0 ? 1u : 0u);
+                        }
+                    }
+                    umma_commit(bars + Lay::B_SFULL + sb);
+                    umma_commit(bars + Lay::B_KEMPTY + ks);
+                    if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
+                    if (prev_g >= 0) issue_pv(prev_g, prev_first, prev_to);
+                    prev_g = g;
+                    prev_first = (j == 0);
+                    prev_to = t_o;
+                }
+            }
+            if (prev_g >= 0) issue_pv(prev_g, prev_first, prev_to);
+            umma_commit(bars + Lay::B_DRAIN);
+            mbar_wait_drain(bars + Lay::B_DRAIN, 0);
+        }
+    } else {
+        // ------------------------------------------------------------ softmax warps
+        const int qd = warp & 3;                 // TMEM lane quadrant of this warp
+        const int h = warp >> 2;                 // key half: keys [64h, 64h + 64) of a tile
+        const int q = qd * 32 + lane;            // query row (tree token) of this thread
+        const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
+        const float sl2 = p.scale_log2;
+        const bool vec_out = (reinterpret_cast<uintptr_t>(p.out) & 15u) == 0;
+
+        float m = -INFINITY;    // running maximum of the row (log2 units), same in both threads
+        float l = 0.f;          // this thread's share of the row sum
+        uint64_t abits = 0;     // bit i: tree node 64h + i is an ancestor of (or is) node q
+        int cur_b = -1;
+        int g = 0;
+        bool pend = false;      // a finished unit whose output still sits in TMEM
+        int pend_u = 0, pend_ob = 0, pend_g = 0;
+        float pend_linv = 0.f;
+
+        // Probabilities of this thread's 64 keys from its raw scores s against the
+        // maximum mx (exponents clamped at 64), split into bf16 hi + lo and stored
+        // over the scores in TMEM; `lt` gets their sum and `maxd` the largest
+        // unclamped exponent.
+        auto emit = [&](auto kind_c, const uint32_t (&s)[4][16], float mx, int n_valid,
+                        uint32_t t_s, float &lt, float &maxd) {
+            constexpr int KIND = decltype(kind_c)::value;
+            float lt4[4] = {0.f, 0.f, 0.f, 0.f};
+            float md2[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                uint32_t wh[16], wl[16];
+#pragma unroll
+                for (int e = 0; e < 32; e += 2) {
+                    float pv[2];
+                    uint32_t hb[2];
+#pragma unroll
+                    for (int x = 0; x < 2; ++x) {
+                        const int i = 32 * c + e + x;          // key 64h + i of the tile
+                        float d = fmaf(__uint_as_float(s[i >> 4][i & 15]), sl2, -mx);
+                        if (KIND == kMaskRows) d = (64 * h + i < n_valid) ? d : -INFINITY;
+                        if (KIND == kMaskTree) d = ((abits >> i) & 1ull) ? d : -INFINITY;
+                        md2[x] = fmaxf(md2[x], d);
+                        pv[x] = ex2(fminf(d, 64.f));
+                        lt4[(e >> 1) & 3] += pv[x];
+                        hb[x] = __float_as_uint(pv[x]) & 0xFFFF0000u;
+                    }
+                    wh[e >> 1] = __byte_perm(hb[0], hb[1], 0x7632);
+                    const __nv_bfloat162 lo = __floats2bfloat162_rn(pv[0] - __uint_as_float(hb[0]),
+                                                                    pv[1] - __uint_as_float(hb[1]));
+                    wl[e >> 1] = *reinterpret_cast<const uint32_t *>(&lo);
+                }
+                tmem_st16(t_s + 32u * c, wh);
+                tmem_st16(t_s + 32u * c + 16u, wl);
+            }
+            lt = (lt4[0] + lt4[1]) + (lt4[2] + lt4[3]);
+            maxd = fmaxf(md2[0], md2[1]);
+        };
+
+        // Largest visible scaled score among this thread's 64 keys.
+        auto part_max = [&](auto kind_c, const uint32_t (&s)[4][16], int n_valid) {
+            constexpr int KIND = decltype(kind_c)::value;
+            float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int i = 0; i < 64; ++i) {
+                const float v = __uint_as_float(s[i >> 4][i & 15]) * sl2;
+                bool vis = true;
+                if (KIND == kMaskRows) vis = 64 * h + i < n_valid;
+                if (KIND == kMaskTree) vis = ((abits >> i) & 1ull) != 0;
+                mx[i & 3] = fmaxf(mx[i & 3], vis ? v : -INFINITY);
+            }
+            return fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+        };
+
+        // Output of a finished unit: this thread's half of the row of O times 1 / l.
+        auto read_back = [&](int u_out, int ob, int g_last, float linv) {
+            mbar_wait(bars + Lay::B_PDONE + (g_last & 1), (g_last >> 1) & 1, abort_flag);
+            tc_fence_after();
+            const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * Lay::O_STRIDE +
+                                 (uint32_t)h * (D / 2);
+            float *orow = p.out + ((size_t)u_out * T + q) * D + h * (D / 2);
+#pragma unroll
+            for (int ch = 0; ch < D / 32; ++ch) {
+                uint32_t r[16];
+                tmem_ld16(t_o + ch * 16, r);
+                tmem_wait_ld();
+                if (q < T) {
+                    if (vec_out) {
+#pragma unroll
+                        for (int e = 0; e < 16; e += 4)
+                            *reinterpret_cast<float4 *>(orow + ch * 16 + e) =
+                                make_float4(__uint_as_float(r[e]) * linv, __uint_as_float(r[e + 1]) * linv,
+                                            __uint_as_float(r[e + 2]) * linv,
+                                            __uint_as_float(r[e + 3]) * linv);
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) orow[ch * 16 + e] = __uint_as_float(r[e]) * linv;
+                    }
+                }
+            }
+            tc_fence_before();
+        };
+
+        int k = 0;
+        for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
+            const UnitInfo ui = unit_info(p, u);
+            const int ob = k & 1;
+            if (ui.b != cur_b) {
+                // ancestors of node q among tree nodes [64h, 64h + 64)
+                abits = 0;
+                if (q < T) {
+                    bool bad = false;
+                    int a = q;
+                    while (true) {
+                        if ((a >> 6) == h) abits |= 1ull << (a & 63);
+                        const int pa = __ldg(p.parent + (size_t)ui.b * T + a);
+                        if (a == 0) {
+                            bad = (pa != -1);
+                            break;
+                        }
+                        if (pa < 0 || pa >= a) {
+                            bad = true;
+                            break;
+                        }
+                        a = pa;
+                    }
+                    if (bad && h == 0 && p.dev_status) p.dev_status[ui.b] = kErrTree;
+                }
+                if (q == 0 && h == 0 && p.dev_status && (ui.P_raw < 0 || ui.P_raw > p.S_max))
+                    p.dev_status[ui.b] = kErrCapacity;
+                cur_b = ui.b;
+            }
+
+            for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                const bool tree = (j == ui.n_pref);
+                const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
+                const int kind = tree ? kMaskTree : (n_valid < Lay::KT ? kMaskRows : kMaskNone);
+                const int sb = g & 1;
+                mbar_wait(bars + Lay::B_SFULL + sb, (g >> 1) & 1, abort_flag);
+                tc_fence_after();
+                const uint32_t t_s = tmem_base + lane_off + Lay::T_S + (uint32_t)sb * 128u +
+                                     (uint32_t)h * 64u;
+                uint32_t s[4][16];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) tmem_ld16(t_s + 16u * i, s[i]);
+                tmem_wait_ld();
+
+                float lt = 0.f;
+                bool exact = (j == 0);
+                if (!exact) {
+                    // optimistic pass against the current maximum
+                    float maxd = -INFINITY;
+                    if (kind == kMaskNone) emit(kind_t<kMaskNone>{}, s, m, n_valid, t_s, lt, maxd);
+                    else if (kind == kMaskRows) emit(kind_t<kMaskRows>{}, s, m, n_valid, t_s, lt, maxd);
+                    else emit(kind_t<kMaskTree>{}, s, m, n_valid, t_s, lt, maxd);
+                    exact = named_bar_or(1, 256, maxd > 16.f);
+                }
+                if (exact) {
+                    float pm;
+                    if (kind == kMaskNone) pm = part_max(kind_t<kMaskNone>{}, s, n_valid);
+                    else if (kind == kMaskRows) pm = part_max(kind_t<kMaskRows>{}, s, n_valid);
+                    else pm = part_max(kind_t<kMaskTree>{}, s, n_valid);
+                    xm[h * Lay::M + q] = pm;
+                    named_bar_sync(1, 256);
+                    const float mn = fmaxf(m, fmaxf(xm[q], xm[Lay::M + q]));
+                    const float alpha = (mn == m) ? 1.f : ex2(m - mn);
+                    if (j > 0) {
+                        if (__any_sync(0xffffffffu, alpha != 1.f)) {
+                            // rescale this thread's half of the row of O once the PV
+                            // product of the previous tile has landed
+                            mbar_wait(bars + Lay::B_PDONE + ((g - 1) & 1), ((g - 1) >> 1) & 1,
+                                      abort_flag);
+                            tc_fence_after();
+                            const uint32_t t_o = tmem_base + lane_off + Lay::T_O +
+                                                 (uint32_t)ob * Lay::O_STRIDE + (uint32_t)h * (D / 2);
+#pragma unroll
+                            for (int ch = 0; ch < D / 32; ++ch) {
+                                uint32_t r[16];
+                                tmem_ld16(t_o + ch * 16, r);
+                                tmem_wait_ld();
+#pragma unroll
+                                for (int e = 0; e < 16; ++e)
+                                    r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+                                tmem_st16(t_o + ch * 16, r);
+                            }
+                        }
+                        l *= alpha;
+                    }
+                    m = mn;
+                    tmem_wait_st();   // optimistic probabilities are overwritten below
+                    float unused;
+                    if (kind == kMaskNone) emit(kind_t<kMaskNone>{}, s, m, n_valid, t_s, lt, unused);
+                    else if (kind == kMaskRows) emit(kind_t<kMaskRows>{}, s, m, n_valid, t_s, lt, unused);
+                    else emit(kind_t<kMaskTree>{}, s, m, n_valid, t_s, lt, unused);
+                }
+                l += lt;
+
+                // V rows of invisible keys in a partial prefix tile may be NaN: zero them
+                if (kind == kMaskRows && h == 0) {
+                    const int vs = g % Lay::VS;
+                    mbar_wait(bars + Lay::B_VFULL + vs, (g / Lay::VS) & 1, abort_flag);
+                    if (q >= n_valid) {
+                        const uint32_t vrow = smem_addr(smem + Lay::OFF_V + vs * Lay::TILE_BYTES) + q * 128u;
+#pragma unroll
+                        for (int c = 0; c < Lay::DCH; ++c)
+#pragma unroll
+                            for (int x = 0; x < 8; ++x)
+                                st_shared_v4(vrow + c * Lay::GROUP_BYTES + x * 16, 0u, 0u, 0u, 0u);
+                    }
+                }
+                tmem_wait_st();
+                fence_proxy_async_smem();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bars + Lay::B_PFULL + sb);
+
+                // the previous unit's output, once this unit's first tile is on its way
+                if (j == 0 && pend) {
+                    read_back(pend_u, pend_ob, pend_g, pend_linv);
+                    pend = false;
+                }
+
+                if (j == ui.n_tiles - 1) {
+                    // ------------------------------------------ unit end: row sum, LSE
+                    xl[h * Lay::M + q] = l;
+                    named_bar_sync(1, 256);
+                    const float L = xl[q] + xl[Lay::M + q];
+                    if (h == 0 && q < T && p.lse)
+                        p.lse[(size_t)u * T + q] = (m + lg2(L)) * 0.69314718055994530942f;
+                    pend = true;
+                    pend_u = u;
+                    pend_ob = ob;
+                    pend_g = g;
+                    pend_linv = rcp(L);
+                    m = -INFINITY;
+                    l = 0.f;
+                }
+            }
+        }
+        if (pend) read_back(pend_u, pend_ob, pend_g, pend_linv);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (*abort_flag && threadIdx.x == 0) {
+        for (int b = 0; b < p.B; ++b) {
+            if (p.dev_status) p.dev_status[b] = kErrTimeout;
+            if (p.fused) atomicMax(p.fs.status + b, (int)kErrTimeout);
+        }
+    }
+    if (warp == 9) tmem_dealloc(tmem_base, Lay::TMEM_COLS);
+}
+
+template <int D>
+static cudaError_t launch_rows_t(const AttnMaps &m, const AttnParams &p, int num_sms,
+                                 bool programmatic, cudaStream_t stream)
+{
+    using Lay = RowsLayout<D>;
+    auto kern = tree_attention_rows_kernel<D>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)Lay::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(p.n_units < num_sms ? p.n_units : num_sms));
+    cfg.blockDim = dim3(352);
+    cfg.dynamicSmemBytes = Lay::SMEM_BYTES;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = programmatic ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, m.q, m.kc, m.vc, m.kt, m.vt, p);
+}
+
+cudaError_t launch_tree_attention_rows(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
+                                       bool programmatic, cudaStream_t stream)
+{
+    if (D == 128) return launch_rows_t<128>(m, p, num_sms, programmatic, stream);
+    return launch_rows_t<64>(m, p, num_sms, programmatic, stream);
+}
+
+}  // namespace ppd

@@ -202,6 +202,20 @@ PPD_DEV void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32
         : "memory");
 }
 
+// D(tmem) (+)= A(tmem) * B(smem), bf16 inputs, fp32 accumulator.  A is M x K
+// with row m in TMEM lane m, two consecutive k per 32-bit column (the lower k in
+// the low half); a_tmem addresses its first column (lane field 0).
+PPD_DEV void umma_bf16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                          uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // Arrive once on `bar` when every tcgen05.mma issued so far by this thread is done.
 PPD_DEV void umma_commit(uint64_t *bar)
 {

@@ -54,8 +54,12 @@ struct AttnParams {
 // Batches up to this size run the fused two-grid step.
 constexpr int kFusedMaxB = 64;
 
+// Dispatches on the padded tree size: up to 64 tokens the key-row kernel
+// (ppd_attention.cu), 65..128 the query-row kernel (ppd_attention_rows.cu).
 cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
                                   bool programmatic, cudaStream_t stream);
+cudaError_t launch_tree_attention_rows(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
+                                       bool programmatic, cudaStream_t stream);
 
 // Splits per node row of the argmax: about 512 blocks over all rows, chunks of
 // at least 2048 logits, at most 64 splits.
@@ -101,7 +105,7 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_tree,
 
 cudaError_t launch_round_bf16(const float *src, uint16_t *dst, int64_t n, cudaStream_t stream);
 
-cudaError_t launch_selftest_umma(const CUtensorMap &ma, const CUtensorMap &mb, const void *b_raw,
-                                 float *d, int mode, int N, cudaStream_t stream);
+cudaError_t launch_selftest_umma(const CUtensorMap &ma, const CUtensorMap &mb, const void *a_raw,
+                                 const void *b_raw, float *d, int mode, int N, cudaStream_t stream);
 
 }  // namespace ppd

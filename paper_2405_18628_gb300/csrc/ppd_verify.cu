@@ -221,7 +221,7 @@ constexpr uint32_t kSelfTestSmem = 200 * 1024;   // generous: operands use < 96 
 
 __global__ void __launch_bounds__(128, 1)
 selftest_umma_kernel(const __grid_constant__ CUtensorMap ma, const __grid_constant__ CUtensorMap mb,
-                     const uint16_t *b_raw, float *d, int mode, int N)
+                     const uint16_t *a_raw, const uint16_t *b_raw, float *d, int mode, int N)
 {
     extern __shared__ __align__(1024) uint8_t smem[];
     if (smem_addr(smem) & 1023u) return;
@@ -258,18 +258,40 @@ selftest_umma_kernel(const __grid_constant__ CUtensorMap ma, const __grid_consta
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_ptr;
+    if (mode == 3) {
+        // a given [128][256]: columns [0,128) the hi parts, [128,256) the lo parts of
+        // a 128 x 128 A.  Thread t writes row t into TMEM columns 128.. in the layout
+        // of the row-layout attention kernel's probability tile: per 32 keys, 16
+        // columns of hi pairs followed by 16 columns of lo pairs.
+        const int t = threadIdx.x;
+        const uint32_t *row = reinterpret_cast<const uint32_t *>(a_raw + (size_t)t * 256);
+        const uint32_t lane_off = (uint32_t)((t >> 5) * 32) << 16;
+        for (int c = 0; c < 4; ++c) {
+            uint32_t wh[16], wl[16];
+            for (int i = 0; i < 16; ++i) {
+                wh[i] = row[16 * c + i];
+                wl[i] = row[64 + 16 * c + i];
+            }
+            tmem_st16(tmem + lane_off + 128 + 32 * c, wh);
+            tmem_st16(tmem + lane_off + 128 + 32 * c + 16, wl);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    }
 
     if (threadIdx.x == 0) {
         uint32_t tx = 0;
         if (mode == 0) tx = 128 * 128 * 2 + (uint32_t)N * 128 * 2;
-        else tx = (mode == 1 ? 2u : 1u) * 16384u;
+        else if (mode != 3) tx = (mode == 1 ? 2u : 1u) * 16384u;
         mbar_arrive_expect_tx(bar, tx);
         if (mode == 0) {
             tma_load_2d(sa, &ma, bar, 0, 0);
             tma_load_2d(sa + 16384, &ma, bar, 64, 0);
             tma_load_2d(sb, &mb, bar, 0, 0);
             tma_load_2d(sb + (size_t)N * 128, &mb, bar, 64, 0);
-        } else {
+        } else if (mode != 3) {
             tma_load_2d(sa, &ma, bar, 0, 0);
             if (mode == 1) tma_load_2d(sa + 16384, &ma, bar, 64, 0);
         }
@@ -277,7 +299,14 @@ selftest_umma_kernel(const __grid_constant__ CUtensorMap ma, const __grid_consta
         tc_fence_after();
         if (!*abort_flag) {
             const uint32_t a0 = smem_addr(sa), b0 = smem_addr(sb);
-            for (int kk = 0; kk < 8; ++kk) {
+            for (int kk = 0; kk < 8 && mode == 3; ++kk) {
+                const uint32_t a_hi = tmem + 128 + 32 * (kk >> 1) + 8 * (kk & 1);
+                const uint64_t db = make_smem_desc(b0 + kk * 2048, 16384, 1024);
+                const uint32_t idesc = make_idesc_bf16(128, N, 0, 1);
+                umma_bf16_ta(tmem, a_hi, db, idesc, kk > 0 ? 1u : 0u);
+                umma_bf16_ta(tmem, a_hi + 16, db, idesc, 1u);
+            }
+            for (int kk = 0; kk < 8 && mode != 3; ++kk) {
                 uint64_t da, db;
                 uint32_t idesc;
                 if (mode == 0) {
@@ -312,15 +341,16 @@ selftest_umma_kernel(const __grid_constant__ CUtensorMap ma, const __grid_consta
     if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
-cudaError_t launch_selftest_umma(const CUtensorMap &ma, const CUtensorMap &mb, const void *b_raw,
-                                 float *d, int mode, int N, cudaStream_t stream)
+cudaError_t launch_selftest_umma(const CUtensorMap &ma, const CUtensorMap &mb, const void *a_raw,
+                                 const void *b_raw, float *d, int mode, int N, cudaStream_t stream)
 {
     cudaError_t e = cudaFuncSetAttribute(selftest_umma_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSelfTestSmem);
     if (e != cudaSuccess) return e;
     selftest_umma_kernel<<<1, 128, kSelfTestSmem, stream>>>(
-        ma, mb, static_cast<const uint16_t *>(b_raw), d, mode, N);
+        ma, mb, static_cast<const uint16_t *>(a_raw), static_cast<const uint16_t *>(b_raw), d, mode,
+        N);
     return cudaGetLastError();
 }
 
