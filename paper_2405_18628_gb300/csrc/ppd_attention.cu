@@ -17,16 +17,19 @@
 //
 // Warp roles (352 threads): warps 0-7 softmax (two warpgroups, each owning
 // half of the query columns), warp 8 TMA producer, warp 9 MMA issuer and TMEM
-// owner, warp 10 the fused step's argmax / acceptance / compaction.  The running row maximum m is updated lazily: a tile is first done
+// owner, warp 10 the fused step's argmax / acceptance / compaction.  This
+// kernel serves trees of up to 64 tokens; larger trees fill the tensor core's
+// M side with queries and run the query-row kernel (ppd_attention_rows.cu).
+// The running row maximum m is updated lazily: a tile is first done
 // with the current m, and only if a score exceeds m by more than 2^16 (or on
 // a unit's first tile) does it take the exact path -- a cross-lane maximum,
 // a rescale of O and of the row sums, and recomputed probabilities.  The
 // tree mask is an ancestor bitset built from the parent array; rows beyond
 // the prefix (which may hold anything, NaN included) are masked by select
-// and their V rows are zeroed in shared memory before the PV product.  For
-// trees of up to 64 tokens O is double-buffered in TMEM and a unit's output
-// is read back only after the next unit's first tile, so the stream of tiles
-// never waits for a unit's last PV product.
+// and their V rows are zeroed in shared memory before the PV product.  O is
+// double-buffered in TMEM and a unit's output is read back only after the
+// next unit's first tile, so the stream of tiles never waits for a unit's
+// last PV product.
 #include "ppd_attention_common.cuh"
 
 #include <cmath>
@@ -34,10 +37,10 @@
 
 namespace ppd {
 
-template <int D_, int TPMAX_>
+template <int D_>
 struct AttnLayout {
     static constexpr int D = D_;
-    static constexpr int TPMAX = TPMAX_;          // largest padded tree size served
+    static constexpr int TPMAX = 64;              // largest padded tree size served
     static constexpr int KT = 128;                // keys per tile
     static constexpr int DCH = D / 64;            // 64-column (128-byte) groups along D
     static constexpr uint32_t GROUP_BYTES = KT * 128;   // one column group of a tile
@@ -46,13 +49,13 @@ struct AttnLayout {
     static constexpr uint32_t Q_BYTES = TPMAX * D * 2;
     static constexpr int P_GROUPS = 2 * TPMAX / 64;      // [hi | lo] columns / 64
     static constexpr uint32_t P_BYTES = P_GROUPS * GROUP_BYTES;
-    static constexpr int OB = (TPMAX <= 64) ? 2 : 1;     // O accumulators in TMEM
-    static constexpr int QS = (TPMAX <= 64) ? 2 : 1;     // Q buffers
-    // With D = 128 and trees of <= 64 tokens a tile's probabilities fit exactly in
-    // its own K slot, free once S^T = K Q^T is done: no dedicated probability
-    // tiles, and the freed shared memory buys a third K and V stage.
-    static constexpr bool P_IN_K = (D == 128) && (TPMAX <= 64);
-    static constexpr int PS = P_IN_K ? 0 : ((TPMAX <= 64) ? 2 : 1);   // dedicated P tiles
+    static constexpr int OB = 2;                          // O accumulators in TMEM
+    static constexpr int QS = 2;                          // Q buffers
+    // With D = 128 a tile's probabilities fit exactly in its own K slot, free
+    // once S^T = K Q^T is done: no dedicated probability tiles, and the freed
+    // shared memory buys a third K and V stage.
+    static constexpr bool P_IN_K = (D == 128);
+    static constexpr int PS = P_IN_K ? 0 : 2;             // dedicated P tiles
     static constexpr int PB = P_IN_K ? 2 : PS;            // P full/free barrier pairs
     static constexpr int KS = P_IN_K ? 3 : 2;             // K tile ring
     static constexpr int VS = P_IN_K ? 3 : 2;             // V tile ring
@@ -80,18 +83,16 @@ struct AttnLayout {
     static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
     static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
     static constexpr uint32_t OFF_M2 = (OFF_ABORT + 4 + 15) & ~15u;
-    // [OB][TPMAX] reciprocal row sums; with one accumulator they share the
-    // running maxima's storage (read back before the maxima are reset)
-    static constexpr uint32_t OFF_LINV = (OB == 1) ? OFF_M2 : OFF_M2 + TPMAX * 4;
-    static constexpr uint32_t OFF_UNION = OFF_M2 + TPMAX * 4 + (OB == 1 ? 0 : OB * TPMAX * 4);
+    static constexpr uint32_t OFF_LINV = OFF_M2 + TPMAX * 4;      // [OB][TPMAX] 1 / row sums
+    static constexpr uint32_t OFF_UNION = OFF_LINV + OB * TPMAX * 4;
     // union: ancestor bitsets [TPMAX][ANC_WORDS] u32, or reduction scratch [2][4][NC_MAX] f32
     static constexpr uint32_t ANC_BYTES = TPMAX * ANC_WORDS * 4;
     static constexpr uint32_t RED_BYTES = 2 * 4 * NC_MAX * 4;
     static constexpr uint32_t UNION_BYTES = ANC_BYTES > RED_BYTES ? ANC_BYTES : RED_BYTES;
     static constexpr uint32_t SMEM_BYTES = OFF_UNION + UNION_BYTES;
-    // TMEM columns: S0 | S1 | O0 (hi | lo) [| O1 (hi | lo)]
+    // TMEM columns: S0 | S1 | O0 (hi | lo) | O1 (hi | lo)
     static constexpr uint32_t T_S = 0, T_O = 2 * TPMAX;
-    static constexpr uint32_t TMEM_COLS = (2 + 2 * OB) * TPMAX <= 256 ? 256 : 512;
+    static constexpr uint32_t TMEM_COLS = 512;
 
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
     static_assert(!P_IN_K || P_BYTES <= TILE_BYTES, "probability tile fits in a K slot");
@@ -108,7 +109,7 @@ PPD_DEV uint32_t p_offset(int g)
 }
 
 
-template <int D, int TPMAX>
+template <int D>
 __global__ void __launch_bounds__(352, 1)
 tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                       const __grid_constant__ CUtensorMap map_kc,
@@ -116,7 +117,8 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                       const __grid_constant__ CUtensorMap map_kt,
                       const __grid_constant__ CUtensorMap map_vt, const AttnParams p)
 {
-    using Lay = AttnLayout<D, TPMAX>;
+    using Lay = AttnLayout<D>;
+    constexpr int TPMAX = Lay::TPMAX;
     extern __shared__ __align__(1024) uint8_t smem[];
     // The swizzled operand tiles need a 1024-byte aligned base; the check is
     // uniform over the CTA, before any barrier.
@@ -257,7 +259,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                 if (Lay::P_IN_K) umma_commit(bars + Lay::B_KEMPTY + gp % Lay::KS);
             };
 
+            // Tiles are issued as S(g), PV(g-1) across unit boundaries, so the next
+            // unit's first scores are under way before this unit's last PV product.
             int g = 0, k = 0;
+            int prev_g = -1;
+            bool prev_first = false;
+            uint32_t prev_to = 0;
             for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
                 const UnitInfo ui = unit_info(p, u);
                 const int qs = k % Lay::QS;
@@ -282,10 +289,13 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     umma_commit(bars + Lay::B_SFULL + sb);
                     if (!Lay::P_IN_K) umma_commit(bars + Lay::B_KEMPTY + ks);
                     if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
-                    if (j >= 1) issue_pv(g - 1, j == 1, t_o);
+                    if (prev_g >= 0) issue_pv(prev_g, prev_first, prev_to);
+                    prev_g = g;
+                    prev_first = (j == 0);
+                    prev_to = t_o;
                 }
-                issue_pv(g - 1, ui.n_tiles == 1, t_o);
             }
+            if (prev_g >= 0) issue_pv(prev_g, prev_first, prev_to);
             // all MMAs finished before TMEM can be released
             umma_commit(bars + Lay::B_DRAIN);
             mbar_wait_drain(bars + Lay::B_DRAIN, 0);
@@ -574,7 +584,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     if (g >= Lay::PS)
                         mbar_wait(bars + Lay::B_PFREE + ps, ((g / Lay::PS) - 1) & 1, abort_flag);
                 }
-                bool o_ready = (Lay::PB == 1);   // PV of tile g-1 known to be complete
+                bool o_ready = false;   // PV of tile g-1 known to be complete
 
                 // Column groups of up to 32 queries, done optimistically with the
                 // current running maxima; on a unit's first tile, or when a score
@@ -653,7 +663,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         if (p.lse && q < T)
                             p.lse[(size_t)u * T + q] = (m2[q] + lg2(l)) * 0.69314718055994530942f;
                         linv[ob * TPMAX + q] = rcp(l);
-                        if (Lay::OB > 1) m2[q] = -INFINITY;
+                        m2[q] = -INFINITY;
                     }
 #pragma unroll
                     for (int c = 0; c < NL; ++c) lacc[c] = 0.f;
@@ -661,15 +671,6 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     pend_u = u;
                     pend_ob = ob;
                     pend_g = g;
-                    if (Lay::OB == 1) {
-                        // a single accumulator: read it back before the next unit reuses it,
-                        // then reset the running maxima that share storage with 1 / l
-                        named_bar_sync(1 + wg, 128);
-                        read_back(pend_u, pend_ob, pend_g);
-                        pend = false;
-                        named_bar_sync(1 + wg, 128);
-                        if (t < NC) m2[q0 + t] = -INFINITY;
-                    }
                 }
             }
         }
@@ -691,12 +692,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
     if (warp == 9) tmem_dealloc(tmem_base, Lay::TMEM_COLS);
 }
 
-template <int D, int TPMAX>
+template <int D>
 static cudaError_t launch_tree_attention_t(const AttnMaps &m, const AttnParams &p, int num_sms,
                                            bool programmatic, cudaStream_t stream)
 {
-    using Lay = AttnLayout<D, TPMAX>;
-    auto kern = tree_attention_kernel<D, TPMAX>;
+    using Lay = AttnLayout<D>;
+    auto kern = tree_attention_kernel<D>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)Lay::SMEM_BYTES);
     if (e != cudaSuccess) return e;
@@ -717,8 +718,8 @@ cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D,
                                   bool programmatic, cudaStream_t stream)
 {
     if (p.T_pad > 64) return launch_tree_attention_rows(m, p, D, num_sms, programmatic, stream);
-    if (D == 128) return launch_tree_attention_t<128, 64>(m, p, num_sms, programmatic, stream);
-    return launch_tree_attention_t<64, 64>(m, p, num_sms, programmatic, stream);
+    if (D == 128) return launch_tree_attention_t<128>(m, p, num_sms, programmatic, stream);
+    return launch_tree_attention_t<64>(m, p, num_sms, programmatic, stream);
 }
 
 }  // namespace ppd
