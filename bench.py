@@ -6,8 +6,11 @@ node argmax, acceptance, KV compaction) through libppd's C ABI.
 
 Prints one JSON line.  The default workload is the Vicuna-7B-shaped cache
 (32 layers, 32 heads x 128, bf16 K/V, batch 1, prefix 2048, 64-token tree,
-vocab 32000).  Inputs are seeded synthetic tensors resident in HBM; L2 is
-flushed (a 256 MiB write) before every timed step, outside the step's events.
+vocab 32000).  Inputs are seeded synthetic tensors resident in HBM.  When a
+step's inputs are at least four times the 129 MB L2 (every Vicuna-shaped
+workload: 1.17 GB per step at Vicuna-7B), steps run back to back and no step
+can find the previous one's data in L2; smaller workloads flush L2 (a 256 MiB
+write) before every timed step, outside the step's events.
 
 Under torchrun (N > 1) each rank runs an independent replica of the workload
 on its own GPU (weak scaling: the sequences of different ranks are
@@ -36,6 +39,7 @@ METRIC = "verify steps/s and achieved HBM GB/s (frac of ~8 TB/s), Vicuna-7B shap
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 256 << 20
+L2_BYTES = 129 * 1000 * 1000
 
 # DRAM traffic of one tree-attention launch from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum), keyed by workload, with the
@@ -48,7 +52,8 @@ MEASURED_TRAFFIC = {
 
 def attention_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("ppd_attention.cu", "ppd_device.cuh", "ppd_accept.cuh", "ppd_kernels.h"):
+    for f in ("ppd_attention.cu", "ppd_attention_rows.cu", "ppd_device.cuh", "ppd_accept.cuh",
+              "ppd_kernels.h"):
         with open(os.path.join(ROOT, "paper_2405_18628_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -195,6 +200,10 @@ def parse():
                     help="seconds of oracle work in the CPU baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run the workload with this many layers (profiling captures)")
+    ap.add_argument("--l2", default="auto", choices=["auto", "flush", "none"],
+                    help="auto: flush L2 before each step unless the step's inputs exceed 4x L2")
     return ap.parse_args()
 
 
@@ -266,6 +275,9 @@ def main():
     world, rank, local = dist_setup()
     from paper_2405_18628_gb300 import workloads as W
     w = W.WORKLOADS[args.config]
+    if args.layers:
+        # fewer layers of the same shapes: small cases for profiler captures
+        w = W.scaled(w, L=args.layers)
     if args.impl == "reference":
         run_reference(args, w, world, rank)
         return
@@ -289,8 +301,14 @@ def main():
     parent, cand, prefix = i32(s.parent), i32(s.cand_tokens), i32(s.prefix_len)
     logits = torch.from_numpy(s.logits).to(dev)
     bufs = ppd.StepBuffers(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max, device=dev)
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
+    footprint = step_bytes(w, 0)
+    do_flush = args.l2 == "flush" or (args.l2 == "auto" and footprint < 4 * L2_BYTES)
+    flush = torch.empty(L2_FLUSH_BYTES if do_flush else 0, dtype=torch.uint8, device=dev)
+
+    def maybe_flush():
+        if do_flush:
+            flush.zero_()
 
     def step():
         ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
@@ -299,7 +317,7 @@ def main():
                             stream=stream)
 
     for _ in range(max(3, args.warmup)):
-        flush.zero_()
+        maybe_flush()
         step()
     torch.cuda.synchronize()
     status = bufs.dev_status.cpu().numpy()
@@ -317,7 +335,7 @@ def main():
         torch.cuda.synchronize()
         wall0 = time.perf_counter()
         for k in range(K):
-            flush.zero_()
+            maybe_flush()
             ev[k][0].record(stream)
             step()
             ev[k][1].record(stream)
@@ -326,6 +344,7 @@ def main():
             pg.barrier()
         wall = time.perf_counter() - wall0
     step_ms = [a.elapsed_time(b) for a, b in ev]
+    q10, q50, q90 = np.percentile(step_ms, [10, 50, 90])
     total_ms = max_over_ranks(sum(step_ms), pg, dev)
     ms_per_step = total_ms / K
     value = aggregate_rate(K, world, total_ms)
@@ -337,7 +356,7 @@ def main():
            for _ in range(K2)]
     st_att = torch.empty(w.B, dtype=torch.int32, device=dev)
     for k in range(K2 + 3):
-        flush.zero_()
+        maybe_flush()
         if k >= 3:
             ev2[k - 3][0].record(stream)
         ppd.ppd_tree_attention(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
@@ -349,7 +368,7 @@ def main():
     att_bytes = attention_bytes(w)
     peak, peak_kind = measured_peak_gbs()
     achieved = att_bytes / (att_ms * 1e-3) / 1e9
-    tr = MEASURED_TRAFFIC.get(w.name)
+    tr = None if args.layers else MEASURED_TRAFFIC.get(w.name)
     traffic = tr["bytes_per_launch"] if tr and tr.get("src") == attention_source_hash() else None
 
     # ---------------------------------------------------------------- end to end, host buffers
@@ -378,11 +397,11 @@ def main():
             stream.synchronize()
 
         for _ in range(3):
-            flush.zero_()
+            maybe_flush()
             e2e_step()
         e_ms = []
         for _ in range(K3):
-            flush.zero_()
+            maybe_flush()
             torch.cuda.synchronize()
             t0 = time.perf_counter()
             e2e_step()
@@ -405,11 +424,16 @@ def main():
             "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": w.name, "layers": w.L, "batch": w.B, "heads": w.H,
+            "config": {"workload": w.name + (f" ({w.L} layers)" if args.layers else ""),
+                       "layers": w.L, "batch": w.B, "heads": w.H,
                        "head_dim": w.D, "prefix": w.P, "tree_tokens": w.T, "vocab": w.V,
-                       "S_max": w.S_max, "l2": "flushed before every step (256 MiB write, "
-                                               "outside the step events)",
+                       "S_max": w.S_max,
+                       "l2": ("flushed before every step (256 MiB write, outside the step events)"
+                              if do_flush else
+                              f"not flushed: inputs larger than L2 ({footprint / 1e6:.0f} MB "
+                              f"streamed per step, L2 {L2_BYTES / 1e6:.0f} MB)"),
                        "parallelism": f"replicas x{world}"},
+            "ms_per_step_p10_p50_p90": [float(q10), float(q50), float(q90)],
             "step_gbs": sb / (ms_per_step * 1e-3) / 1e9,
             "step_frac_of_8tbs": sb / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
             "step_bytes": sb,

@@ -8,6 +8,7 @@
 #include "ppd_device.cuh"
 #include "ppd_kernels.h"
 
+#include <atomic>
 #include <type_traits>
 
 namespace ppd {
@@ -122,4 +123,35 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
     }
 }
 
+// Launch one of the persistent attention kernels: one CTA per SM (at most one
+// per unit), `smem` bytes of dynamic shared memory, with programmatic stream
+// serialization when asked.  The shared-memory opt-in is set once per device.
+template <class Kern>
+cudaError_t launch_attention_grid(Kern kern, uint32_t smem, std::atomic<uint64_t> &configured,
+                                  const AttnMaps &m, const AttnParams &p, int num_sms,
+                                  bool programmatic, cudaStream_t stream)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = dev < 64 ? (1ull << dev) : 0ull;
+    if (!bit || !(configured.load(std::memory_order_acquire) & bit)) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured.fetch_or(bit, std::memory_order_acq_rel);
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(p.n_units < num_sms ? p.n_units : num_sms));
+    cfg.blockDim = dim3(352);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = programmatic ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, m.q, m.kc, m.vc, m.kt, m.vt, p);
+}
+
 }  // namespace ppd
+

@@ -500,22 +500,9 @@ template <int D>
 static cudaError_t launch_rows_t(const AttnMaps &m, const AttnParams &p, int num_sms,
                                  bool programmatic, cudaStream_t stream)
 {
-    using Lay = RowsLayout<D>;
-    auto kern = tree_attention_rows_kernel<D>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)Lay::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(p.n_units < num_sms ? p.n_units : num_sms));
-    cfg.blockDim = dim3(352);
-    cfg.dynamicSmemBytes = Lay::SMEM_BYTES;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = programmatic ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, kern, m.q, m.kc, m.vc, m.kt, m.vt, p);
+    static std::atomic<uint64_t> configured{0};
+    return launch_attention_grid(tree_attention_rows_kernel<D>, RowsLayout<D>::SMEM_BYTES, configured,
+                                 m, p, num_sms, programmatic, stream);
 }
 
 cudaError_t launch_tree_attention_rows(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
