@@ -41,12 +41,16 @@ FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 256 << 20
 L2_BYTES = 129 * 1000 * 1000
 
-# DRAM traffic of one tree-attention launch from an ncu capture
-# (dram__bytes_read.sum + dram__bytes_write.sum), keyed by workload, with the
-# hash of the attention source it was taken on: a stale entry reports null.
+# DRAM traffic of one tree-attention launch (dram__bytes_read.sum +
+# dram__bytes_write.sum), keyed by workload, with the hash of the attention
+# sources it was taken on: a stale entry reports null.  The captures ran the
+# same shapes with 19 layers (608 / 760 units: whole rounds of 152 CTAs) and
+# are scaled to the full layer count, since traffic grows with the units.
 MEASURED_TRAFFIC = {
-    # one full ncu capture of the Vicuna-7B-shaped launch (dram read + write)
-    "vicuna7b": {"bytes_per_launch": 1_131_670_696, "src": "a117ccfb4fc9baa9"},
+    # 675,677,440 B at 19 layers x 32/19
+    "vicuna7b": {"bytes_per_launch": 1_138_004_109, "src": "d710315aa21f4d5a"},
+    # 1,659,421,696 B at 19 layers x 40/19
+    "vicuna13b": {"bytes_per_launch": 3_493_519_360, "src": "d710315aa21f4d5a"},
 }
 
 
