@@ -70,6 +70,13 @@ def _load():
         lib.oracle_kv_compact.argtypes = [vp, vp, vp, vp, i32p, i32p, i32p, c_int, c_int,
                                           c_int, c_int, c_int, c_int, c_int]
         lib.oracle_kv_compact.restype = c_int
+        c_dbl = ctypes.c_double
+        lib.oracle_node_stats.argtypes = [vp, c_i64, c_i64, c_dbl, f64p, f64p]
+        lib.oracle_node_stats.restype = None
+        lib.oracle_typical_accept.argtypes = [vp, i32p, i32p, i32p, i32p, c_int, c_int, c_int,
+                                              c_int, c_dbl, c_dbl, c_dbl, i32p, i32p, i32p, i32p,
+                                              i32p, f64p, f64p]
+        lib.oracle_typical_accept.restype = c_int
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = c_int
         _lib = lib
@@ -193,6 +200,45 @@ def accept_path(argmax, cand_tokens, parent, prefix_len, V: int, S_max: int):
     return res
 
 
+def node_stats(logits, temperature: float):
+    """lse and entropy (fp64 numpy arrays of logits.shape[:-1]) of
+    softmax(logits / temperature) over the last axis."""
+    a, _ = _host(logits)
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    V = a.shape[-1]
+    rows = a.size // V if V else 0
+    lse = np.empty(a.shape[:-1], np.float64)
+    ent = np.empty(a.shape[:-1], np.float64)
+    _load().oracle_node_stats(_ptr(a), rows, V, float(temperature), _ptr(lse, ctypes.c_double),
+                              _ptr(ent, ctypes.c_double))
+    return lse, ent
+
+
+def typical_accept(logits, argmax, cand_tokens, parent, prefix_len, S_max: int,
+                   temperature: float, epsilon: float, delta: float):
+    """Typical acceptance.  logits [B,T,V] fp32.  Returns dict of accept_len,
+    path, next_token, new_prefix_len, status (int32) and p_tok, threshold
+    ([B,T] fp64, NaN where no test applies)."""
+    lg, _ = _host(logits)
+    lg = np.ascontiguousarray(lg, dtype=np.float32)
+    am, cd, par, pl = _i32(argmax), _i32(cand_tokens), _i32(parent), _i32(prefix_len)
+    B, T = par.shape
+    V = lg.shape[-1]
+    res = {k: np.empty(B, np.int32) for k in ("accept_len", "next_token", "new_prefix_len", "status")}
+    res["path"] = np.empty((B, T), np.int32)
+    res["p_tok"] = np.empty((B, T), np.float64)
+    res["threshold"] = np.empty((B, T), np.float64)
+    p = lambda a: _ptr(a, ctypes.c_int32)
+    d = lambda a: _ptr(a, ctypes.c_double)
+    rc = _load().oracle_typical_accept(
+        _ptr(lg), p(am), p(cd), p(par), p(pl), B, T, int(V), int(S_max), float(temperature),
+        float(epsilon), float(delta), p(res["accept_len"]), p(res["path"]), p(res["next_token"]),
+        p(res["new_prefix_len"]), p(res["status"]), d(res["p_tok"]), d(res["threshold"]))
+    if rc != 0:
+        raise ValueError(f"oracle_typical_accept rejected its arguments (code {rc})")
+    return res
+
+
 def kv_compact(k_cache, v_cache, k_tree, v_tree, path, accept_len, prefix_len):
     """Returns new (k_cache, v_cache) numpy copies with the accepted rows written."""
     kc, tagk = _host(k_cache)
@@ -222,6 +268,22 @@ def verify_step(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, cand_to
     S_max = _host(k_cache)[0].shape[3]
     V = _host(logits)[0].shape[-1]
     acc = accept_path(am, cand_tokens, parent, prefix_len, V, S_max)
+    kc, vc = kv_compact(k_cache, v_cache, k_tree, v_tree, acc["path"], acc["accept_len"],
+                        prefix_len)
+    return dict(out=out, lse=lse, rowsum=rowsum, argmax=am, k_cache=kc, v_cache=vc, **acc)
+
+
+def verify_step_typical(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, cand_tokens,
+                        logits, temperature: float, epsilon: float, delta: float,
+                        scale: float = 0.0, units=None, n_threads: int = 0):
+    """The verification step with typical acceptance instead of exact matching:
+    attention, node argmax, typical acceptance and compaction, in that order."""
+    out, lse, rowsum, att_status = tree_attention(q, k_cache, v_cache, k_tree, v_tree,
+                                                  prefix_len, parent, scale, units, n_threads)
+    am = node_argmax(logits)
+    S_max = _host(k_cache)[0].shape[3]
+    acc = typical_accept(logits, am, cand_tokens, parent, prefix_len, S_max, temperature,
+                         epsilon, delta)
     kc, vc = kv_compact(k_cache, v_cache, k_tree, v_tree, acc["path"], acc["accept_len"],
                         prefix_len)
     return dict(out=out, lse=lse, rowsum=rowsum, argmax=am, k_cache=kc, v_cache=vc, **acc)

@@ -22,6 +22,9 @@
  *                          steps (2)-(3), exact matching)
  *   oracle_kv_compact      copy the accepted nodes' K/V into the cache
  *                          (Section 3 step (3), "KV cache is updated")
+ *   oracle_node_stats      log-sum-exp and entropy of softmax(logits / tau)
+ *   oracle_typical_accept  typical acceptance (Section 3 step (2), the
+ *                          second verification scheme the paper names)
  *
  * Status codes (per sequence): 0 ok, 3 malformed tree, 4 capacity / prefix
  * length out of range.  Whole-call argument errors return 1.
@@ -253,21 +256,74 @@ void oracle_node_argmax(const float *logits, int64_t rows, int64_t V, int32_t *o
 /* ------------------------------------------------------------------ accept */
 
 /*
- * Exact-matching acceptance of one tree per sequence.
- *
- * Node 0 (the root, the last accepted token) is always accepted.  A node i > 0
- * is accepted when it is a candidate token (cand[i] >= 0) equal to the top-1
- * token predicted at its parent, argmax[parent[i]], and its parent is
- * accepted (recursive definition along the parent pointer).  The chosen end
- * node is the accepted node of greatest depth, the smallest index among equal
- * depths; the path is its root path in depth order, accept_len its length
- * (root included), next_token the top-1 token at the end node and
- * new_prefix_len = prefix_len + accept_len.
- *
- * Errors (status 3: malformed tree or a token id outside [-1, V), root id
- * outside [0, V); status 4: prefix_len outside [0, S_max] or the path does
- * not fit in the cache) leave accept_len 0, path all -1, next_token -1 and
- * new_prefix_len = prefix_len.
+ * Checks shared by both acceptance rules for one sequence: status 3 for a
+ * malformed tree, a root id outside [0, V) or another id outside [-1, V);
+ * status 4 for a prefix length outside [0, S_max].
+ */
+static int check_sequence(const int32_t *par, const int32_t *tok, int T, int V, int P, int S_max)
+{
+    if (!tree_is_valid(par, T) || tok[0] < 0 || tok[0] >= V)
+        return ORC_ERR_TREE;
+    for (int i = 1; i < T; ++i)
+        if (tok[i] < -1 || tok[i] >= V)
+            return ORC_ERR_TREE;
+    if (P < 0 || P > S_max)
+        return ORC_ERR_CAPACITY;
+    return ORC_OK;
+}
+
+/*
+ * Given ok[i] (node i passes its verification test; ok[0] ignored) for a
+ * checked sequence (err == ORC_OK on entry), accept node 0 always and node
+ * i > 0 when ok[i] holds and its parent is accepted (recursive definition
+ * along the parent pointer).  The end node is the accepted node of greatest
+ * depth, the smallest index among equal depths; the path is its root path in
+ * depth order, accept_len its length (root included), next_token the top-1
+ * token at the end node and new_prefix_len = prefix_len + accept_len.  A path
+ * that does not fit in the cache is status 4.  On any error: accept_len 0,
+ * path all -1, next_token -1, new_prefix_len = prefix_len.
+ */
+static int choose_path(const int32_t *par, const int *ok, const int32_t *top, int T, int P,
+                       int S_max, int err, int *depth, int *acc, int32_t *pth,
+                       int32_t *accept_len, int32_t *next_token, int32_t *new_prefix_len)
+{
+    int best = 0;
+    if (err == ORC_OK) {
+        depth[0] = 0;
+        acc[0] = 1;
+        for (int i = 1; i < T; ++i) {
+            int p = par[i];
+            depth[i] = depth[p] + 1;
+            acc[i] = ok[i] && acc[p];
+        }
+        for (int i = 1; i < T; ++i)
+            if (acc[i] && depth[i] > depth[best])
+                best = i;
+        if ((int64_t)P + depth[best] + 1 > S_max)
+            err = ORC_ERR_CAPACITY;
+    }
+    for (int i = 0; i < T; ++i)
+        pth[i] = -1;
+    if (err != ORC_OK) {
+        *accept_len = 0;
+        *next_token = -1;
+        *new_prefix_len = P;
+    } else {
+        int n = depth[best] + 1;
+        int k = n - 1;
+        for (int a = best; a >= 0; a = par[a])
+            pth[k--] = a;
+        *accept_len = n;
+        *next_token = top[best];
+        *new_prefix_len = P + n;
+    }
+    return err;
+}
+
+/*
+ * Exact-matching acceptance of one tree per sequence: node i > 0 passes when
+ * it is a candidate token (cand[i] >= 0) equal to the top-1 token predicted at
+ * its parent, argmax[parent[i]].  Path choice and errors as in choose_path.
  */
 int oracle_accept_path(const int32_t *argmax, const int32_t *cand, const int32_t *parent,
                        const int32_t *prefix_len, int B, int T, int V, int S_max,
@@ -278,58 +334,126 @@ int oracle_accept_path(const int32_t *argmax, const int32_t *cand, const int32_t
         return ORC_ERR_INVALID_ARG;
     int *depth = (int *)malloc(sizeof(int) * (size_t)T);
     int *acc = (int *)malloc(sizeof(int) * (size_t)T);
+    int *ok = (int *)malloc(sizeof(int) * (size_t)T);
     for (int b = 0; b < B; ++b) {
         const int32_t *par = parent + (int64_t)b * T;
         const int32_t *tok = cand + (int64_t)b * T;
         const int32_t *top = argmax + (int64_t)b * T;
-        int32_t *pth = path + (int64_t)b * T;
         int P = prefix_len[b];
-        int err = ORC_OK;
-
-        if (!tree_is_valid(par, T) || tok[0] < 0 || tok[0] >= V)
-            err = ORC_ERR_TREE;
+        int err = check_sequence(par, tok, T, V, P, S_max);
+        ok[0] = 1;
         for (int i = 1; i < T && err == ORC_OK; ++i)
-            if (tok[i] < -1 || tok[i] >= V)
-                err = ORC_ERR_TREE;
-        if (err == ORC_OK && (P < 0 || P > S_max))
-            err = ORC_ERR_CAPACITY;
-
-        int best = 0;
-        if (err == ORC_OK) {
-            depth[0] = 0;
-            acc[0] = 1;
-            for (int i = 1; i < T; ++i) {
-                int p = par[i];
-                depth[i] = depth[p] + 1;
-                int ok = tok[i] >= 0 && tok[i] == top[p];
-                acc[i] = ok && acc[p];
-            }
-            for (int i = 1; i < T; ++i)
-                if (acc[i] && depth[i] > depth[best])
-                    best = i;
-            if ((int64_t)P + depth[best] + 1 > S_max)
-                err = ORC_ERR_CAPACITY;
-        }
-
-        for (int i = 0; i < T; ++i)
-            pth[i] = -1;
-        if (err != ORC_OK) {
-            accept_len[b] = 0;
-            next_token[b] = -1;
-            new_prefix_len[b] = P;
-        } else {
-            int n = depth[best] + 1;
-            int k = n - 1;
-            for (int a = best; a >= 0; a = par[a])
-                pth[k--] = a;
-            accept_len[b] = n;
-            next_token[b] = top[best];
-            new_prefix_len[b] = P + n;
-        }
-        status[b] = err;
+            ok[i] = tok[i] >= 0 && tok[i] == top[par[i]];
+        status[b] = choose_path(par, ok, top, T, P, S_max, err, depth, acc, path + (int64_t)b * T,
+                                accept_len + b, next_token + b, new_prefix_len + b);
     }
     free(depth);
     free(acc);
+    free(ok);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------ typical acceptance */
+
+/*
+ * Statistics of the distribution p = softmax(x / tau) of each logits row
+ * [rows, V] (fp32), tau > 0: lse = log sum_v exp(x_v / tau) and the entropy
+ * H = -sum_v p_v log p_v, with p_v = exp(x_v / tau - lse).  Written as
+ * defined, max-shifted, in fp64; a row holding a NaN gets NaN for both.
+ */
+void oracle_node_stats(const float *logits, int64_t rows, int64_t V, double tau, double *lse,
+                       double *entropy)
+{
+    for (int64_t r = 0; r < rows; ++r) {
+        const float *x = logits + r * V;
+        int has_nan = 0;
+        double m = -INFINITY;
+        for (int64_t v = 0; v < V; ++v) {
+            if (isnan(x[v]))
+                has_nan = 1;
+            else if ((double)x[v] / tau > m)
+                m = (double)x[v] / tau;
+        }
+        if (has_nan) {
+            lse[r] = NAN;
+            entropy[r] = NAN;
+            continue;
+        }
+        double s = 0.0;
+        for (int64_t v = 0; v < V; ++v)
+            s += exp((double)x[v] / tau - m);
+        double l = m + log(s);
+        double h = 0.0;
+        for (int64_t v = 0; v < V; ++v) {
+            double pv = exp((double)x[v] / tau - l);
+            if (pv > 0.0)
+                h -= pv * ((double)x[v] / tau - l);
+        }
+        lse[r] = l;
+        entropy[r] = h;
+    }
+}
+
+/*
+ * Typical acceptance of one tree per sequence (the paper names it in Section 3
+ * step (2) as its second verification scheme and gives no formula; this is
+ * the usual form of that rule).  With p = softmax(logits[parent[i]] / tau)
+ * and H its entropy, node i > 0 passes when it is a candidate token t =
+ * cand[i] >= 0 with
+ *     p_t > min(epsilon, delta * exp(-H)).
+ * Path choice and errors as in choose_path (next_token is still the top-1
+ * token at the end node).  p_tok and threshold [B,T] receive p_t and the
+ * right-hand side for every candidate node of a checked sequence and NaN
+ * elsewhere.  tau must be positive.
+ */
+int oracle_typical_accept(const float *logits, const int32_t *argmax, const int32_t *cand,
+                          const int32_t *parent, const int32_t *prefix_len, int B, int T, int V,
+                          int S_max, double tau, double epsilon, double delta,
+                          int32_t *accept_len, int32_t *path, int32_t *next_token,
+                          int32_t *new_prefix_len, int32_t *status, double *p_tok,
+                          double *threshold)
+{
+    if (B < 1 || T < 1 || V < 1 || !(tau > 0.0))
+        return ORC_ERR_INVALID_ARG;
+    int *depth = (int *)malloc(sizeof(int) * (size_t)T);
+    int *acc = (int *)malloc(sizeof(int) * (size_t)T);
+    int *ok = (int *)malloc(sizeof(int) * (size_t)T);
+    double *lse = (double *)malloc(sizeof(double) * (size_t)T);
+    double *ent = (double *)malloc(sizeof(double) * (size_t)T);
+    for (int b = 0; b < B; ++b) {
+        const int32_t *par = parent + (int64_t)b * T;
+        const int32_t *tok = cand + (int64_t)b * T;
+        const int32_t *top = argmax + (int64_t)b * T;
+        const float *x = logits + (int64_t)b * T * V;
+        int P = prefix_len[b];
+        int err = check_sequence(par, tok, T, V, P, S_max);
+        for (int i = 0; i < T; ++i) {
+            p_tok[(int64_t)b * T + i] = NAN;
+            threshold[(int64_t)b * T + i] = NAN;
+        }
+        ok[0] = 1;
+        if (err == ORC_OK) {
+            oracle_node_stats(x, T, V, tau, lse, ent);
+            for (int i = 1; i < T; ++i) {
+                ok[i] = 0;
+                if (tok[i] < 0)
+                    continue;
+                int p = par[i];
+                double pt = exp((double)x[(int64_t)p * V + tok[i]] / tau - lse[p]);
+                double th = fmin(epsilon, delta * exp(-ent[p]));
+                p_tok[(int64_t)b * T + i] = pt;
+                threshold[(int64_t)b * T + i] = th;
+                ok[i] = pt > th;
+            }
+        }
+        status[b] = choose_path(par, ok, top, T, P, S_max, err, depth, acc, path + (int64_t)b * T,
+                                accept_len + b, next_token + b, new_prefix_len + b);
+    }
+    free(depth);
+    free(acc);
+    free(ok);
+    free(lse);
+    free(ent);
     return ORC_OK;
 }
 
