@@ -39,6 +39,7 @@ METRIC = "verify steps/s and achieved HBM GB/s (frac of ~8 TB/s), Vicuna-7B shap
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 256 << 20
+TYPICAL = (0.7, 0.09, 0.3)   # temperature, epsilon, delta of --accept typical
 L2_BYTES = 129 * 1000 * 1000
 
 # DRAM traffic of one tree-attention launch (dram__bytes_read.sum +
@@ -204,6 +205,9 @@ def parse():
                     help="seconds of oracle work in the CPU baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--accept", default="exact", choices=["exact", "typical"],
+                    help="verification rule: exact matching, or typical acceptance at "
+                         "temperature 0.7, epsilon 0.09, delta 0.3")
     ap.add_argument("--layers", type=int, default=0,
                     help="run the workload with this many layers (profiling captures)")
     ap.add_argument("--l2", default="auto", choices=["auto", "flush", "none"],
@@ -315,10 +319,17 @@ def main():
             flush.zero_()
 
     def step():
-        ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
-                            parent, cand, logits, bufs.out, bufs.argmax, bufs.accept_len, bufs.path,
-                            bufs.next_token, bufs.new_prefix_len, bufs.dev_status, bufs.workspace,
-                            stream=stream)
+        if args.accept == "typical":
+            ppd.ppd_verify_step_typical(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
+                                        prefix, parent, cand, logits, *TYPICAL, bufs.out,
+                                        bufs.argmax, bufs.accept_len, bufs.path, bufs.next_token,
+                                        bufs.new_prefix_len, bufs.dev_status, bufs.workspace,
+                                        stream=stream)
+        else:
+            ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
+                                parent, cand, logits, bufs.out, bufs.argmax, bufs.accept_len,
+                                bufs.path, bufs.next_token, bufs.new_prefix_len, bufs.dev_status,
+                                bufs.workspace, stream=stream)
 
     for _ in range(max(3, args.warmup)):
         maybe_flush()
@@ -391,11 +402,14 @@ def main():
         def e2e_step():
             for k, v in h_in.items():
                 d_in[k].copy_(v, non_blocking=True)
-            ppd.ppd_verify_step(d_in["q"], t["k_cache"], t["v_cache"], d_in["k_tree"],
-                                d_in["v_tree"], d_in["prefix"], d_in["parent"], d_in["cand"],
-                                d_in["logits"], bufs.out, bufs.argmax, bufs.accept_len, bufs.path,
-                                bufs.next_token, bufs.new_prefix_len, bufs.dev_status,
-                                bufs.workspace, stream=stream)
+            common = (d_in["q"], t["k_cache"], t["v_cache"], d_in["k_tree"], d_in["v_tree"],
+                      d_in["prefix"], d_in["parent"], d_in["cand"], d_in["logits"])
+            outs_ = (bufs.out, bufs.argmax, bufs.accept_len, bufs.path, bufs.next_token,
+                     bufs.new_prefix_len, bufs.dev_status, bufs.workspace)
+            if args.accept == "typical":
+                ppd.ppd_verify_step_typical(*common, *TYPICAL, *outs_, stream=stream)
+            else:
+                ppd.ppd_verify_step(*common, *outs_, stream=stream)
             for k in outs:
                 h_out[k].copy_(getattr(bufs, k), non_blocking=True)
             stream.synchronize()
@@ -436,7 +450,10 @@ def main():
                               if do_flush else
                               f"not flushed: inputs larger than L2 ({footprint / 1e6:.0f} MB "
                               f"streamed per step, L2 {L2_BYTES / 1e6:.0f} MB)"),
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": f"replicas x{world}",
+                       "accept": ("exact matching" if args.accept == "exact" else
+                                  "typical acceptance (temperature %g, epsilon %g, delta %g)"
+                                  % TYPICAL)},
             "ms_per_step_p10_p50_p90": [float(q10), float(q50), float(q90)],
             "step_gbs": sb / (ms_per_step * 1e-3) / 1e9,
             "step_frac_of_8tbs": sb / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS,

@@ -73,7 +73,8 @@ typedef enum { PPD_BF16 = 0, PPD_F32 = 1 } ppd_dtype;
  * Scratch bytes the entry points below need in `workspace` for these sizes
  * (device memory, any contents, 256-byte aligned, caller-owned; it may be
  * reused between calls that are ordered on one stream).  Covers the per-split
- * partial maxima of the node argmax and, for PPD_F32, the bf16 copies of Q/K/V.
+ * partial maxima (and softmax statistics) of the node argmax, the fused step's
+ * per-CTA scratch and, for PPD_F32, the bf16 copies of Q/K/V.
  */
 size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt);
 
@@ -159,6 +160,59 @@ ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
                            int32_t *accept_len, int32_t *path, int32_t *next_token,
                            int32_t *new_prefix_len, int32_t *dev_status,
                            void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Node softmax statistics for typical acceptance (Section 3 step (2): the
+ * paper's second verification scheme, typical acceptance, tests each candidate
+ * against the distribution predicted at its parent).  For every row of logits
+ * fp32 [B,T,V], with p = softmax(logits / temperature):
+ *   argmax_out  int32 [B,T]  top-1 index (lowest index on ties, first NaN wins)
+ *   lse_out     fp32 [B,T]   log sum_v exp(logits_v / temperature)
+ *   entropy_out fp32 [B,T]   -sum_v p_v log p_v (natural log)
+ * A row holding a NaN gives NaN statistics.  temperature > 0.  One pass over the
+ * logits.  Workspace: ppd_workspace_bytes(...) bytes.
+ */
+ppd_status ppd_node_stats(const float *logits, int B, int T, int V, float temperature,
+                          int32_t *argmax_out, float *lse_out, float *entropy_out,
+                          void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Typical acceptance (Section 3 steps (2)-(3); the paper names the scheme and
+ * gives no formula, so the rule below is the one this library adopts).  Node 0
+ * is always accepted; node i > 0 with parent j and candidate token
+ * t = cand_tokens[b][i] >= 0 is accepted when its parent is accepted and
+ *     p_t > min(epsilon, delta * exp(-H_j)),
+ * where p = softmax(logits[b][j] / temperature) and H_j its entropy, taken from
+ * lse / entropy (as written by ppd_node_stats at the same temperature).  Path
+ * choice (deepest accepted node, smallest index among equal depths), outputs and
+ * errors as in ppd_accept_path; next_token is the argmax at the end node.
+ *   logits fp32 [B,T,V]; lse, entropy fp32 [B,T]; argmax, cand_tokens, parent
+ *   int32 [B,T]; prefix_len int32 [B].  temperature > 0; epsilon, delta finite.
+ * A decision whose two sides agree to within float rounding may differ from a
+ * higher-precision evaluation.
+ */
+ppd_status ppd_typical_accept(const float *logits, const float *lse, const float *entropy,
+                              const int32_t *argmax, const int32_t *cand_tokens,
+                              const int32_t *parent, const int32_t *prefix_len, int B, int T,
+                              int V, int S_max, float temperature, float epsilon, float delta,
+                              int32_t *accept_len, int32_t *path, int32_t *next_token,
+                              int32_t *new_prefix_len, int32_t *dev_status, void *stream);
+
+/*
+ * The verification step with typical acceptance in place of exact matching:
+ * ppd_verify_step's arguments plus temperature, epsilon and delta of
+ * ppd_typical_accept.  argmax_out still receives every node's top-1 token.
+ */
+ppd_status ppd_verify_step_typical(const void *q, void *k_cache, void *v_cache,
+                                   const void *k_tree, const void *v_tree,
+                                   const int32_t *prefix_len, const int32_t *parent,
+                                   const int32_t *cand_tokens, const float *logits,
+                                   int L, int B, int H, int T, int D, int V, int S_max,
+                                   ppd_dtype dt, float scale, float temperature, float epsilon,
+                                   float delta, float *out, float *lse, int32_t *argmax_out,
+                                   int32_t *accept_len, int32_t *path, int32_t *next_token,
+                                   int32_t *new_prefix_len, int32_t *dev_status,
+                                   void *workspace, size_t ws_bytes, void *stream);
 
 /*
  * Node argmax without a workspace (no paper counterpart; an interface for

@@ -38,6 +38,83 @@ PPD_DEV int combine_partials(const float *part_val, const int32_t *part_idx, int
     return bi;
 }
 
+// ------------------------------------------------------------------ softmax statistics
+//
+// Running statistics of the distribution softmax(x / tau) over a stream of
+// logits, kept in base-2 units y = x * k with k = log2(e) / tau:
+//   m = max y,  s = sum 2^(y - m),  t = sum 2^(y - m) * (y - m).
+// Then lse = ln2 * (m + log2 s) is log sum exp(x / tau) and the entropy is
+// H = ln2 * (log2 s - t / s).  A NaN anywhere makes s (and so both) NaN;
+// -inf logits contribute nothing.
+struct SoftStats {
+    float m = -INFINITY, s = 0.f, t = 0.f;
+};
+
+// Fold four scaled logits into st.
+PPD_DEV void stats_add4(SoftStats &st, float y0, float y1, float y2, float y3)
+{
+    const float mg = fmaxf(fmaxf(y0, y1), fmaxf(y2, y3));
+    if (mg > st.m) {
+        if (st.s != 0.f) {
+            const float a = ex2(st.m - mg);
+            st.t = a * (st.t + (st.m - mg) * st.s);
+            st.s *= a;
+        }
+        st.m = mg;
+    }
+    const float y[4] = {y0, y1, y2, y3};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float d = y[k] - st.m;
+        const float e = (y[k] == -INFINITY) ? 0.f : ex2(d);
+        st.s += e;
+        st.t += (e > 0.f) ? e * d : ((e == e) ? 0.f : e);
+    }
+}
+
+// st <- st (+) o.
+PPD_DEV void stats_merge(SoftStats &st, const SoftStats &o)
+{
+    const float M = fmaxf(st.m, o.m);
+    float s = 0.f, t = 0.f;
+    if (st.s != 0.f) {
+        const float a = ex2(st.m - M);
+        s += a * st.s;
+        t += a * (st.t + (st.m - M) * st.s);
+    }
+    if (o.s != 0.f) {
+        const float a = ex2(o.m - M);
+        s += a * o.s;
+        t += a * (o.t + (o.m - M) * o.s);
+    }
+    st.m = M;
+    st.s = s;
+    st.t = t;
+}
+
+// Statistics of one row from its `splits` partial (m, s, t) triples.
+PPD_DEV SoftStats combine_stats(const float *part_stats, int64_t row, int splits)
+{
+    SoftStats st;
+    for (int k = 0; k < splits; ++k) {
+        const float *ps = part_stats + 3 * (row * splits + k);
+        SoftStats o;
+        o.m = __ldcg(ps);
+        o.s = __ldcg(ps + 1);
+        o.t = __ldcg(ps + 2);
+        stats_merge(st, o);
+    }
+    return st;
+}
+
+// Natural-log log-sum-exp and entropy from the statistics.
+PPD_DEV void stats_finish(const SoftStats &st, float &lse, float &entropy)
+{
+    const float l2s = __log2f(st.s);
+    lse = 0.69314718055994530942f * (st.m + l2s);
+    entropy = 0.69314718055994530942f * (l2s - st.t / st.s);
+}
+
 struct AcceptResult {
     int n_acc;           // accepted tokens, root included; 0 on error
     int next_token;      // top-1 token at the end node; -1 on error
@@ -45,17 +122,21 @@ struct AcceptResult {
     int status;          // kOk, kErrTree or kErrCapacity
 };
 
-// Exact-matching acceptance of one sequence by one warp (all lanes call it).
+// Acceptance of one sequence by one warp (all lanes call it).
 //   top     the sequence's T top-1 tokens (node i: the model's prediction after i)
+//   pass    pass(i, parent, token): does candidate node i (token >= 0) pass its
+//           verification test
 //   par,tok the sequence's parent array and candidate token ids (global memory)
-//   s_par   T ints of per-warp shared scratch
+//   s_par   T ints of per-warp scratch
 //   path    T outputs: accepted nodes in depth order, then -1
-// Node 0 is always accepted; node i > 0 when tok[i] >= 0 equals top[par[i]] and
-// its parent is accepted.  The end node is the deepest accepted node, the
-// smallest index among equal depths.  Every lane gets the same result.
-template <class TopLoad>
-PPD_DEV AcceptResult accept_warp(TopLoad top, const int32_t *par, const int32_t *tok, int P,
-                                 int T, int V, int S_max, int lane, int *s_par, int32_t *path)
+// Node 0 is always accepted; node i > 0 when tok[i] >= 0, pass(i, par[i],
+// tok[i]) holds and its parent is accepted.  The end node is the deepest
+// accepted node, the smallest index among equal depths.  Every lane gets the
+// same result.
+template <class TopLoad, class Pass>
+PPD_DEV AcceptResult accept_warp_pass(TopLoad top, Pass pass, const int32_t *par,
+                                      const int32_t *tok, int P, int T, int V, int S_max, int lane,
+                                      int *s_par, int32_t *path)
 {
     bool bad = false;
 #pragma unroll
@@ -85,7 +166,7 @@ PPD_DEV AcceptResult accept_warp(TopLoad top, const int32_t *par, const int32_t 
                 ok = true;
             } else {
                 const int tk = __ldg(tok + i);
-                ok = tk >= 0 && tk == top(s_par[i]);
+                ok = tk >= 0 && pass(i, s_par[i], tk);
             }
         }
         okw[k] = __ballot_sync(0xffffffffu, ok);
@@ -134,6 +215,37 @@ PPD_DEV AcceptResult accept_warp(TopLoad top, const int32_t *par, const int32_t 
     r.status = err;
     __syncwarp();
     return r;
+}
+
+// Exact matching (Section 3 step (2)): a candidate passes when it equals the
+// top-1 token predicted at its parent.
+template <class TopLoad>
+PPD_DEV AcceptResult accept_warp(TopLoad top, const int32_t *par, const int32_t *tok, int P, int T,
+                                 int V, int S_max, int lane, int *s_par, int32_t *path)
+{
+    return accept_warp_pass(
+        top, [&](int, int pa, int tk) { return tk == top(pa); }, par, tok, P, T, V, S_max, lane,
+        s_par, path);
+}
+
+// Typical acceptance (Section 3 step (2), the second scheme the paper names):
+// a candidate t below node j passes when p_t > min(epsilon, delta * exp(-H_j)),
+// with p = softmax(logits[j] / tau), from the natural-log log-sum-exp lse[j]
+// and entropy ent[j] of that distribution.  `x` is the sequence's logits
+// [T][V]; lse / ent load node j's values.
+template <class TopLoad, class Lse, class Ent>
+PPD_DEV AcceptResult accept_warp_typical(TopLoad top, const float *x, Lse lse, Ent ent,
+                                         float inv_temp, float epsilon, float delta,
+                                         const int32_t *par, const int32_t *tok, int P, int T,
+                                         int V, int S_max, int lane, int *s_par, int32_t *path)
+{
+    return accept_warp_pass(
+        top,
+        [&](int, int pa, int tk) {
+            const float pt = expf(__ldg(x + (size_t)pa * V + tk) * inv_temp - lse(pa));
+            return pt > fminf(epsilon, delta * expf(-ent(pa)));
+        },
+        par, tok, P, T, V, S_max, lane, s_par, path);
 }
 
 }  // namespace ppd

@@ -50,7 +50,7 @@ int num_sms()
 int argmax_splits(int64_t rows, int V) { return ppd::argmax_split_count(rows, V); }
 
 struct WsLayout {
-    size_t part_val, part_idx, side, conv, total;
+    size_t part_val, part_idx, part_stats, node_lse, node_ent, side, conv, total;
     int splits;
 };
 
@@ -64,6 +64,12 @@ WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, p
     off = align_up(off + (size_t)rows * w.splits * 4);
     w.part_idx = off;
     off = align_up(off + (size_t)rows * w.splits * 4);
+    w.part_stats = off;   // softmax statistics partials (typical acceptance)
+    off = align_up(off + (size_t)rows * w.splits * 12);
+    w.node_lse = off;
+    off = align_up(off + (size_t)rows * 4);
+    w.node_ent = off;
+    off = align_up(off + (size_t)rows * 4);
     w.side = off;
     off = align_up(off + (size_t)num_sms() * ppd::kSideScratchInts * 4);
     w.conv = off;
@@ -209,6 +215,119 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
 
 }  // namespace
 
+// Parameters of typical acceptance (null: exact matching).
+struct TypicalParams {
+    float temperature, epsilon, delta;
+};
+
+static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
+                                   const void *k_tree, const void *v_tree,
+                                   const int32_t *prefix_len, const int32_t *parent,
+                                   const int32_t *cand_tokens, const float *logits, int L, int B,
+                                   int H, int T, int D, int V, int S_max, ppd_dtype dt, float scale,
+                                   const TypicalParams *typ, float *out, float *lse,
+                                   int32_t *argmax_out, int32_t *accept_len, int32_t *path,
+                                   int32_t *next_token, int32_t *new_prefix_len,
+                                   int32_t *dev_status, void *workspace, size_t ws_bytes,
+                                   void *stream)
+{
+    if (!q || !k_cache || !v_cache || !k_tree || !v_tree || !prefix_len || !parent ||
+        !cand_tokens || !logits || !out || !argmax_out || !accept_len || !path || !next_token ||
+        !new_prefix_len || !dev_status || !workspace)
+        return PPD_ERR_INVALID_ARG;
+    if (!attn_dims_ok(L, B, H, T, D, S_max, dt) || V < 1 || !std::isfinite(scale))
+        return PPD_ERR_INVALID_ARG;
+    if ((double)B * T * V > 9.0e15) return PPD_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(k_tree, 16) ||
+        !aligned(v_tree, 16) || !aligned(out, 4) || !aligned(lse, 4))
+        return PPD_ERR_INVALID_ARG;
+    const int eb = dt == PPD_BF16 ? 2 : 4;
+    const size_t lbh = (size_t)L * B * H;
+    const size_t nc = lbh * S_max * D * eb, nt = lbh * T * D * eb;
+    if (overlaps(k_cache, nc, k_tree, nt) || overlaps(k_cache, nc, v_tree, nt) ||
+        overlaps(v_cache, nc, k_tree, nt) || overlaps(v_cache, nc, v_tree, nt) ||
+        overlaps(k_cache, nc, v_cache, nc))
+        return PPD_ERR_INVALID_ARG;
+    const WsLayout wl = workspace_layout(L, B, H, T, D, V, S_max, dt);
+    if (ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    float *pv = reinterpret_cast<float *>(ws + wl.part_val);
+    int32_t *pi = reinterpret_cast<int32_t *>(ws + wl.part_idx);
+    float *pst = typ ? reinterpret_cast<float *>(ws + wl.part_stats) : nullptr;
+    const float temp = typ ? typ->temperature : 1.f;
+    const int64_t rows = (int64_t)B * T;
+
+    if (B <= ppd::kFusedMaxB) {
+        // 1. partial maxima (and statistics) of every node's logits; also zeroes dev_status
+        if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temp, dev_status, B,
+                                        s) != cudaSuccess)
+            return PPD_ERR_CUDA;
+        // 2. attention over every layer, overlapping step 1; its end phase combines
+        //    the argmax, decides acceptance and compacts the accepted rows
+        ppd::FusedStep f{};
+        f.part_val = pv;
+        f.part_idx = pi;
+        f.splits = wl.splits;
+        f.cand_tokens = cand_tokens;
+        f.argmax_out = argmax_out;
+        f.accept_len = accept_len;
+        f.path = path;
+        f.next_token = next_token;
+        f.new_prefix_len = new_prefix_len;
+        f.status = dev_status;
+        f.k_cache = static_cast<uint8_t *>(k_cache);
+        f.v_cache = static_cast<uint8_t *>(v_cache);
+        f.k_tree = static_cast<const uint8_t *>(k_tree);
+        f.v_tree = static_cast<const uint8_t *>(v_tree);
+        f.row_bytes = D * eb;
+        f.V = V;
+        f.scratch = reinterpret_cast<int *>(ws + wl.side);
+        if (typ) {
+            f.typical = 1;
+            f.part_stats = pst;
+            f.logits = logits;
+            f.inv_temp = 1.f / typ->temperature;
+            f.epsilon = typ->epsilon;
+            f.delta = typ->delta;
+        }
+        return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B,
+                                     H, T, D, S_max, dt, scale, out, lse, nullptr, ws, wl, &f, s);
+    }
+
+    // large batches: the same steps as separate grids
+    AcceptArgs a{cand_tokens, parent, prefix_len, accept_len, path, next_token, new_prefix_len,
+                 dev_status, T, V, S_max};
+    if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temp, nullptr, 0, s) !=
+        cudaSuccess)
+        return PPD_ERR_CUDA;
+    if (typ) {
+        float *nl = reinterpret_cast<float *>(ws + wl.node_lse);
+        float *ne = reinterpret_cast<float *>(ws + wl.node_ent);
+        if (ppd::launch_node_stats_combine(pv, pi, pst, rows, wl.splits, argmax_out, nl, ne, s) !=
+                cudaSuccess ||
+            ppd::launch_typical_accept(logits, nl, ne, argmax_out, a, B, typ->temperature,
+                                       typ->epsilon, typ->delta, s) != cudaSuccess)
+            return PPD_ERR_CUDA;
+    } else {
+        if (ppd::launch_argmax_combine(pv, pi, rows, wl.splits, argmax_out, s) != cudaSuccess ||
+            ppd::launch_accept_path(argmax_out, a, B, s) != cudaSuccess)
+            return PPD_ERR_CUDA;
+    }
+    ppd_status st = enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent,
+                                          L, B, H, T, D, S_max, dt, scale, out, lse, dev_status,
+                                          ws, wl, nullptr, s);
+    if (st != PPD_OK) return st;
+    return cuda_status(ppd::launch_kv_compact(k_cache, v_cache, k_tree, v_tree, path, accept_len,
+                                              prefix_len, L, B, H, T, D, S_max, eb, s));
+}
+
+static bool typical_params_ok(float temperature, float epsilon, float delta)
+{
+    return std::isfinite(temperature) && temperature > 0.f && std::isfinite(epsilon) &&
+           std::isfinite(delta) && std::isfinite(1.f / temperature);
+}
+
 extern "C" {
 
 size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt)
@@ -267,7 +386,8 @@ ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *ar
     float *pv = reinterpret_cast<float *>(ws + wl.part_val);
     int32_t *pi = reinterpret_cast<int32_t *>(ws + wl.part_idx);
     const int64_t rows = (int64_t)B * T;
-    if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, nullptr, 0, s) != cudaSuccess)
+    if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, nullptr, 1.f, nullptr, 0, s) !=
+        cudaSuccess)
         return PPD_ERR_CUDA;
     return cuda_status(ppd::launch_argmax_combine(pv, pi, rows, wl.splits, argmax_out, s));
 }
@@ -321,73 +441,72 @@ ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
                            int32_t *new_prefix_len, int32_t *dev_status,
                            void *workspace, size_t ws_bytes, void *stream)
 {
-    if (!q || !k_cache || !v_cache || !k_tree || !v_tree || !prefix_len || !parent ||
-        !cand_tokens || !logits || !out || !argmax_out || !accept_len || !path || !next_token ||
-        !new_prefix_len || !dev_status || !workspace)
+    return verify_step_impl(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, cand_tokens,
+                            logits, L, B, H, T, D, V, S_max, dt, scale, nullptr, out, lse,
+                            argmax_out, accept_len, path, next_token, new_prefix_len, dev_status,
+                            workspace, ws_bytes, stream);
+}
+
+ppd_status ppd_verify_step_typical(const void *q, void *k_cache, void *v_cache,
+                                   const void *k_tree, const void *v_tree,
+                                   const int32_t *prefix_len, const int32_t *parent,
+                                   const int32_t *cand_tokens, const float *logits,
+                                   int L, int B, int H, int T, int D, int V, int S_max,
+                                   ppd_dtype dt, float scale, float temperature, float epsilon,
+                                   float delta, float *out, float *lse, int32_t *argmax_out,
+                                   int32_t *accept_len, int32_t *path, int32_t *next_token,
+                                   int32_t *new_prefix_len, int32_t *dev_status,
+                                   void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!typical_params_ok(temperature, epsilon, delta)) return PPD_ERR_INVALID_ARG;
+    const TypicalParams typ{temperature, epsilon, delta};
+    return verify_step_impl(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, cand_tokens,
+                            logits, L, B, H, T, D, V, S_max, dt, scale, &typ, out, lse,
+                            argmax_out, accept_len, path, next_token, new_prefix_len, dev_status,
+                            workspace, ws_bytes, stream);
+}
+
+ppd_status ppd_node_stats(const float *logits, int B, int T, int V, float temperature,
+                          int32_t *argmax_out, float *lse_out, float *entropy_out,
+                          void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!logits || !argmax_out || !lse_out || !entropy_out || B < 1 || T < 1 || V < 1)
         return PPD_ERR_INVALID_ARG;
-    if (!attn_dims_ok(L, B, H, T, D, S_max, dt) || V < 1 || !std::isfinite(scale))
+    if (!std::isfinite(temperature) || !(temperature > 0.f) || !std::isfinite(1.f / temperature))
         return PPD_ERR_INVALID_ARG;
-    if ((double)B * T * V > 9.0e15) return PPD_ERR_INVALID_ARG;
-    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(k_tree, 16) ||
-        !aligned(v_tree, 16) || !aligned(out, 4) || !aligned(lse, 4))
-        return PPD_ERR_INVALID_ARG;
-    const int eb = dt == PPD_BF16 ? 2 : 4;
-    const size_t lbh = (size_t)L * B * H;
-    const size_t nc = lbh * S_max * D * eb, nt = lbh * T * D * eb;
-    if (overlaps(k_cache, nc, k_tree, nt) || overlaps(k_cache, nc, v_tree, nt) ||
-        overlaps(v_cache, nc, k_tree, nt) || overlaps(v_cache, nc, v_tree, nt) ||
-        overlaps(k_cache, nc, v_cache, nc))
-        return PPD_ERR_INVALID_ARG;
-    const WsLayout wl = workspace_layout(L, B, H, T, D, V, S_max, dt);
-    if (ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
+    if ((double)B * T * V > 9.0e15 || (double)B * T * 64 > 2147483647.0) return PPD_ERR_INVALID_ARG;
+    const WsLayout wl = workspace_layout(1, B, 1, T, 1, V, 0, PPD_BF16);
+    if (!workspace || ws_bytes < wl.total || !aligned(workspace, kAlign)) return PPD_ERR_INVALID_ARG;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     float *pv = reinterpret_cast<float *>(ws + wl.part_val);
     int32_t *pi = reinterpret_cast<int32_t *>(ws + wl.part_idx);
+    float *pst = reinterpret_cast<float *>(ws + wl.part_stats);
     const int64_t rows = (int64_t)B * T;
-
-    if (B <= ppd::kFusedMaxB) {
-        // 1. partial maxima of every node's logits (also zeroes dev_status)
-        if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, dev_status, B, s) !=
-            cudaSuccess)
-            return PPD_ERR_CUDA;
-        // 2. attention over every layer, overlapping step 1; its end phase combines
-        //    the argmax, decides acceptance and compacts the accepted rows
-        ppd::FusedStep f{};
-        f.part_val = pv;
-        f.part_idx = pi;
-        f.splits = wl.splits;
-        f.cand_tokens = cand_tokens;
-        f.argmax_out = argmax_out;
-        f.accept_len = accept_len;
-        f.path = path;
-        f.next_token = next_token;
-        f.new_prefix_len = new_prefix_len;
-        f.status = dev_status;
-        f.k_cache = static_cast<uint8_t *>(k_cache);
-        f.v_cache = static_cast<uint8_t *>(v_cache);
-        f.k_tree = static_cast<const uint8_t *>(k_tree);
-        f.v_tree = static_cast<const uint8_t *>(v_tree);
-        f.row_bytes = D * eb;
-        f.V = V;
-        f.scratch = reinterpret_cast<int *>(ws + wl.side);
-        return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B,
-                                     H, T, D, S_max, dt, scale, out, lse, nullptr, ws, wl, &f, s);
-    }
-
-    // large batches: the same steps as separate grids
-    if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, nullptr, 0, s) != cudaSuccess ||
-        ppd::launch_argmax_combine(pv, pi, rows, wl.splits, argmax_out, s) != cudaSuccess)
+    if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temperature, nullptr, 0,
+                                    s) != cudaSuccess)
         return PPD_ERR_CUDA;
+    return cuda_status(ppd::launch_node_stats_combine(pv, pi, pst, rows, wl.splits, argmax_out,
+                                                      lse_out, entropy_out, s));
+}
+
+ppd_status ppd_typical_accept(const float *logits, const float *lse, const float *entropy,
+                              const int32_t *argmax, const int32_t *cand_tokens,
+                              const int32_t *parent, const int32_t *prefix_len, int B, int T,
+                              int V, int S_max, float temperature, float epsilon, float delta,
+                              int32_t *accept_len, int32_t *path, int32_t *next_token,
+                              int32_t *new_prefix_len, int32_t *dev_status, void *stream)
+{
+    if (!logits || !lse || !entropy || !argmax || !cand_tokens || !parent || !prefix_len ||
+        !accept_len || !path || !next_token || !new_prefix_len || !dev_status)
+        return PPD_ERR_INVALID_ARG;
+    if (B < 1 || T < 1 || T > kMaxT || V < 1 || S_max < 0) return PPD_ERR_INVALID_ARG;
+    if (!typical_params_ok(temperature, epsilon, delta)) return PPD_ERR_INVALID_ARG;
+    if ((double)B * T * V > 9.0e15) return PPD_ERR_INVALID_ARG;
     AcceptArgs a{cand_tokens, parent, prefix_len, accept_len, path, next_token, new_prefix_len,
                  dev_status, T, V, S_max};
-    if (ppd::launch_accept_path(argmax_out, a, B, s) != cudaSuccess) return PPD_ERR_CUDA;
-    ppd_status st = enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent,
-                                          L, B, H, T, D, S_max, dt, scale, out, lse, dev_status,
-                                          ws, wl, nullptr, s);
-    if (st != PPD_OK) return st;
-    return cuda_status(ppd::launch_kv_compact(k_cache, v_cache, k_tree, v_tree, path, accept_len,
-                                              prefix_len, L, B, H, T, D, S_max, eb, s));
+    return cuda_status(ppd::launch_typical_accept(logits, lse, entropy, argmax, a, B, temperature,
+                                                  epsilon, delta, static_cast<cudaStream_t>(stream)));
 }
 
 ppd_status ppd_selftest_umma(const void *a, const void *b, float *d, int mode, int N, void *stream)

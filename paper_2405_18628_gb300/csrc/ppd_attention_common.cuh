@@ -71,6 +71,8 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
     int *s_par = f.scratch + (size_t)blockIdx.x * kSideScratchInts;
     int *top = s_par + 128;
     int *path = top + 128;
+    float *s_lse = reinterpret_cast<float *>(path + 128);
+    float *s_ent = s_lse + 128;
     const int chunks = f.row_bytes >> 4;
     for (int b = 0; b < B; ++b) {
         const bool designated = (b % (int)gridDim.x) == (int)blockIdx.x;
@@ -86,12 +88,19 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
             for (int k = 1; k < S; ++k) consider(__ldcg(f.part_val + base + k), __ldcg(f.part_idx + base + k), bv, bi);
             top[r] = bi;
             if (designated) f.argmax_out[(size_t)b * T + r] = bi;
+            if (f.typical) stats_finish(combine_stats(f.part_stats, (int64_t)b * T + r, S), s_lse[r], s_ent[r]);
         }
         __syncwarp();
+        const auto top_of = [&](int n) { return top[n]; };
         const AcceptResult res =
-            accept_warp([&](int n) { return top[n]; }, p.parent + (size_t)b * T,
-                        f.cand_tokens + (size_t)b * T, __ldg(p.prefix_len + b), T, f.V, p.S_max,
-                        lane, s_par, path);
+            f.typical
+                ? accept_warp_typical(top_of, f.logits + (size_t)b * T * f.V,
+                                      [&](int n) { return s_lse[n]; }, [&](int n) { return s_ent[n]; },
+                                      f.inv_temp, f.epsilon, f.delta, p.parent + (size_t)b * T,
+                                      f.cand_tokens + (size_t)b * T, __ldg(p.prefix_len + b), T, f.V,
+                                      p.S_max, lane, s_par, path)
+                : accept_warp(top_of, p.parent + (size_t)b * T, f.cand_tokens + (size_t)b * T,
+                              __ldg(p.prefix_len + b), T, f.V, p.S_max, lane, s_par, path);
         if (designated) {
             for (int i = lane; i < T; i += 32) f.path[(size_t)b * T + i] = path[i];
             if (lane == 0) {

@@ -34,10 +34,17 @@ struct FusedStep {
     int row_bytes;               // D * element size
     int V;
     int *scratch;                // [grid][kSideScratchInts] per-CTA scratch of the side warp
+    // typical acceptance (typical != 0): partial softmax statistics from the
+    // preceding grid, the logits for p(token), and the rule's parameters
+    int typical;
+    const float *part_stats;     // [B*T*splits][3]
+    const float *logits;         // [B,T,V]
+    float inv_temp, epsilon, delta;
 };
 
-// Per-CTA scratch of the fused step's side warp: parent copy, top-1 tokens, path.
-constexpr int kSideScratchInts = 3 * 128 + 8;
+// Per-CTA scratch of the fused step's side warp: parent copy, top-1 tokens,
+// path, and (typical acceptance) each node's log-sum-exp and entropy.
+constexpr int kSideScratchInts = 5 * 128 + 8;
 
 struct AttnParams {
     const int32_t *prefix_len;  // [B]
@@ -76,9 +83,12 @@ inline int argmax_split_count(int64_t rows, int V)
 }
 
 // Node argmax in two steps: per-(row, split) partial maxima, then a combine.
+// part_stats (3 floats per partial) non-null: also the softmax statistics at
+// `temperature` (typical acceptance).
 cudaError_t launch_argmax_partials(const float *logits, int64_t rows, int V, int splits,
-                                   float *part_val, int32_t *part_idx, int32_t *zero_status,
-                                   int n_zero, cudaStream_t stream);
+                                   float *part_val, int32_t *part_idx, float *part_stats,
+                                   float temperature, int32_t *zero_status, int n_zero,
+                                   cudaStream_t stream);
 cudaError_t launch_argmax_combine(const float *part_val, const int32_t *part_idx, int64_t rows,
                                   int splits, int32_t *argmax_out, cudaStream_t stream);
 
@@ -96,6 +106,17 @@ struct AcceptArgs {
 
 cudaError_t launch_accept_path(const int32_t *argmax, const AcceptArgs &a, int B,
                                cudaStream_t stream);
+
+// argmax, natural-log log-sum-exp and entropy per row from stats partials.
+cudaError_t launch_node_stats_combine(const float *part_val, const int32_t *part_idx,
+                                      const float *part_stats, int64_t rows, int splits,
+                                      int32_t *argmax_out, float *lse_out, float *ent_out,
+                                      cudaStream_t stream);
+
+cudaError_t launch_typical_accept(const float *logits, const float *lse, const float *ent,
+                                  const int32_t *argmax, const AcceptArgs &a, int B,
+                                  float temperature, float epsilon, float delta,
+                                  cudaStream_t stream);
 
 cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_tree,
                               const void *v_tree, const int32_t *path,

@@ -25,17 +25,22 @@ namespace ppd {
 
 // Partial top-1 of rows of fp32 logits: block (row, s) scans columns
 // [s*chunk, (s+1)*chunk) with 16-byte loads and writes its (value, index) to
-// part_*[row * splits + s].  Block 0 also zeroes `zero_status` (the fused step's
-// per-sequence status, raised later with atomicMax).  A grid launched after
-// this one with programmatic stream serialization may start right away.
-template <bool kVec>
+// part_*[row * splits + s].  With kStats it also accumulates the softmax
+// statistics (SoftStats, scale stat_k = log2(e) / temperature) of the same
+// columns into part_stats[3 * (row * splits + s) ...] (m, s, t).  Block 0 also
+// zeroes `zero_status` (the fused step's per-sequence status, raised later with
+// atomicMax).  A grid launched after this one with programmatic stream
+// serialization may start right away.
+template <bool kVec, bool kStats>
 __global__ void __launch_bounds__(256)
 argmax_partial_kernel(const float *__restrict__ logits, int V, int splits, int chunk,
-                      float *part_val, int32_t *part_idx, int32_t *zero_status, int n_zero)
+                      float *part_val, int32_t *part_idx, float *part_stats, float stat_k,
+                      int32_t *zero_status, int n_zero)
 {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __shared__ float s_v[8];
     __shared__ int s_i[8];
+    __shared__ float s_st[8][3];
     if (zero_status && blockIdx.x == 0)
         for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_status[i] = 0;
     const int64_t row = blockIdx.x / splits;
@@ -45,6 +50,14 @@ argmax_partial_kernel(const float *__restrict__ logits, int V, int splits, int c
     const float *x = logits + row * (int64_t)V;
     float bv = -INFINITY;
     int bi = INT_MAX;
+    SoftStats st;
+    auto take4 = [&](const float4 &f, int base) {
+        consider(f.x, base, bv, bi);
+        consider(f.y, base + 1, bv, bi);
+        consider(f.z, base + 2, bv, bi);
+        consider(f.w, base + 3, bv, bi);
+        if (kStats) stats_add4(st, f.x * stat_k, f.y * stat_k, f.z * stat_k, f.w * stat_k);
+    };
     if (kVec) {
         const float4 *x4 = reinterpret_cast<const float4 *>(x);
         const int n4_lo = lo >> 2, n4_hi = hi >> 2;
@@ -54,40 +67,60 @@ argmax_partial_kernel(const float *__restrict__ logits, int V, int splits, int c
 #pragma unroll
             for (int k = 0; k < 4; ++k) f[k] = __ldcs(x4 + i + k * 256);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int base = 4 * (i + k * 256);
-                consider(f[k].x, base, bv, bi);
-                consider(f[k].y, base + 1, bv, bi);
-                consider(f[k].z, base + 2, bv, bi);
-                consider(f[k].w, base + 3, bv, bi);
-            }
+            for (int k = 0; k < 4; ++k) take4(f[k], 4 * (i + k * 256));
         }
-        for (; i < n4_hi; i += 256) {
-            const float4 f = __ldcs(x4 + i);
-            consider(f.x, 4 * i, bv, bi);
-            consider(f.y, 4 * i + 1, bv, bi);
-            consider(f.z, 4 * i + 2, bv, bi);
-            consider(f.w, 4 * i + 3, bv, bi);
-        }
+        for (; i < n4_hi; i += 256) take4(__ldcs(x4 + i), 4 * i);
     } else {
-        for (int i = lo + threadIdx.x; i < hi; i += 256) consider(__ldcs(x + i), i, bv, bi);
+        // scalar loads; the statistics take one value at a time (three -inf pads)
+        for (int i = lo + threadIdx.x; i < hi; i += 256) {
+            const float v = __ldcs(x + i);
+            consider(v, i, bv, bi);
+            if (kStats) stats_add4(st, v * stat_k, -INFINITY, -INFINITY, -INFINITY);
+        }
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
         const float ov = __shfl_down_sync(0xffffffffu, bv, off);
         const int oi = __shfl_down_sync(0xffffffffu, bi, off);
         consider(ov, oi, bv, bi);
+        if (kStats) {
+            SoftStats o;
+            o.m = __shfl_down_sync(0xffffffffu, st.m, off);
+            o.s = __shfl_down_sync(0xffffffffu, st.s, off);
+            o.t = __shfl_down_sync(0xffffffffu, st.t, off);
+            stats_merge(st, o);
+        }
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
         s_v[warp] = bv;
         s_i[warp] = bi;
+        if (kStats) {
+            s_st[warp][0] = st.m;
+            s_st[warp][1] = st.s;
+            s_st[warp][2] = st.t;
+        }
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        for (int w = 1; w < 8; ++w) consider(s_v[w], s_i[w], bv, bi);
+        for (int w = 1; w < 8; ++w) {
+            consider(s_v[w], s_i[w], bv, bi);
+            if (kStats) {
+                SoftStats o;
+                o.m = s_st[w][0];
+                o.s = s_st[w][1];
+                o.t = s_st[w][2];
+                stats_merge(st, o);
+            }
+        }
         part_val[row * splits + s] = bv;
         part_idx[row * splits + s] = bi;
+        if (kStats) {
+            float *ps = part_stats + 3 * (row * splits + s);
+            ps[0] = st.m;
+            ps[1] = st.s;
+            ps[2] = st.t;
+        }
     }
 }
 
@@ -99,19 +132,30 @@ __global__ void argmax_combine_kernel(const float *part_val, const int32_t *part
 }
 
 cudaError_t launch_argmax_partials(const float *logits, int64_t rows, int V, int splits,
-                                   float *part_val, int32_t *part_idx, int32_t *zero_status,
-                                   int n_zero, cudaStream_t stream)
+                                   float *part_val, int32_t *part_idx, float *part_stats,
+                                   float temperature, int32_t *zero_status, int n_zero,
+                                   cudaStream_t stream)
 {
     const bool vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
     int chunk = (V + splits - 1) / splits;
     chunk = (chunk + 3) & ~3;
     const dim3 grid((unsigned)(rows * splits));
-    if (vec)
-        argmax_partial_kernel<true><<<grid, 256, 0, stream>>>(logits, V, splits, chunk, part_val,
-                                                              part_idx, zero_status, n_zero);
-    else
-        argmax_partial_kernel<false><<<grid, 256, 0, stream>>>(logits, V, splits, chunk, part_val,
-                                                               part_idx, zero_status, n_zero);
+    const float k = part_stats ? 1.4426950408889634f / temperature : 0.f;
+    if (part_stats) {
+        if (vec)
+            argmax_partial_kernel<true, true><<<grid, 256, 0, stream>>>(
+                logits, V, splits, chunk, part_val, part_idx, part_stats, k, zero_status, n_zero);
+        else
+            argmax_partial_kernel<false, true><<<grid, 256, 0, stream>>>(
+                logits, V, splits, chunk, part_val, part_idx, part_stats, k, zero_status, n_zero);
+    } else {
+        if (vec)
+            argmax_partial_kernel<true, false><<<grid, 256, 0, stream>>>(
+                logits, V, splits, chunk, part_val, part_idx, nullptr, 0.f, zero_status, n_zero);
+        else
+            argmax_partial_kernel<false, false><<<grid, 256, 0, stream>>>(
+                logits, V, splits, chunk, part_val, part_idx, nullptr, 0.f, zero_status, n_zero);
+    }
     return cudaGetLastError();
 }
 
@@ -148,6 +192,64 @@ cudaError_t launch_accept_path(const int32_t *argmax, const AcceptArgs &a, int B
                                cudaStream_t stream)
 {
     accept_path_kernel<<<(B + 3) / 4, 128, 0, stream>>>(argmax, a, B);
+    return cudaGetLastError();
+}
+
+// Node statistics: argmax, natural-log log-sum-exp and entropy of each row
+// from its partial results.
+__global__ void node_stats_combine_kernel(const float *part_val, const int32_t *part_idx,
+                                          const float *part_stats, int64_t rows, int splits,
+                                          int32_t *argmax_out, float *lse_out, float *ent_out)
+{
+    const int64_t row = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (row >= rows) return;
+    argmax_out[row] = combine_partials(part_val, part_idx, row, splits);
+    const SoftStats st = combine_stats(part_stats, row, splits);
+    stats_finish(st, lse_out[row], ent_out[row]);
+}
+
+cudaError_t launch_node_stats_combine(const float *part_val, const int32_t *part_idx,
+                                      const float *part_stats, int64_t rows, int splits,
+                                      int32_t *argmax_out, float *lse_out, float *ent_out,
+                                      cudaStream_t stream)
+{
+    node_stats_combine_kernel<<<(unsigned)((rows + 127) / 128), 128, 0, stream>>>(
+        part_val, part_idx, part_stats, rows, splits, argmax_out, lse_out, ent_out);
+    return cudaGetLastError();
+}
+
+// Typical acceptance, one warp per sequence, from the node statistics.
+__global__ void __launch_bounds__(128)
+typical_accept_kernel(const float *logits, const float *lse, const float *ent,
+                      const int32_t *argmax, AcceptArgs a, int B, float inv_temp, float epsilon,
+                      float delta)
+{
+    __shared__ int s_par[4][128];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.x * 4 + warp;
+    if (b >= B) return;
+    const size_t o = (size_t)b * a.T;
+    const int32_t *top = argmax + o;
+    const AcceptResult r = accept_warp_typical(
+        [&](int n) { return __ldg(top + n); }, logits + o * a.V,
+        [&](int n) { return __ldg(lse + o + n); }, [&](int n) { return __ldg(ent + o + n); },
+        inv_temp, epsilon, delta, a.parent + o, a.cand_tokens + o, __ldg(a.prefix_len + b), a.T,
+        a.V, a.S_max, lane, s_par[warp], a.path + o);
+    if (lane == 0) {
+        a.accept_len[b] = r.n_acc;
+        a.next_token[b] = r.next_token;
+        a.new_prefix_len[b] = r.new_prefix_len;
+        a.dev_status[b] = r.status;
+    }
+}
+
+cudaError_t launch_typical_accept(const float *logits, const float *lse, const float *ent,
+                                  const int32_t *argmax, const AcceptArgs &a, int B,
+                                  float temperature, float epsilon, float delta,
+                                  cudaStream_t stream)
+{
+    typical_accept_kernel<<<(B + 3) / 4, 128, 0, stream>>>(logits, lse, ent, argmax, a, B,
+                                                           1.0f / temperature, epsilon, delta);
     return cudaGetLastError();
 }
 
@@ -408,7 +510,8 @@ extern "C" ppd_status ppd_node_argmax_noalloc(const float *logits, int B, int T,
     int32_t *pi = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(scratch) +
                                               ppd::kNoAllocMaxPartials * 4);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (ppd::launch_argmax_partials(logits, rows, V, splits, pv, pi, nullptr, 0, s) != cudaSuccess)
+    if (ppd::launch_argmax_partials(logits, rows, V, splits, pv, pi, nullptr, 1.f, nullptr, 0, s) !=
+        cudaSuccess)
         return PPD_ERR_CUDA;
     return ppd::launch_argmax_combine(pv, pi, rows, splits, argmax_out, s) == cudaSuccess ? PPD_OK
                                                                                           : PPD_ERR_CUDA;

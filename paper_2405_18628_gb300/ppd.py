@@ -50,6 +50,10 @@ def load() -> ctypes.CDLL:
             "ppd_verify_step": ([vp] * 9 + [i32] * 8 + [f32] + [vp] * 8 + [vp, sz, vp], i32),
             "ppd_selftest_umma": ([vp, vp, vp, i32, i32, vp], i32),
             "ppd_node_argmax_noalloc": ([vp, i32, i32, i32, vp, vp], i32),
+            "ppd_node_stats": ([vp, i32, i32, i32, f32, vp, vp, vp, vp, sz, vp], i32),
+            "ppd_typical_accept": ([vp] * 7 + [i32] * 4 + [f32] * 3 + [vp] * 5 + [vp], i32),
+            "ppd_verify_step_typical": ([vp] * 9 + [i32] * 8 + [f32] * 4 + [vp] * 8 +
+                                        [vp, sz, vp], i32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -164,6 +168,45 @@ def ppd_verify_step(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, can
         _ptr(next_token), _ptr(new_prefix_len), _ptr(dev_status), _ptr(workspace),
         workspace.numel(), _stream(stream))
     _check(st, "ppd_verify_step")
+
+
+def ppd_node_stats(logits, temperature: float, argmax_out, lse_out, entropy_out, workspace,
+                   stream=None):
+    """logits fp32 [B,T,V] -> argmax int32 [B,T], log-sum-exp and entropy fp32
+    [B,T] of softmax(logits / temperature)."""
+    B, T, V = logits.shape
+    st = load().ppd_node_stats(_ptr(logits), B, T, V, float(temperature), _ptr(argmax_out),
+                               _ptr(lse_out), _ptr(entropy_out), _ptr(workspace),
+                               workspace.numel(), _stream(stream))
+    _check(st, "ppd_node_stats")
+
+
+def ppd_typical_accept(logits, lse, entropy, argmax, cand_tokens, parent, prefix_len, S_max,
+                       temperature: float, epsilon: float, delta: float, accept_len, path,
+                       next_token, new_prefix_len, dev_status, stream=None):
+    B, T, V = logits.shape
+    st = load().ppd_typical_accept(
+        _ptr(logits), _ptr(lse), _ptr(entropy), _ptr(argmax), _ptr(cand_tokens), _ptr(parent),
+        _ptr(prefix_len), B, T, V, int(S_max), float(temperature), float(epsilon), float(delta),
+        _ptr(accept_len), _ptr(path), _ptr(next_token), _ptr(new_prefix_len), _ptr(dev_status),
+        _stream(stream))
+    _check(st, "ppd_typical_accept")
+
+
+def ppd_verify_step_typical(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, cand_tokens,
+                            logits, temperature: float, epsilon: float, delta: float, out,
+                            argmax_out, accept_len, path, next_token, new_prefix_len, dev_status,
+                            workspace, lse=None, scale: float = 0.0, stream=None):
+    L, B, H, T, D = q.shape
+    S_max = k_cache.shape[3]
+    V = logits.shape[2]
+    st = load().ppd_verify_step_typical(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(k_tree), _ptr(v_tree), _ptr(prefix_len),
+        _ptr(parent), _ptr(cand_tokens), _ptr(logits), L, B, H, T, D, V, S_max, _dtype(q),
+        float(scale), float(temperature), float(epsilon), float(delta), _ptr(out), _ptr(lse),
+        _ptr(argmax_out), _ptr(accept_len), _ptr(path), _ptr(next_token), _ptr(new_prefix_len),
+        _ptr(dev_status), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(st, "ppd_verify_step_typical")
 
 
 def ppd_selftest_umma(a, b, d, mode: int, N: int, stream=None):

@@ -94,3 +94,26 @@ def test_binding_requires_library(monkeypatch, tmp_path):
     monkeypatch.setattr(ppd, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="missing"):
         ppd.load()
+
+
+def test_typical_acceptance_host_checks(lib):
+    """Typical acceptance needs a positive, finite temperature and finite
+    epsilon / delta; bad values are refused before any launch."""
+    from paper_2405_18628_gb300 import ppd
+    vp = ctypes.c_void_p
+    fake = vp(0x10000)
+    s = vp(0)
+    ws = 1 << 20
+    for temp in (0.0, -1.0, float("nan"), float("inf"), 1e-45):
+        assert lib.ppd_node_stats(fake, 1, 4, 100, temp, fake, fake, fake, fake, ws, s) == \
+            ppd.PPD_ERR_INVALID_ARG
+        assert lib.ppd_typical_accept(*[fake] * 7, 1, 4, 100, 10, temp, 0.1, 0.1,
+                                      *[fake] * 5, s) == ppd.PPD_ERR_INVALID_ARG
+    for eps, delta in ((float("nan"), 0.1), (0.1, float("inf"))):
+        assert lib.ppd_typical_accept(*[fake] * 7, 1, 4, 100, 10, 1.0, eps, delta,
+                                      *[fake] * 5, s) == ppd.PPD_ERR_INVALID_ARG
+    args = [fake] * 9 + [1, 1, 1, 4, 64, 100, 16, ppd.PPD_BF16, 0.0, 0.0, 0.1, 0.1] + \
+        [fake] * 8 + [fake, 1 << 30, s]
+    assert lib.ppd_verify_step_typical(*args) == ppd.PPD_ERR_INVALID_ARG
+    assert lib.ppd_node_stats(None, 1, 4, 100, 1.0, fake, fake, fake, fake, ws, s) == \
+        ppd.PPD_ERR_INVALID_ARG
