@@ -245,14 +245,13 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                 mbar_wait(bars + Lay::B_VFULL + vs, (gp / Lay::VS) & 1, abort_flag);
                 tc_fence_after();
                 if (!*abort_flag) {
+                    // descriptors built once; each 16-key step moves 2048 bytes on
+                    const uint64_t a0 = make_smem_desc(sv + vs * Lay::TILE_BYTES, v_lbo, 1024);
+                    const uint64_t b0 = make_smem_desc(s0 + p_offset<Lay>(gp), Lay::GROUP_BYTES, 1024);
 #pragma unroll
-                    for (int kk = 0; kk < Lay::KT / 16; ++kk) {
-                        const uint64_t a = make_smem_desc(sv + vs * Lay::TILE_BYTES + kk * 2048,
-                                                          v_lbo, 1024);
-                        const uint64_t b = make_smem_desc(s0 + p_offset<Lay>(gp) + kk * 2048,
-                                                          Lay::GROUP_BYTES, 1024);
-                        umma_bf16(t_o, a, b, idesc_pv, (first && kk == 0) ? 0u : 1u);
-                    }
+                    for (int kk = 0; kk < Lay::KT / 16; ++kk)
+                        umma_bf16(t_o, desc_advance(a0, kk * 2048), desc_advance(b0, kk * 2048), idesc_pv,
+                                  (first && kk == 0) ? 0u : 1u);
                 }
                 umma_commit(bars + Lay::B_PFREE + ps);
                 umma_commit(bars + Lay::B_VEMPTY + vs);
@@ -277,13 +276,15 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     if (g >= 2) mbar_wait(bars + Lay::B_SFREE + sb, ((g >> 1) - 1) & 1, abort_flag);
                     tc_fence_after();
                     if (!*abort_flag) {
+                        const uint64_t a0 = make_smem_desc(sk + ks * Lay::TILE_BYTES, 16, 1024);
+                        const uint64_t b0 = make_smem_desc(sq + qs * Lay::Q_BYTES, 16, 1024);
+                        const uint32_t d_s = tmem_base + Lay::T_S + sb * TPMAX;
 #pragma unroll
                         for (int kk = 0; kk < D / 16; ++kk) {
                             const uint32_t koff = (kk >> 2) * Lay::GROUP_BYTES + (kk & 3) * 32;
                             const uint32_t qoff = (kk >> 2) * Lay::Q_GROUP_BYTES + (kk & 3) * 32;
-                            const uint64_t a = make_smem_desc(sk + ks * Lay::TILE_BYTES + koff, 16, 1024);
-                            const uint64_t b = make_smem_desc(sq + qs * Lay::Q_BYTES + qoff, 16, 1024);
-                            umma_bf16(tmem_base + Lay::T_S + sb * TPMAX, a, b, idesc_qk, kk > 0 ? 1u : 0u);
+                            umma_bf16(d_s, desc_advance(a0, koff), desc_advance(b0, qoff), idesc_qk,
+                                      kk > 0 ? 1u : 0u);
                         }
                     }
                     umma_commit(bars + Lay::B_SFULL + sb);

@@ -19,9 +19,12 @@
 // unit's first tile, or a score more than 2^16 above the running maximum --
 // decided per tile by a vote over the softmax warps) and partial sums at the
 // end of a unit.  The tree mask is a 64-bit ancestor bitset per thread, built
-// from the parent array in registers.  Warp roles, the unit walk, the
-// double-buffered O with deferred readback and the fused step's side warp are
-// those of the kernel for trees of up to 64 tokens (ppd_attention.cu).
+// from the parent array in registers.  Three score buffers in TMEM let two PV
+// products and the next S product queue in the tensor pipe; the single O
+// accumulator of a finished unit is read back after the next unit's first
+// tile, and that unit's first PV product waits for the readback.  Warp roles,
+// the unit walk and the fused step's side warp are those of the kernel for
+// trees of up to 64 tokens (ppd_attention.cu).
 #include "ppd_attention_common.cuh"
 
 #include <cmath>
@@ -51,18 +54,23 @@ struct RowsLayout {
     static constexpr int B_KEMPTY = B_KFULL + KS;
     static constexpr int B_VFULL = B_KEMPTY + KS;
     static constexpr int B_VEMPTY = B_VFULL + VS;
-    static constexpr int B_SFULL = B_VEMPTY + VS;   // [2] scores of tile g in TMEM
-    static constexpr int B_PFULL = B_SFULL + 2;     // [2] probabilities of tile g in TMEM (8 warps)
-    static constexpr int B_PDONE = B_PFULL + 2;     // [2] PV product of tile g complete
-    static constexpr int B_DRAIN = B_PDONE + 2;
+    // Score tiles in TMEM: P is written over S, so S(g + NSB) waits for PV(g);
+    // three buffers keep two PV products and one S product in the tensor pipe.
+    static constexpr int NSB = 3;
+    static constexpr int B_SFULL = B_VEMPTY + VS;   // [NSB] scores of tile g in TMEM
+    static constexpr int B_PFULL = B_SFULL + NSB;   // [NSB] probabilities of tile g in TMEM (8 warps)
+    static constexpr int B_PDONE = B_PFULL + NSB;   // [NSB] PV product of tile g complete
+    static constexpr int B_OFREE = B_PDONE + NSB;   // a unit's output read back from TMEM (8 warps)
+    static constexpr int B_DRAIN = B_OFREE + 1;
     static constexpr int NBAR = B_DRAIN + 1;
     static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
     static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
     static constexpr uint32_t OFF_XM = (OFF_ABORT + 4 + 15) & ~15u;   // [2][M] partial row maxima
     static constexpr uint32_t OFF_XL = OFF_XM + 2 * M * 4;            // [2][M] partial row sums
     static constexpr uint32_t SMEM_BYTES = OFF_XL + 2 * M * 4;
-    // TMEM columns: S0 | S1 (128 each; P is written over S) | O0 | O1 (D each)
-    static constexpr uint32_t T_S = 0, T_O = 256, O_STRIDE = 128, TMEM_COLS = 512;
+    // TMEM columns: S0 | S1 | S2 (128 each; P is written over S) | O (D)
+    static constexpr uint32_t T_S = 0, T_O = NSB * 128, TMEM_COLS = 512;
+    static_assert(NSB * 128 + D <= 512, "TMEM budget");
 
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
     static_assert((OFF_K | OFF_V | Q_BYTES) % 1024 == 0, "1024-byte aligned operand tiles");
@@ -96,7 +104,8 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < Lay::NBAR; ++i)
-            mbar_init(bars + i, (i >= Lay::B_PFULL && i < Lay::B_PFULL + 2) ? 8u : 1u);
+            mbar_init(bars + i, ((i >= Lay::B_PFULL && i < Lay::B_PFULL + Lay::NSB) || i == Lay::B_OFREE)
+                                    ? 8u : 1u);
         *abort_flag = 0;
         mbar_fence_init();
     }
@@ -183,18 +192,22 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             // O += P_hi V + P_lo V for tile gp.  Per 32 keys the probability columns
             // hold 8 columns of hi pairs for keys 0..15, 8 for keys 16..31, then the
             // lo pairs in the same order.
-            auto issue_pv = [&](int gp, bool first, uint32_t t_o) {
-                const int pb = gp & 1;
-                mbar_wait(bars + Lay::B_PFULL + pb, (gp >> 1) & 1, abort_flag);
+            // A unit's first PV product overwrites O: unit k >= 1 waits until the
+            // softmax warps have read unit k-1's output back.
+            const uint32_t t_o = tmem_base + Lay::T_O;
+            auto issue_pv = [&](int gp, bool first, int kp) {
+                const int pb = gp % Lay::NSB;
+                mbar_wait(bars + Lay::B_PFULL + pb, (gp / Lay::NSB) & 1, abort_flag);
+                if (first && kp >= 1) mbar_wait(bars + Lay::B_OFREE, (kp - 1) & 1, abort_flag);
                 const int vs = gp % Lay::VS;
                 mbar_wait(bars + Lay::B_VFULL + vs, (gp / Lay::VS) & 1, abort_flag);
                 tc_fence_after();
                 if (!*abort_flag) {
                     const uint32_t a0 = tmem_base + Lay::T_S + (uint32_t)pb * 128u;
+                    const uint64_t b0 = make_smem_desc(sv + vs * Lay::TILE_BYTES, Lay::GROUP_BYTES, 1024);
 #pragma unroll
                     for (int kk = 0; kk < Lay::KT / 16; ++kk) {
-                        const uint64_t b = make_smem_desc(sv + vs * Lay::TILE_BYTES + kk * 2048,
-                                                          Lay::GROUP_BYTES, 1024);
+                        const uint64_t b = desc_advance(b0, kk * 2048);
                         const uint32_t a_hi = a0 + 32u * (kk >> 1) + 8u * (kk & 1);
                         umma_bf16_ta(t_o, a_hi, b, idesc_pv, (first && kk == 0) ? 0u : 1u);
                         umma_bf16_ta(t_o, a_hi + 16u, b, idesc_pv, 1u);
@@ -204,43 +217,51 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 umma_commit(bars + Lay::B_VEMPTY + vs);
             };
 
-            // Tiles are issued as S(g), PV(g-1) across unit boundaries, so the next
-            // unit's first scores are under way before this unit's last PV product.
+            // Tiles are issued as S(g), PV(g-2), across unit boundaries: the scores
+            // of the tile after next are queued in the tensor pipe before the PV
+            // product that has to wait for the softmax of the current tile, so the
+            // softmax warps find S(g+1) ready when they finish tile g.  (S(g) reuses
+            // the buffer of tile g-3, whose PV product was issued one tile earlier.)
             int g = 0, k = 0;
-            int prev_g = -1;
-            bool prev_first = false;
-            uint32_t prev_to = 0;
+            int lag_g[2] = {-1, -1}, lag_k[2] = {0, 0};   // tiles g-2 and g-1 awaiting PV
+            bool lag_first[2] = {false, false};
             for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
                 const UnitInfo ui = unit_info(p, u);
                 const int qs = k % Lay::QS;
-                const uint32_t t_o = tmem_base + Lay::T_O + (uint32_t)(k & 1) * Lay::O_STRIDE;
                 mbar_wait(bars + Lay::B_QFULL + qs, (k / Lay::QS) & 1, abort_flag);
                 for (int j = 0; j < ui.n_tiles; ++j, ++g) {
                     const int ks = g % Lay::KS;
-                    const int sb = g & 1;
+                    const int sb = g % Lay::NSB;
                     mbar_wait(bars + Lay::B_KFULL + ks, (g / Lay::KS) & 1, abort_flag);
-                    // P(g-2) lives in this S buffer until its PV product is done
-                    if (g >= 2) mbar_wait(bars + Lay::B_PDONE + sb, ((g - 2) >> 1) & 1, abort_flag);
+                    // P(g - NSB) lives in this S buffer until its PV product is done
+                    if (g >= Lay::NSB)
+                        mbar_wait(bars + Lay::B_PDONE + sb, ((g - Lay::NSB) / Lay::NSB) & 1, abort_flag);
                     tc_fence_after();
                     if (!*abort_flag) {
+                        const uint64_t a0 = make_smem_desc(sq + qs * Lay::Q_BYTES, 16, 1024);
+                        const uint64_t b0 = make_smem_desc(sk + ks * Lay::TILE_BYTES, 16, 1024);
+                        const uint32_t d_s = tmem_base + Lay::T_S + sb * 128u;
 #pragma unroll
                         for (int kk = 0; kk < D / 16; ++kk) {
                             const uint32_t off = (kk >> 2) * Lay::GROUP_BYTES + (kk & 3) * 32;
-                            const uint64_t a = make_smem_desc(sq + qs * Lay::Q_BYTES + off, 16, 1024);
-                            const uint64_t b = make_smem_desc(sk + ks * Lay::TILE_BYTES + off, 16, 1024);
-                            umma_bf16(tmem_base + Lay::T_S + sb * 128u, a, b, idesc_qk, kk > 0 ? 1u : 0u);
+                            umma_bf16(d_s, desc_advance(a0, off), desc_advance(b0, off), idesc_qk,
+                                      kk > 0 ? 1u : 0u);
                         }
                     }
                     umma_commit(bars + Lay::B_SFULL + sb);
                     umma_commit(bars + Lay::B_KEMPTY + ks);
                     if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
-                    if (prev_g >= 0) issue_pv(prev_g, prev_first, prev_to);
-                    prev_g = g;
-                    prev_first = (j == 0);
-                    prev_to = t_o;
+                    if (lag_g[0] >= 0) issue_pv(lag_g[0], lag_first[0], lag_k[0]);
+                    lag_g[0] = lag_g[1];
+                    lag_first[0] = lag_first[1];
+                    lag_k[0] = lag_k[1];
+                    lag_g[1] = g;
+                    lag_first[1] = (j == 0);
+                    lag_k[1] = k;
                 }
             }
-            if (prev_g >= 0) issue_pv(prev_g, prev_first, prev_to);
+            for (int x = 0; x < 2; ++x)
+                if (lag_g[x] >= 0) issue_pv(lag_g[x], lag_first[x], lag_k[x]);
             umma_commit(bars + Lay::B_DRAIN);
             mbar_wait_drain(bars + Lay::B_DRAIN, 0);
         }
@@ -259,7 +280,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
         int cur_b = -1;
         int g = 0;
         bool pend = false;      // a finished unit whose output still sits in TMEM
-        int pend_u = 0, pend_ob = 0, pend_g = 0;
+        int pend_u = 0, pend_g = 0;
         float pend_linv = 0.f;
 
         // Probabilities of this thread's 64 keys from its raw scores s against the
@@ -316,12 +337,12 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             return fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
         };
 
-        // Output of a finished unit: this thread's half of the row of O times 1 / l.
-        auto read_back = [&](int u_out, int ob, int g_last, float linv) {
-            mbar_wait(bars + Lay::B_PDONE + (g_last & 1), (g_last >> 1) & 1, abort_flag);
+        // Output of a finished unit: this thread's half of the row of O times 1 / l;
+        // then O is free for the next unit's first PV product.
+        auto read_back = [&](int u_out, int g_last, float linv) {
+            mbar_wait(bars + Lay::B_PDONE + g_last % Lay::NSB, (g_last / Lay::NSB) & 1, abort_flag);
             tc_fence_after();
-            const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * Lay::O_STRIDE +
-                                 (uint32_t)h * (D / 2);
+            const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)h * (D / 2);
             float *orow = p.out + ((size_t)u_out * T + q) * D + h * (D / 2);
 #pragma unroll
             for (int ch = 0; ch < D / 32; ++ch) {
@@ -343,12 +364,13 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 }
             }
             tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bars + Lay::B_OFREE);
         };
 
         int k = 0;
         for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
             const UnitInfo ui = unit_info(p, u);
-            const int ob = k & 1;
             if (ui.b != cur_b) {
                 // ancestors of node q among tree nodes [64h, 64h + 64)
                 abits = 0;
@@ -379,8 +401,8 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 const bool tree = (j == ui.n_pref);
                 const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
                 const int kind = tree ? kMaskTree : (n_valid < Lay::KT ? kMaskRows : kMaskNone);
-                const int sb = g & 1;
-                mbar_wait(bars + Lay::B_SFULL + sb, (g >> 1) & 1, abort_flag);
+                const int sb = g % Lay::NSB;
+                mbar_wait(bars + Lay::B_SFULL + sb, (g / Lay::NSB) & 1, abort_flag);
                 tc_fence_after();
                 const uint32_t t_s = tmem_base + lane_off + Lay::T_S + (uint32_t)sb * 128u +
                                      (uint32_t)h * 64u;
@@ -412,11 +434,10 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                         if (__any_sync(0xffffffffu, alpha != 1.f)) {
                             // rescale this thread's half of the row of O once the PV
                             // product of the previous tile has landed
-                            mbar_wait(bars + Lay::B_PDONE + ((g - 1) & 1), ((g - 1) >> 1) & 1,
-                                      abort_flag);
+                            mbar_wait(bars + Lay::B_PDONE + (g - 1) % Lay::NSB,
+                                      ((g - 1) / Lay::NSB) & 1, abort_flag);
                             tc_fence_after();
-                            const uint32_t t_o = tmem_base + lane_off + Lay::T_O +
-                                                 (uint32_t)ob * Lay::O_STRIDE + (uint32_t)h * (D / 2);
+                            const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)h * (D / 2);
 #pragma unroll
                             for (int ch = 0; ch < D / 32; ++ch) {
                                 uint32_t r[16];
@@ -460,7 +481,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
                 // the previous unit's output, once this unit's first tile is on its way
                 if (j == 0 && pend) {
-                    read_back(pend_u, pend_ob, pend_g, pend_linv);
+                    read_back(pend_u, pend_g, pend_linv);
                     pend = false;
                 }
 
@@ -473,7 +494,6 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                         p.lse[(size_t)u * T + q] = (m + lg2(L)) * 0.69314718055994530942f;
                     pend = true;
                     pend_u = u;
-                    pend_ob = ob;
                     pend_g = g;
                     pend_linv = rcp(L);
                     m = -INFINITY;
@@ -481,7 +501,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 }
             }
         }
-        if (pend) read_back(pend_u, pend_ob, pend_g, pend_linv);
+        if (pend) read_back(pend_u, pend_g, pend_linv);
     }
 
     tc_fence_before();

@@ -275,6 +275,14 @@ PPD_DEV uint64_t make_smem_desc(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo
     return d;
 }
 
+// The descriptor of the same operand `bytes` further on (bytes a multiple of 16):
+// only the 14-bit start-address field (16-byte units) changes, and shared
+// memory addresses stay below 256 KB, so the field never carries.
+PPD_DEV uint64_t desc_advance(uint64_t desc, uint32_t bytes)
+{
+    return desc + (uint64_t)(bytes >> 4);
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16: bf16 A and B, fp32 D,
 // shape M x N, operand majorness (0 = K-major, 1 = M/N-major).
 __host__ __device__ constexpr uint32_t make_idesc_bf16(int M, int N, int a_mn_major,
