@@ -208,6 +208,12 @@ def parse():
     ap.add_argument("--accept", default="exact", choices=["exact", "typical"],
                     help="verification rule: exact matching, or typical acceptance at "
                          "temperature 0.7, epsilon 0.09, delta 0.3")
+    ap.add_argument("--tree-sizes", default="",
+                    help="comma-separated tree sizes: also report the step latency of each "
+                         "(the hardware half of the paper's hardware-aware tree size)")
+    ap.add_argument("--tau", default="",
+                    help="JSON file {tree size: acceptance length}: with --tree-sizes, also "
+                         "report Speedup(n) = tau(n) / latency(n) and the best size")
     ap.add_argument("--layers", type=int, default=0,
                     help="run the workload with this many layers (profiling captures)")
     ap.add_argument("--l2", default="auto", choices=["auto", "flush", "none"],
@@ -436,6 +442,23 @@ def main():
     if world == 1 and rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, t, s, args.cpu_budget)
 
+    # ---------------------------------------------------------------- tree-size profile
+    profile = None
+    if args.tree_sizes:
+        from paper_2405_18628_gb300 import tree_profile
+        del t, bufs, logits
+        torch.cuda.empty_cache()
+        sizes = [int(x) for x in args.tree_sizes.split(",") if x.strip()]
+        lat = tree_profile.latency_profile(w, sizes, steps=min(K, 50), warmup=3, device=dev,
+                                           flush_bytes=L2_FLUSH_BYTES if do_flush else 0)
+        profile = {"latency": [{"T": n, "ms_per_step": ms} for n, ms in lat]}
+        if args.tau:
+            with open(args.tau) as f:
+                tau = {int(k): float(v) for k, v in json.load(f).items()}
+            rows, best = tree_profile.speedup_table(tau, lat)
+            profile["speedup"] = rows
+            profile["best_tree_size"] = best
+
     sb = step_bytes(w, n_acc)
     if rank == 0:
         line = {
@@ -460,7 +483,8 @@ def main():
             "step_bytes": sb,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
-                         "kernel": "tree_attention_kernel", "launch_us": att_ms * 1e3,
+                         "kernel": ("tree_attention_kernel" if w.T <= 64 else
+                                    "tree_attention_rows_kernel"), "launch_us": att_ms * 1e3,
                          "bytes_per_launch": att_bytes, "peak_kind": peak_kind,
                          "frac_of_8000": achieved / NOMINAL_HBM_GBS},
             "e2e": e2e,
@@ -469,6 +493,8 @@ def main():
             "cpu_baseline": cpu,
             "wall_s_timed": wall,
         }
+        if profile is not None:
+            line["tree_size_profile"] = profile
         print(json.dumps(line), flush=True)
     if pg:
         pg.barrier()

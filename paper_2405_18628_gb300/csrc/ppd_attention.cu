@@ -698,7 +698,7 @@ static cudaError_t launch_tree_attention_t(const AttnMaps &m, const AttnParams &
                                            bool programmatic, cudaStream_t stream)
 {
     static std::atomic<uint64_t> configured{0};
-    return launch_attention_grid(tree_attention_kernel<D>, AttnLayout<D>::SMEM_BYTES, configured, m,
+    return launch_attention_grid(tree_attention_kernel<D>, AttnLayout<D>::SMEM_BYTES, 352, configured, m,
                                  p, num_sms, programmatic, stream);
 }
 

@@ -133,10 +133,11 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
 }
 
 // Launch one of the persistent attention kernels: one CTA per SM (at most one
-// per unit), `smem` bytes of dynamic shared memory, with programmatic stream
+// per unit) of `threads` threads, `smem` bytes of dynamic shared memory, with programmatic stream
 // serialization when asked.  The shared-memory opt-in is set once per device.
 template <class Kern>
-cudaError_t launch_attention_grid(Kern kern, uint32_t smem, std::atomic<uint64_t> &configured,
+cudaError_t launch_attention_grid(Kern kern, uint32_t smem, int threads,
+                                  std::atomic<uint64_t> &configured,
                                   const AttnMaps &m, const AttnParams &p, int num_sms,
                                   bool programmatic, cudaStream_t stream)
 {
@@ -151,7 +152,7 @@ cudaError_t launch_attention_grid(Kern kern, uint32_t smem, std::atomic<uint64_t
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(p.n_units < num_sms ? p.n_units : num_sms));
-    cfg.blockDim = dim3(352);
+    cfg.blockDim = dim3((unsigned)threads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];

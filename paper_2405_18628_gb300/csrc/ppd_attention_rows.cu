@@ -22,9 +22,10 @@
 // from the parent array in registers.  Three score buffers in TMEM let two PV
 // products and the next S product queue in the tensor pipe; the single O
 // accumulator of a finished unit is read back after the next unit's first
-// tile, and that unit's first PV product waits for the readback.  Warp roles,
-// the unit walk and the fused step's side warp are those of the kernel for
-// trees of up to 64 tokens (ppd_attention.cu).
+// tile, and that unit's first PV product waits for the readback.  The unit
+// walk and the fused step's side warp are those of the kernel for trees of up
+// to 64 tokens (ppd_attention.cu); the warp roles (384 threads) differ in one
+// point: warp 8 loads Q and K, warp 11 loads V.
 #include "ppd_attention_common.cuh"
 
 #include <cmath>
@@ -77,7 +78,7 @@ struct RowsLayout {
 };
 
 template <int D>
-__global__ void __launch_bounds__(352, 1)
+__global__ void __launch_bounds__(384, 1)
 tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                            const __grid_constant__ CUtensorMap map_kc,
                            const __grid_constant__ CUtensorMap map_vc,
@@ -121,63 +122,78 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
     if (warp == 10) {
         // ------------------------------------------------------------ fused-step side work
         if (p.fused) fused_side_warp(p, lane);
-    } else if (warp == 8) {
-        // ------------------------------------------------------------ TMA producer
+    } else if (warp == 8 || warp == 11) {
+        // ------------------------------------------------------------ TMA producers
+        // warp 8 loads Q and the K tiles, warp 11 the V tiles: a V slot is released
+        // only by its PV product, so the K stream never queues behind it.
         if (lane == 0) {
-            tma_prefetch_map(&map_q);
-            tma_prefetch_map(&map_kc);
-            tma_prefetch_map(&map_vc);
-            tma_prefetch_map(&map_kt);
-            tma_prefetch_map(&map_vt);
+            const bool kq = (warp == 8);
+            if (kq) {
+                tma_prefetch_map(&map_q);
+                tma_prefetch_map(&map_kc);
+                tma_prefetch_map(&map_kt);
+            } else {
+                tma_prefetch_map(&map_vc);
+                tma_prefetch_map(&map_vt);
+            }
             const uint64_t pol = l2_policy_evict_first();
             int g = 0, k = 0;
             for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
                 const UnitInfo ui = unit_info(p, u);
                 const int qs = k % Lay::QS;
-                if (k >= Lay::QS)
-                    mbar_wait(bars + Lay::B_QEMPTY + qs, ((k / Lay::QS) - 1) & 1, abort_flag);
-                if (!*abort_flag) {
-                    // rows T..127 of the box lie beyond the tensor and arrive as zeros
-                    mbar_arrive_expect_tx(bars + Lay::B_QFULL + qs, Lay::Q_BYTES);
+                if (kq) {
+                    if (k >= Lay::QS)
+                        mbar_wait(bars + Lay::B_QEMPTY + qs, ((k / Lay::QS) - 1) & 1, abort_flag);
+                    if (!*abort_flag) {
+                        // rows T..127 of the box lie beyond the tensor and arrive as zeros
+                        mbar_arrive_expect_tx(bars + Lay::B_QFULL + qs, Lay::Q_BYTES);
 #pragma unroll
-                    for (int c = 0; c < Lay::DCH; ++c)
-                        tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::GROUP_BYTES,
-                                    &map_q, bars + Lay::B_QFULL + qs, c * 64, 0, u, pol);
+                        for (int c = 0; c < Lay::DCH; ++c)
+                            tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::GROUP_BYTES,
+                                        &map_q, bars + Lay::B_QFULL + qs, c * 64, 0, u, pol);
+                    }
                 }
                 for (int j = 0; j < ui.n_tiles; ++j, ++g) {
                     const bool tree = (j == ui.n_pref);
                     const int row = tree ? 0 : j * Lay::KT;
-                    const int ks = g % Lay::KS;
-                    if (g >= Lay::KS)
-                        mbar_wait(bars + Lay::B_KEMPTY + ks, ((g / Lay::KS) - 1) & 1, abort_flag);
-                    if (!*abort_flag) {
-                        mbar_arrive_expect_tx(bars + Lay::B_KFULL + ks, Lay::TILE_BYTES);
+                    if (kq) {
+                        const int ks = g % Lay::KS;
+                        if (g >= Lay::KS)
+                            mbar_wait(bars + Lay::B_KEMPTY + ks, ((g / Lay::KS) - 1) & 1, abort_flag);
+                        if (!*abort_flag) {
+                            mbar_arrive_expect_tx(bars + Lay::B_KFULL + ks, Lay::TILE_BYTES);
 #pragma unroll
-                        for (int c = 0; c < Lay::DCH; ++c)
-                            tma_load_3d(smem + Lay::OFF_K + ks * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
-                                        tree ? &map_kt : &map_kc, bars + Lay::B_KFULL + ks, c * 64,
-                                        row, u, pol);
-                    }
-                    const int vs = g % Lay::VS;
-                    if (g >= Lay::VS)
-                        mbar_wait(bars + Lay::B_VEMPTY + vs, ((g / Lay::VS) - 1) & 1, abort_flag);
-                    if (!*abort_flag) {
-                        mbar_arrive_expect_tx(bars + Lay::B_VFULL + vs, Lay::TILE_BYTES);
+                            for (int c = 0; c < Lay::DCH; ++c)
+                                tma_load_3d(smem + Lay::OFF_K + ks * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                            tree ? &map_kt : &map_kc, bars + Lay::B_KFULL + ks, c * 64,
+                                            row, u, pol);
+                        }
+                    } else {
+                        const int vs = g % Lay::VS;
+                        if (g >= Lay::VS)
+                            mbar_wait(bars + Lay::B_VEMPTY + vs, ((g / Lay::VS) - 1) & 1, abort_flag);
+                        if (!*abort_flag) {
+                            mbar_arrive_expect_tx(bars + Lay::B_VFULL + vs, Lay::TILE_BYTES);
 #pragma unroll
-                        for (int c = 0; c < Lay::DCH; ++c)
-                            tma_load_3d(smem + Lay::OFF_V + vs * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
-                                        tree ? &map_vt : &map_vc, bars + Lay::B_VFULL + vs, c * 64,
-                                        row, u, pol);
+                            for (int c = 0; c < Lay::DCH; ++c)
+                                tma_load_3d(smem + Lay::OFF_V + vs * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                            tree ? &map_vt : &map_vc, bars + Lay::B_VFULL + vs, c * 64,
+                                            row, u, pol);
+                        }
                     }
                 }
             }
             if (*abort_flag) {
-                for (int i = max(0, g - Lay::KS); i < g; ++i)
-                    mbar_wait_drain(bars + Lay::B_KFULL + i % Lay::KS, (i / Lay::KS) & 1);
-                for (int i = max(0, g - Lay::VS); i < g; ++i)
-                    mbar_wait_drain(bars + Lay::B_VFULL + i % Lay::VS, (i / Lay::VS) & 1);
-                for (int i = max(0, k - Lay::QS); i < k; ++i)
-                    mbar_wait_drain(bars + Lay::B_QFULL + i % Lay::QS, (i / Lay::QS) & 1);
+                // let every copy already issued land before the CTA can exit
+                if (kq) {
+                    for (int i = max(0, g - Lay::KS); i < g; ++i)
+                        mbar_wait_drain(bars + Lay::B_KFULL + i % Lay::KS, (i / Lay::KS) & 1);
+                    for (int i = max(0, k - Lay::QS); i < k; ++i)
+                        mbar_wait_drain(bars + Lay::B_QFULL + i % Lay::QS, (i / Lay::QS) & 1);
+                } else {
+                    for (int i = max(0, g - Lay::VS); i < g; ++i)
+                        mbar_wait_drain(bars + Lay::B_VFULL + i % Lay::VS, (i / Lay::VS) & 1);
+                }
             }
         }
     } else if (warp == 9) {
@@ -521,8 +537,8 @@ static cudaError_t launch_rows_t(const AttnMaps &m, const AttnParams &p, int num
                                  bool programmatic, cudaStream_t stream)
 {
     static std::atomic<uint64_t> configured{0};
-    return launch_attention_grid(tree_attention_rows_kernel<D>, RowsLayout<D>::SMEM_BYTES, configured,
-                                 m, p, num_sms, programmatic, stream);
+    return launch_attention_grid(tree_attention_rows_kernel<D>, RowsLayout<D>::SMEM_BYTES, 384,
+                                 configured, m, p, num_sms, programmatic, stream);
 }
 
 cudaError_t launch_tree_attention_rows(const AttnMaps &m, const AttnParams &p, int D, int num_sms,

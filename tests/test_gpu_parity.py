@@ -106,6 +106,55 @@ def test_attention_edge_sizes(cuda_device, T, P):
     assert_attn_close(out.cpu().numpy().reshape(ref.shape), ref, f"T={T} P={P}")
 
 
+def test_attention_values_beyond_f16(cuda_device):
+    """Trees of 65..128 tokens apply P V in f16 wherever a V tile fits f16 and in
+    bf16 hi + lo elsewhere: tiles holding values beyond the f16 range (a prefix
+    tile, the tree tile) must still match the oracle."""
+    w = W.scaled(W.WORKLOADS["vicuna13b"], L=1, H=2, P=700)
+    pl = np.array([700], np.int32)
+    s = W.make_step_inputs(w, prefix_len=pl)
+    t = tensors(w, prefix_len=pl)
+    vc = t["v_cache"].float()
+    vc[0, 0, 0, 130:140] *= 2.0e5                    # head 0, second prefix tile
+    vc[0, 0, 1, 650, :7] = -7.0e4                    # head 1, last (partial) prefix tile
+    t["v_cache"] = vc.to(torch.bfloat16)
+    vt = t["v_tree"].float()
+    vt[0, 0, 1, 5] *= 1.0e5                          # head 1, tree tile
+    t["v_tree"] = vt.to(torch.bfloat16)
+    out, _, st = run_attention({k: v.to(cuda_device) for k, v in t.items()}, pl, s.parent,
+                               cuda_device)
+    ref, _, _, _ = oracle.tree_attention(t["q"], t["k_cache"], t["v_cache"], t["k_tree"],
+                                         t["v_tree"], pl, s.parent)
+    got = out.cpu().numpy().reshape(ref.shape).astype(np.float64)
+    assert np.isfinite(got).all()
+    for u in range(ref.shape[0]):                    # per slice, relative to its magnitude
+        scale = np.abs(ref[u]).max()
+        assert np.abs(got[u] - ref[u]).max() <= 5e-3 * max(scale, 1.0), u
+        assert np.linalg.norm(got[u] - ref[u]) <= 1e-3 * np.linalg.norm(ref[u]), u
+
+
+@pytest.mark.parametrize("T,P", [(100, 300), (65, 128)])
+def test_attention_rows_head_dim_64(cuda_device, T, P):
+    """The 65..128-token kernel with 64-wide heads."""
+    rng = np.random.default_rng(T + P)
+    B, H, D = 2, 3, 64
+    parent = np.full((B, T), -1, np.int32)
+    for b in range(B):
+        for i in range(1, T):
+            parent[b, i] = rng.integers(0, i)
+    w = W.Workload("rows64", L=1, B=B, H=H, D=D, P=P, T=T, V=16, n_cand=T, max_depth=T,
+                   chains="every0", match_rate=0.5, seed=T * 7 + P)
+    pl = np.array([P, P // 3], np.int32)
+    t = tensors(w, prefix_len=pl)
+    out, lse, st = run_attention({k: v.to(cuda_device) for k, v in t.items()}, pl, parent,
+                                 cuda_device)
+    ref, ref_lse, _, _ = oracle.tree_attention(t["q"], t["k_cache"], t["v_cache"], t["k_tree"],
+                                               t["v_tree"], pl, parent)
+    assert_attn_close(out.cpu().numpy().reshape(ref.shape), ref, f"D=64 T={T}")
+    np.testing.assert_allclose(lse.cpu().numpy().reshape(ref_lse.shape), ref_lse, rtol=0,
+                               atol=1e-3)
+
+
 def test_attention_peaked_scores_and_scale(cuda_device):
     """Large scores force the running-max rescale path on later tiles."""
     w = W.scaled(W.WORKLOADS["vicuna7b"], L=1, H=2, P=1000)
