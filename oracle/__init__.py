@@ -77,6 +77,11 @@ def _load():
                                               c_int, c_dbl, c_dbl, c_dbl, i32p, i32p, i32p, i32p,
                                               i32p, f64p, f64p]
         lib.oracle_typical_accept.restype = c_int
+        lib.oracle_topk.argtypes = [vp, c_i64, c_i64, c_int, i32p]
+        lib.oracle_topk.restype = None
+        lib.oracle_next_tree.argtypes = [vp, i32p, i32p, i32p, i32p, i32p, c_int, c_int, c_int,
+                                         c_int, c_int, i32p, i32p, c_int, i32p, i32p, i32p, i32p]
+        lib.oracle_next_tree.restype = c_int
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = c_int
         _lib = lib
@@ -236,6 +241,42 @@ def typical_accept(logits, argmax, cand_tokens, parent, prefix_len, S_max: int,
         p(res["new_prefix_len"]), p(res["status"]), d(res["p_tok"]), d(res["threshold"]))
     if rc != 0:
         raise ValueError(f"oracle_typical_accept rejected its arguments (code {rc})")
+    return res
+
+
+def topk(logits, K: int) -> np.ndarray:
+    """The K best tokens of each row (last axis) of fp32 logits, in ranking
+    order: NaN first (lower index first), then larger value, then lower index."""
+    a, _ = _host(logits)
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    V = a.shape[-1]
+    rows = a.size // V if V else 0
+    out = np.empty(a.shape[:-1] + (K,), np.int32)
+    _load().oracle_topk(_ptr(a), rows, V, int(K), _ptr(out, ctypes.c_int32))
+    return out
+
+
+def next_tree(logits, parent, cand_tokens, path, accept_len, next_token, tmpl_parent, tmpl_rank,
+              K: int):
+    """Next-step candidate tree.  logits [B,T,V]; parent, cand_tokens, path
+    [B,T]; accept_len, next_token [B]; tmpl_parent, tmpl_rank [n_states,
+    T_next].  Returns dict of next_parent, next_cand [B,T_next], next_state,
+    status [B]."""
+    lg, _ = _host(logits)
+    lg = np.ascontiguousarray(lg, dtype=np.float32)
+    par, cd, pth, al, nt = (_i32(x) for x in (parent, cand_tokens, path, accept_len, next_token))
+    tp, tr = _i32(tmpl_parent), _i32(tmpl_rank)
+    B, T = par.shape
+    V = lg.shape[-1]
+    n_states, T_next = tp.shape
+    res = {"next_parent": np.empty((B, T_next), np.int32), "next_cand": np.empty((B, T_next), np.int32),
+           "next_state": np.empty(B, np.int32), "status": np.empty(B, np.int32)}
+    p = lambda a: _ptr(a, ctypes.c_int32)
+    rc = _load().oracle_next_tree(_ptr(lg), p(par), p(cd), p(pth), p(al), p(nt), B, T, V, n_states,
+                                  T_next, p(tp), p(tr), int(K), p(res["next_parent"]),
+                                  p(res["next_cand"]), p(res["next_state"]), p(res["status"]))
+    if rc != 0:
+        raise ValueError(f"oracle_next_tree rejected its arguments (code {rc})")
     return res
 
 

@@ -25,6 +25,10 @@
  *   oracle_node_stats      log-sum-exp and entropy of softmax(logits / tau)
  *   oracle_typical_accept  typical acceptance (Section 3 step (2), the
  *                          second verification scheme the paper names)
+ *   oracle_topk            the K best tokens of logits rows (ranking order)
+ *   oracle_next_tree       next-step candidate tree from the accepted node's
+ *                          prompt tokens (Section 3 step (1); Appendix,
+ *                          tree states T_k)
  *
  * Status codes (per sequence): 0 ok, 3 malformed tree, 4 capacity / prefix
  * length out of range.  Whole-call argument errors return 1.
@@ -454,6 +458,149 @@ int oracle_typical_accept(const float *logits, const int32_t *argmax, const int3
     free(ok);
     free(lse);
     free(ent);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------ next-step candidates */
+
+/* Ranking of tokens by logit: a NaN before any number (the lower index first
+ * among NaNs), then the larger value, then the lower index -- the argmax rule
+ * extended to an order. */
+static int ranks_before(float av, int64_t ai, float bv, int64_t bi)
+{
+    int an = isnan(av), bn = isnan(bv);
+    if (an || bn)
+        return an && bn ? ai < bi : an;
+    if (av != bv)
+        return av > bv;
+    return ai < bi;
+}
+
+/*
+ * The K best tokens of each logits row [rows, V] in ranking order, out
+ * [rows][K], by repeated selection of the best token not yet taken.
+ * Requires 1 <= K <= V.
+ */
+void oracle_topk(const float *logits, int64_t rows, int64_t V, int K, int32_t *out)
+{
+    char *taken = (char *)malloc((size_t)V);
+    for (int64_t r = 0; r < rows; ++r) {
+        const float *x = logits + r * V;
+        memset(taken, 0, (size_t)V);
+        for (int k = 0; k < K; ++k) {
+            int64_t best = -1;
+            for (int64_t v = 0; v < V; ++v)
+                if (!taken[v] && (best < 0 || ranks_before(x[v], v, x[best], best)))
+                    best = v;
+            taken[best] = 1;
+            out[r * K + k] = (int32_t)best;
+        }
+    }
+    free(taken);
+}
+
+/*
+ * Next-step candidate tree of each sequence (Section 3 step (1): the prompt
+ * tokens appended to a guess token predict the tokens after it; Appendix,
+ * Definition of tree states: a tree exists in states T_k whose candidate
+ * subtree has depth at most k, k being set by the prompt tokens available).
+ *
+ * e = path[b][accept_len[b] - 1] is the accepted end node.  Its prompt chain:
+ * c_1 = the lowest-index child of e with cand_tokens -1, c_(j+1) the
+ * lowest-index such child of c_j; k = the chain length, capped at n_states-1.
+ * The K best tokens (oracle_topk order) of the logits at c_d are the guesses
+ * for depth d of the next tree.  Template state k: tmpl_parent[k][i] (node 0
+ * the root, parent -1) and tmpl_rank[k][i] (rank r >= 0: a candidate node, -1:
+ * a prompt node; ignored for the root).  Outputs: next_parent[b] =
+ * tmpl_parent[k]; next_cand[b][0] = next_token[b]; a candidate node at
+ * candidate depth d (candidate nodes on its path, root excluded) gets guess r
+ * of depth d; prompt nodes get -1; next_state[b] = k.  Status 3 (and outputs
+ * all -1, next_state -1) when accept_len[b] < 1, next_token[b] < 0, or
+ * template k is not a tree in topological order, has a candidate below a
+ * prompt node, a candidate deeper than k, or a rank outside [0, K).
+ */
+int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *cand,
+                     const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
+                     int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
+                     const int32_t *tmpl_rank, int K, int32_t *next_parent, int32_t *next_cand,
+                     int32_t *next_state, int32_t *status)
+{
+    if (B < 1 || T < 1 || V < 1 || n_states < 1 || T_next < 1 || K < 1 || K > V)
+        return ORC_ERR_INVALID_ARG;
+    int32_t *top = (int32_t *)malloc(sizeof(int32_t) * (size_t)K);
+    int *cdepth = (int *)malloc(sizeof(int) * (size_t)T_next);
+    int *chain = (int *)malloc(sizeof(int) * (size_t)(T + 1));
+    for (int b = 0; b < B; ++b) {
+        const int32_t *par = parent + (int64_t)b * T;
+        const int32_t *tok = cand + (int64_t)b * T;
+        int32_t *np = next_parent + (int64_t)b * T_next;
+        int32_t *nc = next_cand + (int64_t)b * T_next;
+        int err = ORC_OK, k = 0;
+        int n = accept_len[b];
+        if (n < 1 || n > T || next_token[b] < 0)
+            err = ORC_ERR_TREE;
+        if (err == ORC_OK) {
+            int e = path[(int64_t)b * T + n - 1];
+            /* the prompt chain below the end node */
+            int cur = e;
+            while (1) {
+                int nxt = -1;
+                for (int i = cur + 1; i < T; ++i)
+                    if (par[i] == cur && tok[i] == -1) {
+                        nxt = i;
+                        break;
+                    }
+                if (nxt < 0)
+                    break;
+                chain[k++] = nxt;
+                cur = nxt;
+            }
+            if (k > n_states - 1)
+                k = n_states - 1;
+            /* template k */
+            const int32_t *tp = tmpl_parent + (int64_t)k * T_next;
+            const int32_t *tr = tmpl_rank + (int64_t)k * T_next;
+            if (!tree_is_valid(tp, T_next))
+                err = ORC_ERR_TREE;
+            for (int i = 1; i < T_next && err == ORC_OK; ++i) {
+                int p = tp[i];
+                if (tr[i] >= 0) {
+                    if (p > 0 && tr[p] < 0)
+                        err = ORC_ERR_TREE;          /* a candidate below a prompt node */
+                    cdepth[i] = (p == 0 ? 0 : cdepth[p]) + 1;
+                    if (cdepth[i] > k || tr[i] >= K)
+                        err = ORC_ERR_TREE;
+                } else {
+                    cdepth[i] = -1;
+                }
+            }
+            if (err == ORC_OK) {
+                for (int i = 0; i < T_next; ++i) {
+                    np[i] = tp[i];
+                    nc[i] = -1;
+                }
+                nc[0] = next_token[b];
+                for (int d = 1; d <= k; ++d) {
+                    oracle_topk(logits + ((int64_t)b * T + chain[d - 1]) * V, 1, V, K, top);
+                    for (int i = 1; i < T_next; ++i)
+                        if (tr[i] >= 0 && cdepth[i] == d)
+                            nc[i] = top[tr[i]];
+                }
+                next_state[b] = k;
+            }
+        }
+        if (err != ORC_OK) {
+            for (int i = 0; i < T_next; ++i) {
+                np[i] = -1;
+                nc[i] = -1;
+            }
+            next_state[b] = -1;
+        }
+        status[b] = err;
+    }
+    free(top);
+    free(cdepth);
+    free(chain);
     return ORC_OK;
 }
 

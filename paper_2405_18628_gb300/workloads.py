@@ -140,6 +140,56 @@ def _chain_lengths(rng, recipe: str, parent, depth, n_prompt: int) -> List[Tuple
     raise ValueError(f"unknown chain recipe {recipe!r}")
 
 
+def make_tree_templates(n_states: int, T_next: int, K: int, rng: np.random.Generator):
+    """Next-step tree templates, one per state k = 0..n_states-1 (the paper's
+    T_k, Appendix: the candidate subtree of T_k is at most k deep).  Node 0 is
+    the root; candidate nodes carry the rank (0..K-1) of the guess they take at
+    their depth, prompt nodes rank -1.  Candidates: up to K children of the root
+    at depth 1, then at each further depth up to K children of the depth's
+    rank-0 node and of one other random candidate, within a budget of
+    T_next // 4 candidates; prompt chains of up to n_states-1 tokens then hang
+    below the root and the candidates, in index order, filling exactly T_next
+    nodes.  Returns (parent, rank), both int32 [n_states, T_next]."""
+    m = n_states - 1
+    parent = np.full((n_states, T_next), -1, np.int32)
+    rank = np.full((n_states, T_next), -1, np.int32)
+    for k in range(n_states):
+        par, rk, depth = [-1], [0], [0]
+        budget = max(1, T_next // 4)
+        level = [0]
+        for d in range(1, k + 1):
+            anchors = [level[0]]
+            if len(level) > 1:
+                anchors.append(level[1 + int(rng.integers(len(level) - 1))])
+            nxt = []
+            for a in anchors:
+                for r in range(K):
+                    if len(par) >= budget:
+                        break
+                    par.append(a)
+                    rk.append(r)
+                    depth.append(d)
+                    nxt.append(len(par) - 1)
+            if not nxt:
+                break
+            level = nxt
+        n_cand = len(par)
+        for a in range(n_cand):
+            prev = a
+            for _ in range(m):
+                if len(par) >= T_next:
+                    break
+                par.append(prev)
+                rk.append(-1)
+                prev = len(par) - 1
+        while len(par) < T_next:                  # more room than chains: extend the root's
+            par.append(len(par) - 1 if rk[-1] == -1 else 0)
+            rk.append(-1)
+        parent[k] = par[:T_next]
+        rank[k] = rk[:T_next]
+    return parent, rank
+
+
 def make_tree(rng: np.random.Generator, w: Workload):
     """One sequence's tree.  Returns (parent int32[T], is_prompt bool[T]).
 

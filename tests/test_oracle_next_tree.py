@@ -1,0 +1,146 @@
+"""Pins for the oracle's next-step candidate generation (Section 3 step (1):
+the prompt tokens appended to the accepted token predict the following
+tokens; Appendix, Definition of tree states: the next tree takes state T_k,
+whose candidate subtree is at most k deep).
+
+Expected values come from numpy's stable argsort (top-k order), a hand-worked
+example, an independent restatement on small random cases (chain found by a
+breadth-first search over the tree, ranks by numpy), and the state rule."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2405_18628_gb300 import workloads as W
+
+
+def test_topk_matches_numpy_stable_sort():
+    rng = np.random.default_rng(0)
+    x = (rng.standard_normal((7, 301)) * 2).astype(np.float32)
+    x[0, [10, 20, 30]] = x[0].max() + 1.0          # a three-way tie at the top: lower index first
+    x[1, :] = 0.0                                   # all equal: indices 0, 1, 2, ...
+    got = oracle.topk(x, 9)
+    for r in range(x.shape[0]):
+        ref = np.lexsort((np.arange(x.shape[1]), -x[r]))[:9]
+        assert got[r].tolist() == ref.tolist(), r
+    assert got[0, :3].tolist() == [10, 20, 30]
+    assert got[1].tolist() == list(range(9))
+
+
+def test_topk_nan_first_then_values():
+    x = np.array([[1.0, np.nan, 5.0, np.nan, 3.0, 5.0]], np.float32)
+    assert oracle.topk(x, 6)[0].tolist() == [1, 3, 2, 5, 4, 0]
+    # rank 0 is the argmax rule
+    rng = np.random.default_rng(4)
+    y = rng.standard_normal((20, 77)).astype(np.float32)
+    assert (oracle.topk(y, 1)[:, 0] == oracle.node_argmax(y)).all()
+
+
+def test_hand_worked_example():
+    # this step's tree: 0 root; 1, 2 candidates under 0; 3 candidate under 1;
+    # 4 -> 5 -> 6 a prompt chain under 3; 7 a prompt node under 2.
+    parent = np.array([[-1, 0, 0, 1, 3, 4, 5, 2]])
+    cand = np.array([[9, 4, 7, 2, -1, -1, -1, -1]])
+    V = 6
+    logits = np.zeros((1, 8, V), np.float32)
+    logits[0, 4] = [0, 1, 5, 3, 2, 4]      # chain node c_1 -> ranking 2, 5, 3, 4, 1, 0
+    logits[0, 5] = [6, 0, 0, 7, 0, 1]      # c_2 -> 3, 0, 5, 1, 2, 4
+    logits[0, 6] = [9, 9, 9, 9, 9, 9]      # c_3 -> 0, 1, 2, ...
+    path = np.array([[0, 1, 3, -1, -1, -1, -1, -1]])
+    accept_len, next_token = np.array([3]), np.array([4])
+    # templates for states 0..2 with T_next = 6
+    tp = np.array([[-1, 0, 1, 2, 3, 4],            # k=0: root + a prompt chain
+                   [-1, 0, 0, 1, 2, 3],            # k=1: two depth-1 candidates (ranks 1, 0)
+                   [-1, 0, 1, 1, 0, 4]])           # k=2: depth1 r0, depth2 r0 and r2, prompts
+    tr = np.array([[0, -1, -1, -1, -1, -1],
+                   [0, 1, 0, -1, -1, -1],
+                   [0, 0, 0, 2, -1, -1]])
+    r = oracle.next_tree(logits, parent, cand, path, accept_len, next_token, tp, tr, K=3)
+    # end node 3 has the chain 4, 5, 6 (k = 3), capped at n_states - 1 = 2
+    assert r["status"].tolist() == [0] and r["next_state"].tolist() == [2]
+    assert r["next_parent"][0].tolist() == [-1, 0, 1, 1, 0, 4]
+    # node 1: depth 1 rank 0 -> c_1's best (2); nodes 2, 3: depth 2 ranks 0, 2 -> c_2's 3 and 5
+    assert r["next_cand"][0].tolist() == [4, 2, 3, 5, -1, -1]
+
+
+def _independent(logits, parent, cand, path, accept_len, next_token, tp, tr, K):
+    """Restatement: the chain is found by breadth-first search from the end node
+    over prompt children (lowest index first), ranks come from numpy."""
+    B, T = parent.shape
+    n_states, T_next = tp.shape
+    out_p = np.full((B, T_next), -1)
+    out_c = np.full((B, T_next), -1)
+    out_s = np.full(B, -1)
+    for b in range(B):
+        e = path[b, accept_len[b] - 1]
+        children = {u: sorted(i for i in range(T) if parent[b, i] == u and cand[b, i] == -1)
+                    for u in range(T)}
+        chain, u = [], e
+        while children[u]:
+            u = children[u][0]
+            chain.append(u)
+        k = min(len(chain), n_states - 1)
+        ranks = [np.lexsort((np.arange(logits.shape[2]), -logits[b, c]))[:K] for c in chain]
+        depth = {0: 0}
+        for i in range(1, T_next):
+            depth[i] = depth[tp[k, i]] + 1 if tr[k, i] >= 0 else None
+        out_p[b] = tp[k]
+        out_c[b, 0] = next_token[b]
+        for i in range(1, T_next):
+            if tr[k, i] >= 0:
+                out_c[b, i] = ranks[depth[i] - 1][tr[k, i]]
+        out_s[b] = k
+    return out_p, out_c, out_s
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_random_cases_match_independent_restatement(seed):
+    rng = np.random.default_rng(seed)
+    w = W.scaled(W.WORKLOADS["tiny"], B=5, V=200)
+    s = W.make_step_inputs(w, seed=seed)
+    acc = oracle.accept_path(oracle.node_argmax(s.logits), s.cand_tokens, s.parent, s.prefix_len,
+                             w.V, w.S_max)
+    n_states, T_next, K = 3 + seed % 3, 24 + 8 * (seed % 2), 4
+    tp, tr = W.make_tree_templates(n_states, T_next, K, rng)
+    r = oracle.next_tree(s.logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                         acc["next_token"], tp, tr, K)
+    ref_p, ref_c, ref_s = _independent(s.logits, s.parent, s.cand_tokens, acc["path"],
+                                       acc["accept_len"], acc["next_token"], tp, tr, K)
+    assert (r["status"] == 0).all()
+    np.testing.assert_array_equal(r["next_parent"], ref_p)
+    np.testing.assert_array_equal(r["next_cand"], ref_c)
+    np.testing.assert_array_equal(r["next_state"], ref_s)
+
+
+def test_templates_respect_the_state_depth_rule():
+    tp, tr = W.make_tree_templates(5, 64, 4, np.random.default_rng(2))
+    for k in range(5):
+        depth = {0: 0}
+        for i in range(1, 64):
+            assert 0 <= tp[k, i] < i
+            if tr[k, i] >= 0:
+                assert tp[k, i] == 0 or tr[k, tp[k, i]] >= 0
+                depth[i] = depth[tp[k, i]] + 1
+                assert depth[i] <= k
+        assert k == 0 or max(depth.values()) >= 1    # every state with k >= 1 has guesses
+
+
+def test_next_tree_errors():
+    parent = np.array([[-1, 0, 1], [-1, 0, 1]])
+    cand = np.array([[3, -1, -1], [3, -1, -1]])
+    logits = np.zeros((2, 3, 4), np.float32)
+    path = np.array([[0, -1, -1], [0, -1, -1]])
+    tp = np.array([[-1, 0, 1], [-1, 0, 1]])
+    bad_rank = np.array([[0, -1, -1], [0, 7, -1]])      # state 1 asks for rank 7 of K = 2
+    r = oracle.next_tree(logits, parent, cand, path, np.array([1, 0]), np.array([1, 1]), tp,
+                         bad_rank, K=2)
+    assert r["status"].tolist() == [3, 3]                # rank outside K; failed acceptance
+    assert (r["next_parent"] == -1).all() and (r["next_state"] == -1).all()
+    deep = np.array([[0, -1, -1], [0, 0, 0]])           # state 1 with a depth-2 candidate
+    r = oracle.next_tree(logits, parent, cand, path, np.array([1, 1]), np.array([1, 1]), tp,
+                         deep, K=2)
+    assert r["status"].tolist() == [3, 3]
+    ok = np.array([[0, -1, -1], [0, 1, -1]])
+    r = oracle.next_tree(logits, parent, cand, path, np.array([1, 1]), np.array([1, 2]), tp, ok,
+                         K=2)
+    assert r["status"].tolist() == [0, 0] and r["next_state"].tolist() == [1, 1]
+    assert r["next_cand"].tolist() == [[1, 1, -1], [2, 1, -1]]   # c_1 logits all 0: rank 1 is token 1
