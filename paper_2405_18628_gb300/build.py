@@ -1,6 +1,6 @@
 """Build libppd.so (sm_103a) in-tree with nvcc.
 
-The library is compiled from the four CUDA translation units under csrc/
+The library is compiled from the five CUDA translation units under csrc/
 in parallel and linked with the static CUDA runtime.  The result lands next
 to this file as ``libppd.so`` and is what the Python binding loads.
 """
@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libppd.so")
-SOURCES = ["ppd_api.cu", "ppd_attention.cu", "ppd_attention_rows.cu", "ppd_verify.cu"]
+SOURCES = ["ppd_api.cu", "ppd_attention.cu", "ppd_attention_rows.cu", "ppd_verify.cu", "ppd_next.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

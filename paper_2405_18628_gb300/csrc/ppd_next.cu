@@ -1,0 +1,259 @@
+// ppd_next.cu -- next-step candidate tree of the PPD decode loop (paper
+// Section 3 step (1): the prompt tokens appended to a guess token predict the
+// tokens that follow it; Appendix, Definition of tree states: the next tree
+// takes state T_k, whose candidate subtree is at most k deep, k being the
+// number of prompt tokens left below the accepted token).
+//
+// Kernel 1, one block per (sequence, chain position d): finds the prompt
+// chain below the accepted end node (warp ballots over the parent array) and,
+// if d is within the state, the K best tokens of the chain node's logits --
+// every thread keeps its own top-K over a strided slice of the row, then K
+// rounds of a block-wide best-of-heads merge.  Kernel 2, one warp per
+// sequence: fills the state's template with the root token and the guesses.
+#include "ppd.h"
+#include "ppd_accept.cuh"
+#include "ppd_device.cuh"
+#include "ppd_kernels.h"
+
+#include <climits>
+
+namespace ppd {
+
+// The prompt chain below node e of one sequence (lowest-index prompt child at
+// each step), computed by one warp; returns its length (<= cap) and writes the
+// nodes to chain[0..len).
+PPD_DEV int prompt_chain(const int32_t *par, const int32_t *tok, int T, int e, int cap, int lane,
+                         int *chain)
+{
+    int len = 0, cur = e;
+    while (len < cap) {
+        int nxt = INT_MAX;
+        for (int i0 = 0; i0 < T; i0 += 32) {
+            const int i = i0 + lane;
+            const bool hit = i < T && i > cur && __ldg(par + i) == cur && __ldg(tok + i) == -1;
+            const unsigned m = __ballot_sync(0xffffffffu, hit);
+            if (m) {
+                nxt = i0 + __ffs(m) - 1;
+                break;
+            }
+        }
+        if (nxt == INT_MAX) break;
+        if (lane == 0) chain[len] = nxt;
+        ++len;
+        cur = nxt;
+    }
+    __syncwarp();
+    return len;
+}
+
+// Top-K (K <= kNextMaxK) of the logits of chain node d (1-based) of sequence
+// b, written to topk[(b * (n_states - 1) + d - 1) * K ...] in ranking order
+// (NaN first, then larger value, then lower index).
+__global__ void __launch_bounds__(256)
+next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const int32_t *cand,
+                 const int32_t *path, const int32_t *accept_len, int T, int V, int n_states, int K,
+                 int32_t *topk)
+{
+    __shared__ int s_chain[128];
+    __shared__ int s_len;
+    __shared__ float s_v[8];
+    __shared__ int s_i[8], s_t[8];
+    __shared__ int s_win;
+    const int b = blockIdx.x;
+    const int d = blockIdx.y + 1;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n = __ldg(accept_len + b);
+    if (warp == 0) {
+        int len = 0;
+        if (n >= 1 && n <= T) {
+            const int e = __ldg(path + (size_t)b * T + n - 1);
+            if (e >= 0 && e < T)
+                len = prompt_chain(parent + (size_t)b * T, cand + (size_t)b * T, T, e, n_states - 1,
+                                   lane, s_chain);
+        }
+        if (lane == 0) s_len = len;
+    }
+    __syncthreads();
+    if (d > s_len) return;   // uniform over the block
+    const float *x = logits + ((size_t)b * T + s_chain[d - 1]) * V;
+
+    // this thread's best K over its slice, best first
+    float hv[kNextMaxK];
+    int hi[kNextMaxK];
+#pragma unroll
+    for (int r = 0; r < kNextMaxK; ++r) {
+        hv[r] = -INFINITY;
+        hi[r] = INT_MAX;
+    }
+    float tv = -INFINITY;   // the K-th best so far (the entry a new token must beat)
+    int ti = INT_MAX;
+    for (int v = threadIdx.x; v < V; v += 256) {
+        const float xv = __ldcs(x + v);
+        if (!ranks_before(xv, v, tv, ti)) continue;
+        // insert, shifting worse entries down (slots K.. stay unused)
+        float cv = xv;
+        int ci = v;
+#pragma unroll
+        for (int r = 0; r < kNextMaxK; ++r) {
+            if (r < K && ranks_before(cv, ci, hv[r], hi[r])) {
+                const float sv = hv[r];
+                const int si = hi[r];
+                hv[r] = cv;
+                hi[r] = ci;
+                cv = sv;
+                ci = si;
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < kNextMaxK; ++r)
+            if (r == K - 1) {
+                tv = hv[r];
+                ti = hi[r];
+            }
+    }
+
+    // K rounds: the best head over the block is the next token; its owner pops it
+    for (int r = 0; r < K; ++r) {
+        float bv = hv[0];
+        int bi = hi[0], bt = threadIdx.x;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+            const int ot = __shfl_xor_sync(0xffffffffu, bt, off);
+            if (ranks_before(ov, oi, bv, bi)) {
+                bv = ov;
+                bi = oi;
+                bt = ot;
+            }
+        }
+        if (lane == 0) {
+            s_v[warp] = bv;
+            s_i[warp] = bi;
+            s_t[warp] = bt;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            for (int w = 1; w < 8; ++w)
+                if (ranks_before(s_v[w], s_i[w], bv, bi)) {
+                    bv = s_v[w];
+                    bi = s_i[w];
+                    bt = s_t[w];
+                }
+            topk[((size_t)b * (n_states - 1) + d - 1) * K + r] = bi;
+            s_win = bt;
+        }
+        __syncthreads();
+        if ((int)threadIdx.x == s_win) {
+#pragma unroll
+            for (int q = 0; q + 1 < kNextMaxK; ++q) {
+                hv[q] = hv[q + 1];
+                hi[q] = hi[q + 1];
+            }
+            hv[kNextMaxK - 1] = -INFINITY;
+            hi[kNextMaxK - 1] = INT_MAX;
+        }
+        __syncthreads();
+    }
+}
+
+// One warp per sequence: state, template checks, and the next tree.
+__global__ void __launch_bounds__(128)
+next_assemble_kernel(const int32_t *parent, const int32_t *cand, const int32_t *path,
+                     const int32_t *accept_len, const int32_t *next_token, int B, int T,
+                     int n_states, int T_next, const int32_t *tmpl_parent, const int32_t *tmpl_rank,
+                     int K, const int32_t *topk, int32_t *next_parent, int32_t *next_cand,
+                     int32_t *next_state, int32_t *status)
+{
+    __shared__ int s_chain[4][128];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.x * 4 + warp;
+    if (b >= B) return;
+    const int n = __ldg(accept_len + b);
+    const int nt = __ldg(next_token + b);
+    bool bad = !(n >= 1 && n <= T && nt >= 0);
+    int k = 0;
+    if (!bad) {
+        const int e = __ldg(path + (size_t)b * T + n - 1);
+        bad = !(e >= 0 && e < T);
+        if (!bad)
+            k = prompt_chain(parent + (size_t)b * T, cand + (size_t)b * T, T, e, n_states - 1, lane,
+                             s_chain[warp]);
+    }
+    const int32_t *tp = tmpl_parent + (size_t)k * T_next;
+    const int32_t *tr = tmpl_rank + (size_t)k * T_next;
+    int32_t *np = next_parent + (size_t)b * T_next;
+    int32_t *nc = next_cand + (size_t)b * T_next;
+    // template checks and each node's candidate depth (walk to the root)
+    for (int i = lane; i < T_next && !bad; i += 32) {
+        const int pi = __ldg(tp + i);
+        if (i == 0) {
+            bad |= pi != -1;
+            continue;
+        }
+        bad |= pi < 0 || pi >= i;
+        const int r = __ldg(tr + i);
+        if (r >= 0) bad |= r >= K;
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    if (!bad) {
+        for (int i = lane; i < T_next; i += 32) {
+            const int r = __ldg(tr + i);
+            int tokv = -1;
+            if (i == 0) {
+                tokv = nt;
+            } else if (r >= 0) {
+                int depth = 0, a = i;
+                bool ok = true;
+                while (a > 0) {
+                    ok &= __ldg(tr + a) >= 0;     // every node above a candidate is a candidate
+                    ++depth;
+                    a = __ldg(tp + a);
+                }
+                if (!ok || depth > k) {
+                    tokv = INT_MIN;               // marks a bad template
+                } else {
+                    tokv = __ldg(topk + ((size_t)b * (n_states - 1) + depth - 1) * K + r);
+                }
+            }
+            nc[i] = tokv;
+            np[i] = __ldg(tp + i);
+        }
+        __syncwarp();
+        bool inv = false;
+        for (int i = lane; i < T_next; i += 32) inv |= nc[i] == INT_MIN;
+        bad = __any_sync(0xffffffffu, inv);
+    }
+    if (bad) {
+        for (int i = lane; i < T_next; i += 32) {
+            np[i] = -1;
+            nc[i] = -1;
+        }
+    }
+    if (lane == 0) {
+        next_state[b] = bad ? -1 : k;
+        status[b] = bad ? kErrTree : kOk;
+    }
+}
+
+cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const int32_t *cand,
+                             const int32_t *path, const int32_t *accept_len,
+                             const int32_t *next_token, int B, int T, int V, int n_states,
+                             int T_next, const int32_t *tmpl_parent, const int32_t *tmpl_rank, int K,
+                             int32_t *topk, int32_t *next_parent, int32_t *next_cand,
+                             int32_t *next_state, int32_t *status, cudaStream_t stream)
+{
+    if (n_states > 1) {
+        next_topk_kernel<<<dim3((unsigned)B, (unsigned)(n_states - 1)), 256, 0, stream>>>(
+            logits, parent, cand, path, accept_len, T, V, n_states, K, topk);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    next_assemble_kernel<<<(B + 3) / 4, 128, 0, stream>>>(parent, cand, path, accept_len, next_token,
+                                                          B, T, n_states, T_next, tmpl_parent,
+                                                          tmpl_rank, K, topk, next_parent,
+                                                          next_cand, next_state, status);
+    return cudaGetLastError();
+}
+
+}  // namespace ppd

@@ -1,0 +1,101 @@
+"""Next-step candidate tree on the GPU (through the C ABI) against the oracle,
+bit for bit: the state k picked from the accepted node's prompt chain, the
+top-K guesses per chain position (including ties, NaNs and -inf logits), and
+the assembled parent / candidate arrays; bad templates and failed sequences
+report PPD_ERR_TREE."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2405_18628_gb300 import ppd
+from paper_2405_18628_gb300 import workloads as W
+
+from test_gpu_parity import i32
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(dev, logits, parent, cand, path, accept_len, next_token, tp, tr, K):
+    B, T = parent.shape
+    n_states, T_next = tp.shape
+    out = {"next_parent": torch.full((B, T_next), -9, dtype=torch.int32, device=dev),
+           "next_cand": torch.full((B, T_next), -9, dtype=torch.int32, device=dev),
+           "next_state": torch.full((B,), -9, dtype=torch.int32, device=dev),
+           "status": torch.full((B,), -9, dtype=torch.int32, device=dev)}
+    ppd.ppd_next_tree(torch.from_numpy(np.ascontiguousarray(logits)).to(dev), i32(parent, dev),
+                      i32(cand, dev), i32(path, dev), i32(accept_len, dev), i32(next_token, dev),
+                      i32(tp, dev), i32(tr, dev), K, out["next_parent"], out["next_cand"],
+                      out["next_state"], out["status"])
+    torch.cuda.synchronize()
+    return {k: v.cpu().numpy() for k, v in out.items()}
+
+
+def _compare(got, ref):
+    for k in ("next_parent", "next_cand", "next_state", "status"):
+        np.testing.assert_array_equal(got[k], ref[k], err_msg=k)
+
+
+@pytest.mark.parametrize("name,overrides,n_states,T_next,K", [
+    ("tiny", {"B": 6}, 4, 48, 4),
+    ("mobilellama", {}, 5, 64, 8),
+    ("vicuna7b", {"B": 3}, 4, 96, 16),
+    ("sweep_t32", {"B": 8}, 3, 32, 1),
+])
+def test_next_tree_matches_oracle(cuda_device, name, overrides, n_states, T_next, K):
+    w = W.scaled(W.WORKLOADS[name], **overrides)
+    s = W.make_step_inputs(w)
+    logits = s.logits.copy()
+    logits[0, :, 5] = logits[0, :, 7] = 40.0          # ties at the top of every row of sequence 0
+    if w.B > 1:
+        logits[1, :, 11] = np.nan                     # NaN ranks first
+        logits[1, :, :3] = -np.inf
+    acc = oracle.accept_path(oracle.node_argmax(logits), s.cand_tokens, s.parent, s.prefix_len,
+                             w.V, w.S_max)
+    tp, tr = W.make_tree_templates(n_states, T_next, K, np.random.default_rng(w.T + K))
+    ref = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                           acc["next_token"], tp, tr, K)
+    assert (ref["status"] == 0).all()
+    got = _run(cuda_device, logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+               acc["next_token"], tp, tr, K)
+    _compare(got, ref)
+
+
+def test_next_tree_every_state(cuda_device):
+    """Hand-built trees whose accepted node carries prompt chains of length 0..5:
+    every state (capped at n_states - 1) is taken."""
+    B, T, V, K = 6, 12, 300, 3
+    parent = np.zeros((B, T), np.int32)
+    cand = np.zeros((B, T), np.int32)
+    path = np.full((B, T), -1, np.int32)
+    for b in range(B):
+        # root 0 -> candidate 1; chain of b prompt tokens under 1; the rest prompt nodes under 0
+        parent[b] = [-1, 0] + [1 + j for j in range(b)] + [0] * (T - 2 - b)
+        parent[b, 2] = 1 if b >= 1 else 0
+        cand[b] = [3, 4] + [-1] * (T - 2)
+        path[b, :2] = [0, 1]
+    rng = np.random.default_rng(9)
+    logits = rng.standard_normal((B, T, V)).astype(np.float32)
+    accept_len = np.full(B, 2, np.int32)
+    next_token = np.arange(B, dtype=np.int32) + 10
+    tp, tr = W.make_tree_templates(4, 40, K, rng)
+    ref = oracle.next_tree(logits, parent, cand, path, accept_len, next_token, tp, tr, K)
+    assert ref["next_state"].tolist() == [0, 1, 2, 3, 3, 3]
+    got = _run(cuda_device, logits, parent, cand, path, accept_len, next_token, tp, tr, K)
+    _compare(got, ref)
+
+
+def test_next_tree_errors(cuda_device):
+    B, T, V, K = 3, 4, 50, 2
+    parent = np.array([[-1, 0, 1, 2]] * B, np.int32)
+    cand = np.array([[3, -1, -1, -1]] * B, np.int32)
+    path = np.array([[0, -1, -1, -1]] * B, np.int32)
+    logits = np.random.default_rng(1).standard_normal((B, T, V)).astype(np.float32)
+    tp = np.array([[-1, 0, 1], [-1, 0, 0], [-1, 0, 1]], np.int32)
+    tr = np.array([[0, -1, -1], [0, 0, 1], [0, 0, 3]], np.int32)   # state 2: rank 3 >= K
+    accept_len = np.array([1, 0, 1], np.int32)                      # sequence 1 failed
+    next_token = np.array([5, 5, -1], np.int32)                     # sequence 2: no next token
+    ref = oracle.next_tree(logits, parent, cand, path, accept_len, next_token, tp, tr, K)
+    got = _run(cuda_device, logits, parent, cand, path, accept_len, next_token, tp, tr, K)
+    _compare(got, ref)
+    assert got["status"].tolist() == [3, 3, 3]       # state 2 template bad; failed; no token
