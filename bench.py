@@ -214,6 +214,9 @@ def parse():
     ap.add_argument("--tau", default="",
                     help="JSON file {tree size: acceptance length}: with --tree-sizes, also "
                          "report Speedup(n) = tau(n) / latency(n) and the best size")
+    ap.add_argument("--next-tree", action="store_true",
+                    help="also time next-step candidate generation (ppd_next_tree, 5 tree "
+                         "states, 8 guesses per depth) after each step")
     ap.add_argument("--layers", type=int, default=0,
                     help="run the workload with this many layers (profiling captures)")
     ap.add_argument("--l2", default="auto", choices=["auto", "flush", "none"],
@@ -442,6 +445,40 @@ def main():
     if world == 1 and rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, t, s, args.cpu_budget)
 
+    # ---------------------------------------------------------------- next-step candidates
+    next_tree = None
+    if args.next_tree:
+        n_states, K_guess = 5, 8
+        tp, tr = W.make_tree_templates(n_states, w.T, K_guess, np.random.default_rng(w.seed))
+        tp_d, tr_d = i32(tp), i32(tr)
+        nxt = {k: torch.empty(shape, dtype=torch.int32, device=dev) for k, shape in
+               (("parent", (w.B, w.T)), ("cand", (w.B, w.T)), ("state", (w.B,)), ("status", (w.B,)))}
+        ws_nt = torch.empty(max(256, ppd.load().ppd_next_tree_workspace_bytes(w.B, n_states, K_guess)),
+                            dtype=torch.uint8, device=dev)
+
+        def next_step():
+            ppd.ppd_next_tree(logits, parent, cand, bufs.path, bufs.accept_len, bufs.next_token,
+                              tp_d, tr_d, K_guess, nxt["parent"], nxt["cand"], nxt["state"],
+                              nxt["status"], workspace=ws_nt, stream=stream)
+
+        K4 = min(K, 200)
+        ev4 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(K4)]
+        for k in range(K4 + 3):
+            step()
+            if k >= 3:
+                ev4[k - 3][0].record(stream)
+            next_step()
+            if k >= 3:
+                ev4[k - 3][1].record(stream)
+        torch.cuda.synchronize()
+        if (nxt["status"].cpu().numpy() != 0).any():
+            raise SystemExit("next-step candidate generation reported an error")
+        nt_ms = statistics.median(a.elapsed_time(b) for a, b in ev4)
+        next_tree = {"us": nt_ms * 1e3, "states": n_states, "guesses_per_depth": K_guess,
+                     "state_histogram": np.bincount(nxt["state"].cpu().numpy(),
+                                                    minlength=n_states).tolist()}
+
     # ---------------------------------------------------------------- tree-size profile
     profile = None
     if args.tree_sizes:
@@ -495,6 +532,8 @@ def main():
         }
         if profile is not None:
             line["tree_size_profile"] = profile
+        if next_tree is not None:
+            line["next_tree"] = next_tree
         print(json.dumps(line), flush=True)
     if pg:
         pg.barrier()

@@ -26,7 +26,7 @@
  *    host-side checks and the work was enqueued; errors found on the device
  *    are reported per sequence in `dev_status`.
  *  - Shapes: L layers, B sequences, H heads (K/V heads == query heads), D head
- *    dim (64 or 128), T tree tokens (1..128), S_max cache rows per
+ *    dim (64 or 128), T tree tokens (1..512), S_max cache rows per
  *    (layer, sequence, head), V vocab size.
  *  - Q, tree K/V and the attention output are [L,B,H,T,D]; the K/V cache is
  *    [L,B,H,S_max,D]; rows [0, prefix_len[b]) of sequence b are the valid
@@ -234,7 +234,7 @@ ppd_status ppd_verify_step_typical(const void *q, void *k_cache, void *v_cache,
  * next_token[b] < 0, or template k is not a tree in topological order, has a
  * candidate below a prompt node, a candidate deeper than k or a rank >= K.
  * logits, parent, cand_tokens, path as for the verification step that just ran.
- * 1 <= K <= 16, K <= V; n_states, T_next <= 128.  Workspace:
+ * 1 <= K <= 16, K <= V; n_states <= 128; T_next <= 512.  Workspace:
  * ppd_next_tree_workspace_bytes(B, n_states, K) bytes.
  */
 size_t ppd_next_tree_workspace_bytes(int B, int n_states, int K);

@@ -5,6 +5,7 @@
 #pragma once
 
 #include "ppd_device.cuh"
+#include "ppd_kernels.h"
 
 #include <climits>
 
@@ -127,20 +128,21 @@ struct AcceptResult {
 //   pass    pass(i, parent, token): does candidate node i (token >= 0) pass its
 //           verification test
 //   par,tok the sequence's parent array and candidate token ids (global memory)
-//   s_par   T ints of per-warp scratch
+//   s_par   kAcceptScratchInts ints of per-warp scratch
 //   path    T outputs: accepted nodes in depth order, then -1
 // Node 0 is always accepted; node i > 0 when tok[i] >= 0, pass(i, par[i],
 // tok[i]) holds and its parent is accepted.  The end node is the deepest
 // accepted node, the smallest index among equal depths.  Every lane gets the
-// same result.
+// same result.  T <= kMaxTree.
 template <class TopLoad, class Pass>
 PPD_DEV AcceptResult accept_warp_pass(TopLoad top, Pass pass, const int32_t *par,
                                       const int32_t *tok, int P, int T, int V, int S_max, int lane,
                                       int *s_par, int32_t *path)
 {
+    uint32_t *s_ok = reinterpret_cast<uint32_t *>(s_par + kMaxTree);
+    const int nw = (T + 31) >> 5;
     bool bad = false;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < nw; ++k) {
         const int i = lane + 32 * k;
         if (i < T) {
             const int pa = __ldg(par + i);
@@ -156,9 +158,7 @@ PPD_DEV AcceptResult accept_warp_pass(TopLoad top, Pass pass, const int32_t *par
     bad = __any_sync(0xffffffffu, bad);
     int err = bad ? kErrTree : ((P < 0 || P > S_max) ? kErrCapacity : kOk);
 
-    uint32_t okw[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < nw; ++k) {
         const int i = lane + 32 * k;
         bool ok = false;
         if (i < T && err == kOk) {
@@ -169,35 +169,34 @@ PPD_DEV AcceptResult accept_warp_pass(TopLoad top, Pass pass, const int32_t *par
                 ok = tk >= 0 && pass(i, s_par[i], tk);
             }
         }
-        okw[k] = __ballot_sync(0xffffffffu, ok);
+        const uint32_t w = __ballot_sync(0xffffffffu, ok);
+        if (lane == 0) s_ok[k] = w;
     }
+    __syncwarp();
 
-    int best_key = -1;   // (depth << 8) | (255 - node): deepest, then smallest index
+    int best_key = -1;   // (depth << 10) | (1023 - node): deepest, then smallest index
     if (err == kOk) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
+        for (int k = 0; k < nw; ++k) {
             const int i = lane + 32 * k;
             if (i < T) {
                 int n = i, depth = 0;
                 bool good = true;
                 while (n > 0) {
-                    const uint32_t w = (n < 32) ? okw[0] : (n < 64) ? okw[1] : (n < 96) ? okw[2] : okw[3];
-                    good &= ((w >> (n & 31)) & 1u) != 0;
+                    good &= ((s_ok[n >> 5] >> (n & 31)) & 1u) != 0;
                     n = s_par[n];
                     ++depth;
                 }
-                if (good) best_key = max(best_key, (depth << 8) | (255 - i));
+                if (good) best_key = max(best_key, (depth << 10) | (1023 - i));
             }
         }
     }
     best_key = __reduce_max_sync(0xffffffffu, best_key);
-    const int best = 255 - (best_key & 255);
-    const int n_acc = (best_key >> 8) + 1;
+    const int best = 1023 - (best_key & 1023);
+    const int n_acc = (best_key >> 10) + 1;
     if (err == kOk && (long long)P + n_acc > S_max) err = kErrCapacity;
     const int n_out = (err == kOk) ? n_acc : 0;
 
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < nw; ++k) {
         const int i = lane + 32 * k;
         if (i < T && i >= n_out) path[i] = -1;
     }

@@ -19,7 +19,7 @@ using ppd::AcceptArgs;
 using ppd::AttnMaps;
 using ppd::AttnParams;
 
-constexpr int kMaxT = 128;
+constexpr int kMaxT = ppd::kMaxTree;   // tree tokens per sequence
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
@@ -175,7 +175,11 @@ ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, cons
     p.T = T;
     p.T_pad = T_pad;
     p.S_max = S_max;
-    p.n_units = (int)lbh;
+    // trees of more than 64 tokens: slices split into blocks of 128 query rows,
+    // the tree keys into tiles of 128
+    p.n_qb = T_pad > 64 ? (T + 127) / 128 : 1;
+    p.n_tt = T_pad > 64 ? (T + 127) / 128 : 1;
+    p.n_units = (int)lbh * p.n_qb;
     const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
     p.scale_log2 = sc * 1.4426950408889634f;
     p.fused = fused != nullptr;
@@ -525,7 +529,7 @@ ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32
     if (!logits || !parent || !cand_tokens || !path || !accept_len || !next_token || !tmpl_parent ||
         !tmpl_rank || !next_parent || !next_cand || !next_state || !dev_status || !workspace)
         return PPD_ERR_INVALID_ARG;
-    if (B < 1 || T < 1 || T > kMaxT || V < 1 || n_states < 1 || n_states > kMaxT || T_next < 1 ||
+    if (B < 1 || T < 1 || T > kMaxT || V < 1 || n_states < 1 || n_states > 128 || T_next < 1 ||
         T_next > kMaxT || K < 1 || K > V)
         return PPD_ERR_INVALID_ARG;
     if (K > ppd::kNextMaxK) return PPD_ERR_UNSUPPORTED;

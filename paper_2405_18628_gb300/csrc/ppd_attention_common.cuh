@@ -16,17 +16,21 @@ namespace ppd {
 // A (layer, sequence, head) unit: its sequence, clamped prefix length and tiles
 // (prefix tiles of 128 keys, then one tile of the tree's own keys).
 struct UnitInfo {
-    int b, P, P_raw, n_pref, n_tiles;
+    int lbh, qb, b, P, P_raw, n_pref, n_tiles;
 };
 
+// Unit u = (layer, sequence, head) slice lbh and block qb of its query rows
+// (slices of trees over 128 tokens split their queries into blocks of 128).
 PPD_DEV UnitInfo unit_info(const AttnParams &p, int u)
 {
     UnitInfo ui;
-    ui.b = (u / p.H) % p.B;
+    ui.lbh = u / p.n_qb;
+    ui.qb = u - ui.lbh * p.n_qb;
+    ui.b = (ui.lbh / p.H) % p.B;
     ui.P_raw = __ldg(p.prefix_len + ui.b);
     ui.P = min(max(ui.P_raw, 0), p.S_max);
     ui.n_pref = (ui.P + 127) >> 7;
-    ui.n_tiles = ui.n_pref + 1;
+    ui.n_tiles = ui.n_pref + p.n_tt;
     return ui;
 }
 
@@ -69,16 +73,16 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
     const FusedStep &f = p.fs;
     const int T = p.T, B = p.B, S = f.splits;
     int *s_par = f.scratch + (size_t)blockIdx.x * kSideScratchInts;
-    int *top = s_par + 128;
-    int *path = top + 128;
-    float *s_lse = reinterpret_cast<float *>(path + 128);
-    float *s_ent = s_lse + 128;
+    int *top = s_par + kAcceptScratchInts;
+    int *path = top + kMaxTree;
+    float *s_lse = reinterpret_cast<float *>(path + kMaxTree);
+    float *s_ent = s_lse + kMaxTree;
     const int chunks = f.row_bytes >> 4;
     for (int b = 0; b < B; ++b) {
         const bool designated = (b % (int)gridDim.x) == (int)blockIdx.x;
         bool has_unit = false;
         for (int u = blockIdx.x; u < p.n_units && !has_unit; u += gridDim.x)
-            has_unit = ((u / p.H) % B) == b;
+            has_unit = ((u / p.n_qb / p.H) % B) == b && u % p.n_qb == 0;
         if (!designated && !has_unit) continue;
         for (int r = lane; r < T; r += 32) {
             const size_t base = ((size_t)b * T + r) * S;
@@ -114,13 +118,15 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
             // cache rows [P_b, P_b + n_acc) <- the accepted tree rows
             const int P = __ldg(p.prefix_len + b);
             const int n = res.n_acc;
+            // each slice once: by the CTA holding its first query block
             for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
-                if (((u / p.H) % B) != b) continue;
+                const int lbh = u / p.n_qb;
+                if (u % p.n_qb != 0 || ((lbh / p.H) % B) != b) continue;
                 for (int w = lane; w < n * chunks; w += 32) {
                     const int j = w / chunks, c = w - j * chunks;
                     const int src = path[j];
-                    const size_t so = ((size_t)u * T + src) * f.row_bytes + (size_t)c * 16;
-                    const size_t dof = ((size_t)u * p.S_max + P + j) * f.row_bytes + (size_t)c * 16;
+                    const size_t so = ((size_t)lbh * T + src) * f.row_bytes + (size_t)c * 16;
+                    const size_t dof = ((size_t)lbh * p.S_max + P + j) * f.row_bytes + (size_t)c * 16;
                     const uint4 kx = __ldg(reinterpret_cast<const uint4 *>(f.k_tree + so));
                     const uint4 vx = __ldg(reinterpret_cast<const uint4 *>(f.v_tree + so));
                     *reinterpret_cast<uint4 *>(f.k_cache + dof) = kx;

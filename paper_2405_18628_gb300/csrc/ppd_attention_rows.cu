@@ -1,10 +1,12 @@
 // ppd_attention_rows.cu -- tree-masked attention of the PPD verification step
-// for trees of 65..128 tokens on sm_103a (paper Section 3 step (1): tree
+// for trees of 65..512 tokens on sm_103a (paper Section 3 step (1): tree
 // attention over the candidate tree; Section 4.1: every tree token attends to
 // the cached prefix, its tree ancestors and itself).
 //
 // With more than 64 tree tokens the queries fill the tensor core's M side, so
-// this kernel keeps one query per TMEM lane (queries zero-padded to 128):
+// this kernel keeps one query per TMEM lane (queries zero-padded to 128).  A
+// unit is a (layer, sequence, head) slice and a block of 128 of its query rows;
+// its tiles are the KV prefix and then the tree's keys, 128 per tile:
 //
 //   S  = Q * K_tile^T          tcgen05.mma, M = 128 queries, N = 128 keys, K = D
 //   P  = exp2(S*scale*log2e - m)   two softmax warps per 32 query rows, each
@@ -150,12 +152,13 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 #pragma unroll
                         for (int c = 0; c < Lay::DCH; ++c)
                             tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::GROUP_BYTES,
-                                        &map_q, bars + Lay::B_QFULL + qs, c * 64, 0, u, pol);
+                                        &map_q, bars + Lay::B_QFULL + qs, c * 64, ui.qb * Lay::M,
+                                        ui.lbh, pol);
                     }
                 }
                 for (int j = 0; j < ui.n_tiles; ++j, ++g) {
-                    const bool tree = (j == ui.n_pref);
-                    const int row = tree ? 0 : j * Lay::KT;
+                    const bool tree = (j >= ui.n_pref);
+                    const int row = (tree ? j - ui.n_pref : j) * Lay::KT;
                     if (kq) {
                         const int ks = g % Lay::KS;
                         if (g >= Lay::KS)
@@ -166,7 +169,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                             for (int c = 0; c < Lay::DCH; ++c)
                                 tma_load_3d(smem + Lay::OFF_K + ks * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
                                             tree ? &map_kt : &map_kc, bars + Lay::B_KFULL + ks, c * 64,
-                                            row, u, pol);
+                                            row, ui.lbh, pol);
                         }
                     } else {
                         const int vs = g % Lay::VS;
@@ -178,7 +181,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                             for (int c = 0; c < Lay::DCH; ++c)
                                 tma_load_3d(smem + Lay::OFF_V + vs * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
                                             tree ? &map_vt : &map_vc, bars + Lay::B_VFULL + vs, c * 64,
-                                            row, u, pol);
+                                            row, ui.lbh, pol);
                         }
                     }
                 }
@@ -292,11 +295,14 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
         float m = -INFINITY;    // running maximum of the row (log2 units), same in both threads
         float l = 0.f;          // this thread's share of the row sum
-        uint64_t abits = 0;     // bit i: tree node 64h + i is an ancestor of (or is) node q
-        int cur_b = -1;
+        // anc[t] bit i: tree node 128t + 64h + i is an ancestor of (or is) this
+        // thread's query; tmask: the word of the current tree tile
+        uint64_t anc[kMaxTree / 128] = {};
+        uint64_t tmask = 0;
+        int cur_key = -1;
         int g = 0;
         bool pend = false;      // a finished unit whose output still sits in TMEM
-        int pend_u = 0, pend_g = 0;
+        int pend_lbh = 0, pend_qb = 0, pend_g = 0;
         float pend_linv = 0.f;
 
         // Probabilities of this thread's 64 keys from its raw scores s against the
@@ -320,7 +326,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                         const int i = 32 * c + e + x;          // key 64h + i of the tile
                         float d = fmaf(__uint_as_float(s[i >> 4][i & 15]), sl2, -mx);
                         if (KIND == kMaskRows) d = (64 * h + i < n_valid) ? d : -INFINITY;
-                        if (KIND == kMaskTree) d = ((abits >> i) & 1ull) ? d : -INFINITY;
+                        if (KIND == kMaskTree) d = ((tmask >> i) & 1ull) ? d : -INFINITY;
                         md2[x] = fmaxf(md2[x], d);
                         pv[x] = ex2(fminf(d, 64.f));
                         lt4[(e >> 1) & 3] += pv[x];
@@ -347,7 +353,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 const float v = __uint_as_float(s[i >> 4][i & 15]) * sl2;
                 bool vis = true;
                 if (KIND == kMaskRows) vis = 64 * h + i < n_valid;
-                if (KIND == kMaskTree) vis = ((abits >> i) & 1ull) != 0;
+                if (KIND == kMaskTree) vis = ((tmask >> i) & 1ull) != 0;
                 mx[i & 3] = fmaxf(mx[i & 3], vis ? v : -INFINITY);
             }
             return fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
@@ -355,17 +361,18 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
         // Output of a finished unit: this thread's half of the row of O times 1 / l;
         // then O is free for the next unit's first PV product.
-        auto read_back = [&](int u_out, int g_last, float linv) {
+        auto read_back = [&](int lbh_out, int qb_out, int g_last, float linv) {
             mbar_wait(bars + Lay::B_PDONE + g_last % Lay::NSB, (g_last / Lay::NSB) & 1, abort_flag);
             tc_fence_after();
             const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)h * (D / 2);
-            float *orow = p.out + ((size_t)u_out * T + q) * D + h * (D / 2);
+            const int qg = qb_out * Lay::M + q;
+            float *orow = p.out + ((size_t)lbh_out * T + qg) * D + h * (D / 2);
 #pragma unroll
             for (int ch = 0; ch < D / 32; ++ch) {
                 uint32_t r[16];
                 tmem_ld16(t_o + ch * 16, r);
                 tmem_wait_ld();
-                if (q < T) {
+                if (qg < T) {
                     if (vec_out) {
 #pragma unroll
                         for (int e = 0; e < 16; e += 4)
@@ -387,14 +394,20 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
         int k = 0;
         for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
             const UnitInfo ui = unit_info(p, u);
-            if (ui.b != cur_b) {
-                // ancestors of node q among tree nodes [64h, 64h + 64)
-                abits = 0;
-                if (q < T) {
+            const int qg = ui.qb * Lay::M + q;   // this thread's tree token
+            if (ui.b * p.n_qb + ui.qb != cur_key) {
+                // ancestors of node qg among tree nodes 128t + [64h, 64h + 64)
+#pragma unroll
+                for (int t = 0; t < kMaxTree / 128; ++t) anc[t] = 0;
+                if (qg < T) {
                     bool bad = false;
-                    int a = q;
+                    int a = qg;
                     while (true) {
-                        if ((a >> 6) == h) abits |= 1ull << (a & 63);
+                        if (((a >> 6) & 1) == h) {
+#pragma unroll
+                            for (int t = 0; t < kMaxTree / 128; ++t)
+                                if ((a >> 7) == t) anc[t] |= 1ull << (a & 63);
+                        }
                         const int pa = __ldg(p.parent + (size_t)ui.b * T + a);
                         if (a == 0) {
                             bad = (pa != -1);
@@ -408,14 +421,19 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                     }
                     if (bad && h == 0 && p.dev_status) p.dev_status[ui.b] = kErrTree;
                 }
-                if (q == 0 && h == 0 && p.dev_status && (ui.P_raw < 0 || ui.P_raw > p.S_max))
+                if (qg == 0 && h == 0 && p.dev_status && (ui.P_raw < 0 || ui.P_raw > p.S_max))
                     p.dev_status[ui.b] = kErrCapacity;
-                cur_b = ui.b;
+                cur_key = ui.b * p.n_qb + ui.qb;
             }
 
             for (int j = 0; j < ui.n_tiles; ++j, ++g) {
-                const bool tree = (j == ui.n_pref);
+                const bool tree = (j >= ui.n_pref);
                 const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
+                if (tree) {
+#pragma unroll
+                    for (int t = 0; t < kMaxTree / 128; ++t)
+                        if (j - ui.n_pref == t) tmask = anc[t];
+                }
                 const int kind = tree ? kMaskTree : (n_valid < Lay::KT ? kMaskRows : kMaskNone);
                 const int sb = g % Lay::NSB;
                 mbar_wait(bars + Lay::B_SFULL + sb, (g / Lay::NSB) & 1, abort_flag);
@@ -497,7 +515,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
                 // the previous unit's output, once this unit's first tile is on its way
                 if (j == 0 && pend) {
-                    read_back(pend_u, pend_g, pend_linv);
+                    read_back(pend_lbh, pend_qb, pend_g, pend_linv);
                     pend = false;
                 }
 
@@ -506,10 +524,11 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                     xl[h * Lay::M + q] = l;
                     named_bar_sync(1, 256);
                     const float L = xl[q] + xl[Lay::M + q];
-                    if (h == 0 && q < T && p.lse)
-                        p.lse[(size_t)u * T + q] = (m + lg2(L)) * 0.69314718055994530942f;
+                    if (h == 0 && qg < T && p.lse)
+                        p.lse[(size_t)ui.lbh * T + qg] = (m + lg2(L)) * 0.69314718055994530942f;
                     pend = true;
-                    pend_u = u;
+                    pend_lbh = ui.lbh;
+                    pend_qb = ui.qb;
                     pend_g = g;
                     pend_linv = rcp(L);
                     m = -INFINITY;
@@ -517,7 +536,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 }
             }
         }
-        if (pend) read_back(pend_u, pend_g, pend_linv);
+        if (pend) read_back(pend_lbh, pend_qb, pend_g, pend_linv);
     }
 
     tc_fence_before();

@@ -42,9 +42,14 @@ struct FusedStep {
     float inv_temp, epsilon, delta;
 };
 
-// Per-CTA scratch of the fused step's side warp: parent copy, top-1 tokens,
-// path, and (typical acceptance) each node's log-sum-exp and entropy.
-constexpr int kSideScratchInts = 5 * 128 + 8;
+// Largest tree (nodes) of the verification step, and the per-warp scratch
+// that acceptance needs: parents, then one 32-bit word per 32 nodes of pass bits.
+constexpr int kMaxTree = 512;
+constexpr int kAcceptScratchInts = kMaxTree + kMaxTree / 32;
+
+// Per-CTA scratch of the fused step's side warp: acceptance scratch, top-1
+// tokens, path, and (typical acceptance) each node's log-sum-exp and entropy.
+constexpr int kSideScratchInts = kAcceptScratchInts + 4 * kMaxTree + 8;
 
 struct AttnParams {
     const int32_t *prefix_len;  // [B]
@@ -53,6 +58,8 @@ struct AttnParams {
     float *lse;                 // [L,B,H,T] or null
     int32_t *dev_status;        // [B] or null (main-loop errors; null in the fused step)
     int L, B, H, T, T_pad, S_max, n_units;
+    int n_qb;                   // query blocks of 128 per (layer, sequence, head) slice
+    int n_tt;                   // tree-key tiles of 128 per slice
     float scale_log2;           // softmax scale * log2(e)
     int fused;                  // run the end phase below
     FusedStep fs;

@@ -172,7 +172,7 @@ cudaError_t launch_argmax_combine(const float *part_val, const int32_t *part_idx
 __global__ void __launch_bounds__(128)
 accept_path_kernel(const int32_t *argmax, AcceptArgs a, int B)
 {
-    __shared__ int s_par[4][128];
+    __shared__ int s_par[4][kAcceptScratchInts];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.x * 4 + warp;
     if (b >= B) return;
@@ -224,7 +224,7 @@ typical_accept_kernel(const float *logits, const float *lse, const float *ent,
                       const int32_t *argmax, AcceptArgs a, int B, float inv_temp, float epsilon,
                       float delta)
 {
-    __shared__ int s_par[4][128];
+    __shared__ int s_par[4][kAcceptScratchInts];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.x * 4 + warp;
     if (b >= B) return;

@@ -59,8 +59,8 @@ def test_host_argument_checks(lib):
     null = None
     s = vp(0)
     INVALID = 1
-    # T > 128
-    assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 129, 64, 200,
+    # T > 512
+    assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 513, 64, 200,
                                   0, 0.0, fake, null, fake, null, 0, s) == INVALID
     # D not in {64, 128}
     assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 8, 96, 200,
@@ -76,7 +76,7 @@ def test_host_argument_checks(lib):
                                   1, 0.0, fake, null, fake, null, 0, s) == INVALID
     assert lib.ppd_node_argmax(fake, 0, 4, 10, fake, null, 0, s) == INVALID
     assert lib.ppd_node_argmax(fake, 1, 64, 32000, fake, null, 0, s) == INVALID   # needs workspace
-    assert lib.ppd_accept_path(fake, fake, fake, fake, 1, 200, 10, 10, fake, fake, fake, fake,
+    assert lib.ppd_accept_path(fake, fake, fake, fake, 1, 600, 10, 10, fake, fake, fake, fake,
                                fake, s) == INVALID
     assert lib.ppd_accept_path(fake, fake, null, fake, 1, 4, 10, 10, fake, fake, fake, fake,
                                fake, s) == INVALID

@@ -155,6 +155,33 @@ def test_attention_rows_head_dim_64(cuda_device, T, P):
                                atol=1e-3)
 
 
+@pytest.mark.parametrize("T,P,D", [(200, 700, 128), (285, 300, 128), (512, 130, 128),
+                                   (129, 0, 64), (300, 256, 64)])
+def test_attention_trees_over_128_tokens(cuda_device, T, P, D):
+    """Trees above 128 tokens (the paper's MobileLlama trees reach 285): query
+    rows in blocks of 128, tree keys in tiles of 128, masks from 512-bit
+    ancestor sets."""
+    rng = np.random.default_rng(T * 31 + P + D)
+    B, H = 2, 2
+    parent = np.full((B, T), -1, np.int32)
+    for b in range(B):
+        for i in range(1, T):
+            # long chains mixed with branching: ancestors across every tree tile
+            parent[b, i] = i - 1 if (b == 0 and i % 5) else rng.integers(max(0, i - 150), i)
+    w = W.Workload("big", L=1, B=B, H=H, D=D, P=P, T=T, V=16, n_cand=T, max_depth=T,
+                   chains="every0", match_rate=0.5, seed=T + P + D)
+    pl = np.array([P, max(P - 77, 0)], np.int32)
+    t = tensors(w, prefix_len=pl)
+    out, lse, st = run_attention({k: v.to(cuda_device) for k, v in t.items()}, pl, parent,
+                                 cuda_device)
+    ref, ref_lse, _, ref_st = oracle.tree_attention(t["q"], t["k_cache"], t["v_cache"], t["k_tree"],
+                                                    t["v_tree"], pl, parent)
+    assert (st.cpu().numpy() == 0).all() and (ref_st == 0).all()
+    assert_attn_close(out.cpu().numpy().reshape(ref.shape), ref, f"T={T} P={P} D={D}")
+    np.testing.assert_allclose(lse.cpu().numpy().reshape(ref_lse.shape), ref_lse, rtol=0,
+                               atol=1e-3)
+
+
 def test_attention_peaked_scores_and_scale(cuda_device):
     """Large scores force the running-max rescale path on later tiles."""
     w = W.scaled(W.WORKLOADS["vicuna7b"], L=1, H=2, P=1000)
@@ -307,7 +334,9 @@ def _verify_step(w, s, t, dev, units=None):
 
 @pytest.mark.parametrize("name,overrides", [("tiny", {}), ("tiny", {"B": 4}),
                                             ("mobilellama", {"L": 2, "H": 4}),
-                                            ("vicuna7b", {"L": 1, "H": 2, "B": 2})])
+                                            ("vicuna7b", {"L": 1, "H": 2, "B": 2}),
+                                            ("mobilellama", {"L": 1, "H": 2, "B": 2, "T": 285,
+                                                             "n_cand": 72})])
 def test_verify_step_matches_oracle(cuda_device, name, overrides):
     w = W.scaled(W.WORKLOADS[name], **overrides)
     s = W.make_step_inputs(w)
