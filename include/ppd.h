@@ -216,14 +216,21 @@ ppd_status ppd_verify_step_typical(const void *q, void *k_cache, void *v_cache,
 
 /*
  * Next-step candidate tree (Section 3 step (1): the prompt tokens appended to a
- * guess token predict the tokens after it; Appendix, Definition of tree states:
- * the tree takes state T_k, whose candidate subtree is at most k deep, k being
- * the number of prompt tokens available below the accepted token).
- *   e = path[b][accept_len[b]-1], the accepted end node of sequence b.  Its
- *   prompt chain: c_1 = the lowest-index child of e with cand_tokens -1, c_(j+1)
- *   the lowest-index such child of c_j; k = the chain length, capped at
- *   n_states - 1.  The K best tokens of the logits at c_d (ranking: NaN first,
- *   then larger value, then lower index) are the guesses for depth d.
+ * guess token predict the tokens after it; Section 3, Ensemble Prompt Tokens:
+ * each prompt position holds n_ept tokens, the j-th attending only to the j-th
+ * of the earlier positions, and the guess comes from the average of their
+ * logits; Appendix, Definition of tree states: the tree takes state T_k, whose
+ * candidate subtree is at most k deep, k being the number of prompt positions
+ * available below the accepted token).
+ *   e = path[b][accept_len[b]-1], the accepted end node of sequence b.  The
+ *   first n_ept children of e with cand_tokens -1 (index order) head n_ept
+ *   prompt chains, each continued by the lowest-index such child of its last
+ *   node; k = the shortest chain's length (0 when e has fewer than n_ept
+ *   prompt children), capped at n_states - 1.  The guesses for depth d are
+ *   the K best tokens (ranking: NaN first, then larger value, then lower index)
+ *   of the fp32 average of the chains' logits at position d: summed in chain
+ *   order, then divided by n_ept with IEEE rounding.  n_ept = 1: one chain,
+ *   plain logits.
  *   tmpl_parent, tmpl_rank int32 [n_states][T_next] (device): the next tree of
  *   each state; node 0 is the root (parent -1), rank r >= 0 marks a candidate
  *   taking guess r at its depth, -1 a prompt node.
@@ -234,15 +241,17 @@ ppd_status ppd_verify_step_typical(const void *q, void *k_cache, void *v_cache,
  * next_token[b] < 0, or template k is not a tree in topological order, has a
  * candidate below a prompt node, a candidate deeper than k or a rank >= K.
  * logits, parent, cand_tokens, path as for the verification step that just ran.
- * 1 <= K <= 16, K <= V; n_states <= 128; T_next <= 512.  Workspace:
+ * 1 <= K <= 16, K <= V; 1 <= n_ept <= 128; n_states <= 128; T_next <= 512.
+ * Workspace:
  * ppd_next_tree_workspace_bytes(B, n_states, K) bytes.
  */
 size_t ppd_next_tree_workspace_bytes(int B, int n_states, int K);
 ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32_t *cand_tokens,
                          const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
                          int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
-                         const int32_t *tmpl_rank, int K, int32_t *next_parent, int32_t *next_cand,
-                         int32_t *next_state, int32_t *dev_status, void *workspace, size_t ws_bytes,
+                         const int32_t *tmpl_rank, int K, int n_ept, int32_t *next_parent,
+                         int32_t *next_cand, int32_t *next_state, int32_t *dev_status,
+                         void *workspace, size_t ws_bytes,
                          void *stream);
 
 /*

@@ -80,7 +80,8 @@ def _load():
         lib.oracle_topk.argtypes = [vp, c_i64, c_i64, c_int, i32p]
         lib.oracle_topk.restype = None
         lib.oracle_next_tree.argtypes = [vp, i32p, i32p, i32p, i32p, i32p, c_int, c_int, c_int,
-                                         c_int, c_int, i32p, i32p, c_int, i32p, i32p, i32p, i32p]
+                                         c_int, c_int, i32p, i32p, c_int, c_int, i32p, i32p, i32p,
+                                         i32p]
         lib.oracle_next_tree.restype = c_int
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = c_int
@@ -257,11 +258,11 @@ def topk(logits, K: int) -> np.ndarray:
 
 
 def next_tree(logits, parent, cand_tokens, path, accept_len, next_token, tmpl_parent, tmpl_rank,
-              K: int):
+              K: int, n_ept: int = 1):
     """Next-step candidate tree.  logits [B,T,V]; parent, cand_tokens, path
     [B,T]; accept_len, next_token [B]; tmpl_parent, tmpl_rank [n_states,
-    T_next].  Returns dict of next_parent, next_cand [B,T_next], next_state,
-    status [B]."""
+    T_next]; n_ept ensemble prompt tokens per position.  Returns dict of
+    next_parent, next_cand [B,T_next], next_state, status [B]."""
     lg, _ = _host(logits)
     lg = np.ascontiguousarray(lg, dtype=np.float32)
     par, cd, pth, al, nt = (_i32(x) for x in (parent, cand_tokens, path, accept_len, next_token))
@@ -273,7 +274,7 @@ def next_tree(logits, parent, cand_tokens, path, accept_len, next_token, tmpl_pa
            "next_state": np.empty(B, np.int32), "status": np.empty(B, np.int32)}
     p = lambda a: _ptr(a, ctypes.c_int32)
     rc = _load().oracle_next_tree(_ptr(lg), p(par), p(cd), p(pth), p(al), p(nt), B, T, V, n_states,
-                                  T_next, p(tp), p(tr), int(K), p(res["next_parent"]),
+                                  T_next, p(tp), p(tr), int(K), int(n_ept), p(res["next_parent"]),
                                   p(res["next_cand"]), p(res["next_state"]), p(res["status"]))
     if rc != 0:
         raise ValueError(f"oracle_next_tree rejected its arguments (code {rc})")

@@ -505,11 +505,17 @@ void oracle_topk(const float *logits, int64_t rows, int64_t V, int K, int32_t *o
  * Definition of tree states: a tree exists in states T_k whose candidate
  * subtree has depth at most k, k being set by the prompt tokens available).
  *
- * e = path[b][accept_len[b] - 1] is the accepted end node.  Its prompt chain:
- * c_1 = the lowest-index child of e with cand_tokens -1, c_(j+1) the
- * lowest-index such child of c_j; k = the chain length, capped at n_states-1.
- * The K best tokens (oracle_topk order) of the logits at c_d are the guesses
- * for depth d of the next tree.  Template state k: tmpl_parent[k][i] (node 0
+ * e = path[b][accept_len[b] - 1] is the accepted end node.  With n_ept
+ * ensemble prompt tokens (Section 3, "Ensemble Prompt Tokens": every prompt
+ * token position holds n_ept tokens, each seeing only its own chain, and the
+ * guess comes from the average of their logits): the first n_ept children of
+ * e with cand_tokens -1, in index order, head n_ept chains, each continued by
+ * the lowest-index such child of its last node; k = the shortest chain's
+ * length (0 if e has fewer than n_ept prompt children), capped at
+ * n_states - 1.  The logits for depth d are those of the chains' nodes at
+ * position d averaged in fp32 -- summed in chain order, then divided by
+ * n_ept -- and their K best tokens (oracle_topk order) are the guesses for
+ * depth d of the next tree.  n_ept = 1 is a single chain and plain logits.  Template state k: tmpl_parent[k][i] (node 0
  * the root, parent -1) and tmpl_rank[k][i] (rank r >= 0: a candidate node, -1:
  * a prompt node; ignored for the root).  Outputs: next_parent[b] =
  * tmpl_parent[k]; next_cand[b][0] = next_token[b]; a candidate node at
@@ -522,14 +528,15 @@ void oracle_topk(const float *logits, int64_t rows, int64_t V, int K, int32_t *o
 int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *cand,
                      const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
                      int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
-                     const int32_t *tmpl_rank, int K, int32_t *next_parent, int32_t *next_cand,
-                     int32_t *next_state, int32_t *status)
+                     const int32_t *tmpl_rank, int K, int n_ept, int32_t *next_parent,
+                     int32_t *next_cand, int32_t *next_state, int32_t *status)
 {
-    if (B < 1 || T < 1 || V < 1 || n_states < 1 || T_next < 1 || K < 1 || K > V)
+    if (B < 1 || T < 1 || V < 1 || n_states < 1 || T_next < 1 || K < 1 || K > V || n_ept < 1)
         return ORC_ERR_INVALID_ARG;
     int32_t *top = (int32_t *)malloc(sizeof(int32_t) * (size_t)K);
     int *cdepth = (int *)malloc(sizeof(int) * (size_t)T_next);
-    int *chain = (int *)malloc(sizeof(int) * (size_t)(T + 1));
+    int *chain = (int *)malloc(sizeof(int) * (size_t)(T + 1) * (size_t)n_ept);
+    float *avg = (float *)malloc(sizeof(float) * (size_t)V);
     for (int b = 0; b < B; ++b) {
         const int32_t *par = parent + (int64_t)b * T;
         const int32_t *tok = cand + (int64_t)b * T;
@@ -541,19 +548,33 @@ int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *
             err = ORC_ERR_TREE;
         if (err == ORC_OK) {
             int e = path[(int64_t)b * T + n - 1];
-            /* the prompt chain below the end node */
-            int cur = e;
-            while (1) {
-                int nxt = -1;
-                for (int i = cur + 1; i < T; ++i)
-                    if (par[i] == cur && tok[i] == -1) {
-                        nxt = i;
-                        break;
+            /* the n_ept prompt chains below the end node: chain[j * (T + 1) + d] */
+            int heads = 0;
+            for (int i = e + 1; i < T && heads < n_ept; ++i)
+                if (par[i] == e && tok[i] == -1)
+                    chain[(int64_t)(heads++) * (T + 1)] = i;
+            if (heads < n_ept) {
+                k = 0;
+            } else {
+                k = T;
+                for (int j = 0; j < n_ept; ++j) {
+                    int *cj = chain + (int64_t)j * (T + 1);
+                    int len = 1, cur = cj[0];
+                    while (1) {
+                        int nxt = -1;
+                        for (int i = cur + 1; i < T; ++i)
+                            if (par[i] == cur && tok[i] == -1) {
+                                nxt = i;
+                                break;
+                            }
+                        if (nxt < 0)
+                            break;
+                        cj[len++] = nxt;
+                        cur = nxt;
                     }
-                if (nxt < 0)
-                    break;
-                chain[k++] = nxt;
-                cur = nxt;
+                    if (len < k)
+                        k = len;
+                }
             }
             if (k > n_states - 1)
                 k = n_states - 1;
@@ -581,7 +602,13 @@ int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *
                 }
                 nc[0] = next_token[b];
                 for (int d = 1; d <= k; ++d) {
-                    oracle_topk(logits + ((int64_t)b * T + chain[d - 1]) * V, 1, V, K, top);
+                    for (int64_t v = 0; v < V; ++v) {
+                        float sum = logits[((int64_t)b * T + chain[d - 1]) * V + v];
+                        for (int j = 1; j < n_ept; ++j)
+                            sum += logits[((int64_t)b * T + chain[(int64_t)j * (T + 1) + d - 1]) * V + v];
+                        avg[v] = sum / (float)n_ept;
+                    }
+                    oracle_topk(avg, 1, V, K, top);
                     for (int i = 1; i < T_next; ++i)
                         if (tr[i] >= 0 && cdepth[i] == d)
                             nc[i] = top[tr[i]];
@@ -601,6 +628,7 @@ int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *
     free(top);
     free(cdepth);
     free(chain);
+    free(avg);
     return ORC_OK;
 }
 

@@ -1,15 +1,19 @@
 // ppd_next.cu -- next-step candidate tree of the PPD decode loop (paper
 // Section 3 step (1): the prompt tokens appended to a guess token predict the
-// tokens that follow it; Appendix, Definition of tree states: the next tree
-// takes state T_k, whose candidate subtree is at most k deep, k being the
-// number of prompt tokens left below the accepted token).
+// tokens that follow it; Section 3, Ensemble Prompt Tokens: each prompt
+// position holds n_ept tokens, the j-th seeing only the j-th of the positions
+// before it, and the guess comes from the average of their logits; Appendix,
+// Definition of tree states: the next tree takes state T_k, whose candidate
+// subtree is at most k deep, k being the number of prompt positions left
+// below the accepted token).
 //
-// Kernel 1, one block per (sequence, chain position d): finds the prompt
-// chain below the accepted end node (warp ballots over the parent array) and,
-// if d is within the state, the K best tokens of the chain node's logits --
-// every thread keeps its own top-K over a strided slice of the row, then K
-// rounds of a block-wide best-of-heads merge.  Kernel 2, one warp per
-// sequence: fills the state's template with the root token and the guesses.
+// Kernel 1, one block per (sequence, chain position d): finds the n_ept
+// prompt chains below the accepted end node (warp ballots over the parent
+// array, one warp per chain) and, if d is within the state, the K best tokens
+// of the chains' averaged logits at position d -- every thread keeps its own
+// top-K over a strided slice of the row, then K rounds of a block-wide
+// best-of-heads merge.  Kernel 2, one warp per sequence: fills the state's
+// template with the root token and the guesses.
 #include "ppd.h"
 #include "ppd_accept.cuh"
 #include "ppd_device.cuh"
@@ -19,63 +23,90 @@
 
 namespace ppd {
 
-// The prompt chain below node e of one sequence (lowest-index prompt child at
-// each step), computed by one warp; returns its length (<= cap) and writes the
-// nodes to chain[0..len).
-PPD_DEV int prompt_chain(const int32_t *par, const int32_t *tok, int T, int e, int cap, int lane,
-                         int *chain)
+// The lowest-index child i > cur of node cur with cand -1 (a prompt token), or
+// -1; one warp, the result is warp-uniform.
+PPD_DEV int next_prompt_child(const int32_t *par, const int32_t *tok, int T, int cur, int lane)
 {
-    int len = 0, cur = e;
-    while (len < cap) {
-        int nxt = INT_MAX;
-        for (int i0 = 0; i0 < T; i0 += 32) {
-            const int i = i0 + lane;
-            const bool hit = i < T && i > cur && __ldg(par + i) == cur && __ldg(tok + i) == -1;
-            const unsigned m = __ballot_sync(0xffffffffu, hit);
-            if (m) {
-                nxt = i0 + __ffs(m) - 1;
-                break;
-            }
-        }
-        if (nxt == INT_MAX) break;
-        if (lane == 0) chain[len] = nxt;
-        ++len;
-        cur = nxt;
+    for (int i0 = (cur + 1) & ~31; i0 < T; i0 += 32) {
+        const int i = i0 + lane;
+        const bool hit = i < T && i > cur && __ldg(par + i) == cur && __ldg(tok + i) == -1;
+        const unsigned m = __ballot_sync(0xffffffffu, hit);
+        if (m) return i0 + __ffs(m) - 1;
     }
-    __syncwarp();
-    return len;
+    return -1;
 }
 
-// Top-K (K <= kNextMaxK) of the logits of chain node d (1-based) of sequence
-// b, written to topk[(b * (n_states - 1) + d - 1) * K ...] in ranking order
-// (NaN first, then larger value, then lower index).
+// Top-K (K <= kNextMaxK) of the averaged logits at chain position d (1-based)
+// of sequence b, written to topk[(b * (n_states - 1) + d - 1) * K ...] in
+// ranking order (NaN first, then larger value, then lower index).  The blocks
+// of position 1 also write the state k of their sequence to kstate[b].
 __global__ void __launch_bounds__(256)
 next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const int32_t *cand,
                  const int32_t *path, const int32_t *accept_len, int T, int V, int n_states, int K,
-                 int32_t *topk)
+                 int n_ept, int32_t *topk, int32_t *kstate)
 {
-    __shared__ int s_chain[128];
-    __shared__ int s_len;
+    __shared__ int s_head[kNextMaxEpt];
+    __shared__ int s_len[kNextMaxEpt];
+    __shared__ int s_node[kNextMaxEpt];
+    __shared__ int s_nh, s_k;
     __shared__ float s_v[8];
     __shared__ int s_i[8], s_t[8];
     __shared__ int s_win;
     const int b = blockIdx.x;
     const int d = blockIdx.y + 1;
+    const int cap = n_states - 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n = __ldg(accept_len + b);
+    const int32_t *par = parent + (size_t)b * T;
+    const int32_t *tok = cand + (size_t)b * T;
+    // the chain heads: the first n_ept prompt children of the end node
     if (warp == 0) {
-        int len = 0;
-        if (n >= 1 && n <= T) {
-            const int e = __ldg(path + (size_t)b * T + n - 1);
-            if (e >= 0 && e < T)
-                len = prompt_chain(parent + (size_t)b * T, cand + (size_t)b * T, T, e, n_states - 1,
-                                   lane, s_chain);
+        int cnt = 0;
+        const int n = __ldg(accept_len + b);
+        const int e = (n >= 1 && n <= T) ? __ldg(path + (size_t)b * T + n - 1) : -1;
+        if (e >= 0 && e < T) {
+            for (int i0 = (e + 1) & ~31; i0 < T && cnt < n_ept; i0 += 32) {
+                const int i = i0 + lane;
+                const bool hit = i < T && i > e && __ldg(par + i) == e && __ldg(tok + i) == -1;
+                const unsigned m = __ballot_sync(0xffffffffu, hit);
+                const int pos = cnt + __popc(m & ((1u << lane) - 1u));
+                if (hit && pos < n_ept) s_head[pos] = i;
+                cnt += __popc(m);
+            }
         }
-        if (lane == 0) s_len = len;
+        if (lane == 0) s_nh = min(cnt, n_ept);
     }
     __syncthreads();
-    if (d > s_len) return;   // uniform over the block
-    const float *x = logits + ((size_t)b * T + s_chain[d - 1]) * V;
+    // each chain's length (capped) and its node at position d, one warp a chain
+    if (s_nh == n_ept) {
+        for (int j = warp; j < n_ept; j += 8) {
+            int cur = s_head[j], len = 1, node = d == 1 ? cur : -1;
+            while (len < cap) {
+                const int nxt = next_prompt_child(par, tok, T, cur, lane);
+                if (nxt < 0) break;
+                cur = nxt;
+                ++len;
+                if (len == d) node = cur;
+            }
+            if (lane == 0) {
+                s_len[j] = len;
+                s_node[j] = node;
+            }
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int k = 0;
+        if (s_nh == n_ept) {
+            k = cap;
+            for (int j = 0; j < n_ept; ++j) k = min(k, s_len[j]);
+        }
+        s_k = k;
+        if (d == 1) kstate[b] = k;
+    }
+    __syncthreads();
+    if (d > s_k) return;   // uniform over the block
+    const float *x0 = logits + ((size_t)b * T + s_node[0]) * V;
+    const float n_f = (float)n_ept;
 
     // this thread's best K over its slice, best first
     float hv[kNextMaxK];
@@ -88,7 +119,12 @@ next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const 
     float tv = -INFINITY;   // the K-th best so far (the entry a new token must beat)
     int ti = INT_MAX;
     for (int v = threadIdx.x; v < V; v += 256) {
-        const float xv = __ldcs(x + v);
+        float xv = __ldcs(x0 + v);
+        if (n_ept > 1) {
+            // the EPT average: summed in chain order, then one IEEE division
+            for (int j = 1; j < n_ept; ++j) xv += __ldcs(logits + ((size_t)b * T + s_node[j]) * V + v);
+            xv = xv / n_f;
+        }
         if (!ranks_before(xv, v, tv, ti)) continue;
         // insert, shifting worse entries down (slots K.. stay unused)
         float cv = xv;
@@ -162,10 +198,9 @@ __global__ void __launch_bounds__(128)
 next_assemble_kernel(const int32_t *parent, const int32_t *cand, const int32_t *path,
                      const int32_t *accept_len, const int32_t *next_token, int B, int T,
                      int n_states, int T_next, const int32_t *tmpl_parent, const int32_t *tmpl_rank,
-                     int K, const int32_t *topk, int32_t *next_parent, int32_t *next_cand,
-                     int32_t *next_state, int32_t *status)
+                     int K, const int32_t *topk, const int32_t *kstate, int32_t *next_parent,
+                     int32_t *next_cand, int32_t *next_state, int32_t *status)
 {
-    __shared__ int s_chain[4][128];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.x * 4 + warp;
     if (b >= B) return;
@@ -176,9 +211,7 @@ next_assemble_kernel(const int32_t *parent, const int32_t *cand, const int32_t *
     if (!bad) {
         const int e = __ldg(path + (size_t)b * T + n - 1);
         bad = !(e >= 0 && e < T);
-        if (!bad)
-            k = prompt_chain(parent + (size_t)b * T, cand + (size_t)b * T, T, e, n_states - 1, lane,
-                             s_chain[warp]);
+        if (!bad && n_states > 1) k = __ldg(kstate + b);
     }
     const int32_t *tp = tmpl_parent + (size_t)k * T_next;
     const int32_t *tr = tmpl_rank + (size_t)k * T_next;
@@ -240,19 +273,21 @@ cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const i
                              const int32_t *path, const int32_t *accept_len,
                              const int32_t *next_token, int B, int T, int V, int n_states,
                              int T_next, const int32_t *tmpl_parent, const int32_t *tmpl_rank, int K,
-                             int32_t *topk, int32_t *next_parent, int32_t *next_cand,
-                             int32_t *next_state, int32_t *status, cudaStream_t stream)
+                             int n_ept, int32_t *topk, int32_t *kstate, int32_t *next_parent,
+                             int32_t *next_cand, int32_t *next_state, int32_t *status,
+                             cudaStream_t stream)
 {
     if (n_states > 1) {
         next_topk_kernel<<<dim3((unsigned)B, (unsigned)(n_states - 1)), 256, 0, stream>>>(
-            logits, parent, cand, path, accept_len, T, V, n_states, K, topk);
+            logits, parent, cand, path, accept_len, T, V, n_states, K, n_ept, topk, kstate);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
     next_assemble_kernel<<<(B + 3) / 4, 128, 0, stream>>>(parent, cand, path, accept_len, next_token,
                                                           B, T, n_states, T_next, tmpl_parent,
-                                                          tmpl_rank, K, topk, next_parent,
-                                                          next_cand, next_state, status);
+                                                          tmpl_rank, K, topk, kstate,
+                                                          next_parent, next_cand, next_state,
+                                                          status);
     return cudaGetLastError();
 }
 

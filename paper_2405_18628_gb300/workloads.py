@@ -40,7 +40,7 @@ class Workload:
     V: int            # vocab size
     n_cand: int       # candidate nodes including the root
     max_depth: int    # depth cap of candidate nodes (root depth 0)
-    chains: str       # prompt-chain recipe, see _attach_prompt_chains
+    chains: str       # prompt-chain recipe, see _chain_lengths
     match_rate: float
     dtype: str = "bf16"   # storage type of Q/K/V: "bf16" or "f32"
     seed: int = SEED_BASE
@@ -105,6 +105,10 @@ def _chain_lengths(rng, recipe: str, parent, depth, n_prompt: int) -> List[Tuple
     if recipe.startswith("every"):
         c = int(recipe[len("every"):])
         return [(i, c) for i in range(n_cand)]
+    if recipe.startswith("ept"):
+        # "ept<n>x<c>": n ensemble chains of c prompt tokens on every candidate
+        n, c = (int(x) for x in recipe[len("ept"):].split("x"))
+        return [(i, c) for i in range(n_cand) for _ in range(n)]
     if recipe == "fill3":
         # chains of 3 on leaves in index order, then on the deepest internal
         # nodes; the last chain is truncated to hit the total exactly
@@ -140,16 +144,18 @@ def _chain_lengths(rng, recipe: str, parent, depth, n_prompt: int) -> List[Tuple
     raise ValueError(f"unknown chain recipe {recipe!r}")
 
 
-def make_tree_templates(n_states: int, T_next: int, K: int, rng: np.random.Generator):
+def make_tree_templates(n_states: int, T_next: int, K: int, rng: np.random.Generator,
+                        n_ept: int = 1):
     """Next-step tree templates, one per state k = 0..n_states-1 (the paper's
     T_k, Appendix: the candidate subtree of T_k is at most k deep).  Node 0 is
     the root; candidate nodes carry the rank (0..K-1) of the guess they take at
     their depth, prompt nodes rank -1.  Candidates: up to K children of the root
     at depth 1, then at each further depth up to K children of the depth's
     rank-0 node and of one other random candidate, within a budget of
-    T_next // 4 candidates; prompt chains of up to n_states-1 tokens then hang
-    below the root and the candidates, in index order, filling exactly T_next
-    nodes.  Returns (parent, rank), both int32 [n_states, T_next]."""
+    T_next // 4 candidates; n_ept prompt chains of up to n_states-1 tokens each
+    then hang below the root and the candidates, in index order, filling
+    exactly T_next nodes.  Returns (parent, rank), both int32 [n_states,
+    T_next]."""
     m = n_states - 1
     parent = np.full((n_states, T_next), -1, np.int32)
     rank = np.full((n_states, T_next), -1, np.int32)
@@ -175,13 +181,14 @@ def make_tree_templates(n_states: int, T_next: int, K: int, rng: np.random.Gener
             level = nxt
         n_cand = len(par)
         for a in range(n_cand):
-            prev = a
-            for _ in range(m):
-                if len(par) >= T_next:
-                    break
-                par.append(prev)
-                rk.append(-1)
-                prev = len(par) - 1
+            for _ in range(n_ept):
+                prev = a
+                for _ in range(m):
+                    if len(par) >= T_next:
+                        break
+                    par.append(prev)
+                    rk.append(-1)
+                    prev = len(par) - 1
         while len(par) < T_next:                  # more room than chains: extend the root's
             par.append(len(par) - 1 if rk[-1] == -1 else 0)
             rk.append(-1)

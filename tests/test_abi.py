@@ -117,3 +117,29 @@ def test_typical_acceptance_host_checks(lib):
     assert lib.ppd_verify_step_typical(*args) == ppd.PPD_ERR_INVALID_ARG
     assert lib.ppd_node_stats(None, 1, 4, 100, 1.0, fake, fake, fake, fake, ws, s) == \
         ppd.PPD_ERR_INVALID_ARG
+
+
+def test_next_tree_host_checks(lib):
+    """Next-step tree: K in 1..16 and <= V, n_ept in 1..128, n_states <= 128,
+    T and T_next <= 512, enough workspace; refused before any launch."""
+    from paper_2405_18628_gb300 import ppd
+    vp = ctypes.c_void_p
+    fake = vp(0x10000)
+    s = vp(0)
+    ws = 1 << 20
+
+    def call(B=2, T=16, V=100, n_states=4, T_next=32, K=4, n_ept=1, ws_bytes=ws):
+        return lib.ppd_next_tree(*[fake] * 6, B, T, V, n_states, T_next, fake, fake, K, n_ept,
+                                 *[fake] * 4, fake, ws_bytes, s)
+
+    assert call(n_ept=0) == ppd.PPD_ERR_INVALID_ARG
+    assert call(n_ept=129) == ppd.PPD_ERR_UNSUPPORTED
+    assert call(K=17) == ppd.PPD_ERR_UNSUPPORTED
+    assert call(K=0) == ppd.PPD_ERR_INVALID_ARG
+    assert call(K=8, V=7) == ppd.PPD_ERR_INVALID_ARG
+    assert call(n_states=129) == ppd.PPD_ERR_INVALID_ARG
+    assert call(T=513) == ppd.PPD_ERR_INVALID_ARG
+    assert call(T_next=513) == ppd.PPD_ERR_INVALID_ARG
+    need = lib.ppd_next_tree_workspace_bytes(2, 4, 4)
+    assert need >= 2 * 4 * 4 * 4 + 2 * 4
+    assert call(ws_bytes=need - 1) == ppd.PPD_ERR_INVALID_ARG

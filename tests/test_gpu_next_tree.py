@@ -1,8 +1,9 @@
 """Next-step candidate tree on the GPU (through the C ABI) against the oracle,
-bit for bit: the state k picked from the accepted node's prompt chain, the
-top-K guesses per chain position (including ties, NaNs and -inf logits), and
-the assembled parent / candidate arrays; bad templates and failed sequences
-report PPD_ERR_TREE."""
+bit for bit: the state k picked from the accepted node's prompt chains, the
+top-K guesses per chain position (including ties, NaNs and -inf logits) over
+one chain or the fp32 average of n_ept ensemble chains, and the assembled
+parent / candidate arrays; bad templates and failed sequences report
+PPD_ERR_TREE."""
 import numpy as np
 import pytest
 import torch
@@ -16,7 +17,7 @@ from test_gpu_parity import i32
 pytestmark = pytest.mark.gpu
 
 
-def _run(dev, logits, parent, cand, path, accept_len, next_token, tp, tr, K):
+def _run(dev, logits, parent, cand, path, accept_len, next_token, tp, tr, K, n_ept=1):
     B, T = parent.shape
     n_states, T_next = tp.shape
     out = {"next_parent": torch.full((B, T_next), -9, dtype=torch.int32, device=dev),
@@ -26,7 +27,7 @@ def _run(dev, logits, parent, cand, path, accept_len, next_token, tp, tr, K):
     ppd.ppd_next_tree(torch.from_numpy(np.ascontiguousarray(logits)).to(dev), i32(parent, dev),
                       i32(cand, dev), i32(path, dev), i32(accept_len, dev), i32(next_token, dev),
                       i32(tp, dev), i32(tr, dev), K, out["next_parent"], out["next_cand"],
-                      out["next_state"], out["status"])
+                      out["next_state"], out["status"], n_ept=n_ept)
     torch.cuda.synchronize()
     return {k: v.cpu().numpy() for k, v in out.items()}
 
@@ -99,3 +100,54 @@ def test_next_tree_errors(cuda_device):
     got = _run(cuda_device, logits, parent, cand, path, accept_len, next_token, tp, tr, K)
     _compare(got, ref)
     assert got["status"].tolist() == [3, 3, 3]       # state 2 template bad; failed; no token
+
+
+@pytest.mark.parametrize("n_ept,c,T_next,K", [(2, 3, 64, 8), (3, 2, 96, 16), (5, 1, 48, 4),
+                                           (4, 3, 128, 16)])
+def test_next_tree_ensemble_tokens(cuda_device, n_ept, c, T_next, K):
+    """n_ept ensemble chains on every candidate (Section 3, Ensemble Prompt
+    Tokens): guesses from the chains' averaged logits, state from the
+    shortest chain; NaN and -inf logits included."""
+    w = W.scaled(W.WORKLOADS["mobilellama"], B=6, T=16 * (1 + n_ept * c), n_cand=16,
+                 chains=f"ept{n_ept}x{c}")
+    s = W.make_step_inputs(w, seed=n_ept * 10 + c)
+    logits = s.logits.copy()
+    logits[0, :, 17] = np.nan
+    logits[1, :, :9] = -np.inf
+    logits[2, :, 100] = np.inf                    # +inf + -inf averages to NaN
+    logits[2, ::2, 101] = -np.inf
+    acc = oracle.accept_path(oracle.node_argmax(logits), s.cand_tokens, s.parent, s.prefix_len,
+                             w.V, w.S_max)
+    tp, tr = W.make_tree_templates(c + 2, T_next, K, np.random.default_rng(K), n_ept=n_ept)
+    for ne in (n_ept, 1, n_ept + 1):              # n_ept + 1: too few heads, state 0
+        ref = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                               acc["next_token"], tp, tr, K, n_ept=ne)
+        got = _run(cuda_device, logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                   acc["next_token"], tp, tr, K, n_ept=ne)
+        _compare(got, ref)
+        if ne == n_ept + 1:
+            assert (got["next_state"][got["status"] == 0] == 0).all()
+        elif ne == n_ept:
+            assert (got["next_state"][got["status"] == 0] == min(c, c + 1)).all()
+
+
+def test_next_tree_ensemble_hand_tree(cuda_device):
+    """Two chains under the accepted node whose averaged logits rank
+    differently from either chain alone (the oracle's hand-worked case)."""
+    parent = np.array([[-1, 0, 1, 1, 2, 3, 0]] * 2, np.int32)
+    parent[1, 5] = 0                              # sequence 1: chain 2 one position short
+    cand = np.array([[9, 4, -1, -1, -1, -1, -1]] * 2, np.int32)
+    logits = np.zeros((2, 7, 4), np.float32)
+    logits[:, 2] = [4, 0, 1, 0]
+    logits[:, 3] = [0, 6, 1, 0]
+    logits[:, 4] = [1, 5, 0, 2]
+    logits[:, 5] = [3, -5, 0, 2]
+    path = np.array([[0, 1, -1, -1, -1, -1, -1]] * 2, np.int32)
+    tp = np.array([[-1, 0, 1, 2, 3], [-1, 0, 0, 1, 2], [-1, 0, 1, 1, 0]], np.int32)
+    tr = np.array([[0, -1, -1, -1, -1], [0, 0, -1, -1, -1], [0, 0, 0, 1, -1]], np.int32)
+    alen, nt = np.array([2, 2], np.int32), np.array([7, 8], np.int32)
+    got = _run(cuda_device, logits, parent, cand, path, alen, nt, tp, tr, 2, n_ept=2)
+    assert got["status"].tolist() == [0, 0] and got["next_state"].tolist() == [2, 1]
+    assert got["next_cand"].tolist() == [[7, 1, 0, 3, -1], [8, 1, -1, -1, -1]]
+    ref = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, 2, n_ept=2)
+    _compare(got, ref)

@@ -1,11 +1,14 @@
 """Pins for the oracle's next-step candidate generation (Section 3 step (1):
 the prompt tokens appended to the accepted token predict the following
-tokens; Appendix, Definition of tree states: the next tree takes state T_k,
-whose candidate subtree is at most k deep).
+tokens; Section 3, Ensemble Prompt Tokens: n_ept tokens per prompt position,
+the guess from the average of their logits; Appendix, Definition of tree
+states: the next tree takes state T_k, whose candidate subtree is at most k
+deep).
 
-Expected values come from numpy's stable argsort (top-k order), a hand-worked
-example, an independent restatement on small random cases (chain found by a
-breadth-first search over the tree, ranks by numpy), and the state rule."""
+Expected values come from numpy's stable argsort (top-k order), hand-worked
+examples (one and two ensemble chains), an independent restatement on small
+random cases (chains found from per-node child lists, averages by an explicit
+fp32 loop, ranks by numpy), and the state rule."""
 import numpy as np
 import pytest
 
@@ -62,9 +65,11 @@ def test_hand_worked_example():
     assert r["next_cand"][0].tolist() == [4, 2, 3, 5, -1, -1]
 
 
-def _independent(logits, parent, cand, path, accept_len, next_token, tp, tr, K):
-    """Restatement: the chain is found by breadth-first search from the end node
-    over prompt children (lowest index first), ranks come from numpy."""
+def _independent(logits, parent, cand, path, accept_len, next_token, tp, tr, K, n_ept=1):
+    """Restatement: per-node lists of prompt children (lowest index first); the
+    end node's first n_ept prompt children head the chains, each continued
+    through first children; the average over the chains is an explicit fp32
+    loop; ranks come from numpy."""
     B, T = parent.shape
     n_states, T_next = tp.shape
     out_p = np.full((B, T_next), -1)
@@ -74,12 +79,23 @@ def _independent(logits, parent, cand, path, accept_len, next_token, tp, tr, K):
         e = path[b, accept_len[b] - 1]
         children = {u: sorted(i for i in range(T) if parent[b, i] == u and cand[b, i] == -1)
                     for u in range(T)}
-        chain, u = [], e
-        while children[u]:
-            u = children[u][0]
-            chain.append(u)
-        k = min(len(chain), n_states - 1)
-        ranks = [np.lexsort((np.arange(logits.shape[2]), -logits[b, c]))[:K] for c in chain]
+        chains = []
+        for head in children[e][:n_ept]:
+            chain, u = [head], head
+            while children[u]:
+                u = children[u][0]
+                chain.append(u)
+            chains.append(chain)
+        k = min(len(c) for c in chains) if len(chains) == n_ept else 0
+        k = min(k, n_states - 1)
+        ranks = []
+        for d in range(k):
+            acc = np.array(logits[b, chains[0][d]], np.float32)
+            for c in chains[1:]:
+                acc = (acc + logits[b, c[d]]).astype(np.float32)
+            avg = (acc / np.float32(n_ept)).astype(np.float32)
+            nan = np.isnan(avg)          # NaN ranks first; numpy would sort it last
+            ranks.append(np.lexsort((np.arange(logits.shape[2]), -np.where(nan, 0, avg), ~nan))[:K])
         depth = {0: 0}
         for i in range(1, T_next):
             depth[i] = depth[tp[k, i]] + 1 if tr[k, i] >= 0 else None
@@ -109,6 +125,109 @@ def test_random_cases_match_independent_restatement(seed):
     np.testing.assert_array_equal(r["next_parent"], ref_p)
     np.testing.assert_array_equal(r["next_cand"], ref_c)
     np.testing.assert_array_equal(r["next_state"], ref_s)
+
+
+def _ept_hand_tree():
+    """0 root; 1 candidate under 0; prompt nodes 2, 3 under 1 (two ensemble
+    chains), 4 under 2 and 5 under 3 (their second positions), 6 under 0."""
+    parent = np.array([[-1, 0, 1, 1, 2, 3, 0]])
+    cand = np.array([[9, 4, -1, -1, -1, -1, -1]])
+    logits = np.zeros((1, 7, 4), np.float32)
+    logits[0, 2] = [4, 0, 1, 0]        # chain 1, position 1
+    logits[0, 3] = [0, 6, 1, 0]        # chain 2, position 1 -> average [2, 3, 1, 0]
+    logits[0, 4] = [1, 5, 0, 2]        # chain 1, position 2
+    logits[0, 5] = [3, -5, 0, 2]       # chain 2, position 2 -> average [2, 0, 0, 2]
+    logits[0, 6] = [0, 0, 0, 99]
+    path = np.array([[0, 1, -1, -1, -1, -1, -1]])
+    tp = np.array([[-1, 0, 1, 2, 3],
+                   [-1, 0, 0, 1, 2],
+                   [-1, 0, 1, 1, 0]])
+    tr = np.array([[0, -1, -1, -1, -1],
+                   [0, 0, -1, -1, -1],
+                   [0, 0, 0, 1, -1]])     # state 2: depth 1 rank 0, depth 2 ranks 0 and 1
+    return logits, parent, cand, path, np.array([2]), np.array([7]), tp, tr
+
+
+def test_ept_hand_worked_example():
+    logits, parent, cand, path, alen, nt, tp, tr = _ept_hand_tree()
+    r = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=2)
+    # averaged rankings: position 1 -> 1, 0, 2, 3; position 2 -> 0, 3, 1, 2 (ties: lower index)
+    assert r["status"].tolist() == [0] and r["next_state"].tolist() == [2]
+    assert r["next_parent"][0].tolist() == [-1, 0, 1, 1, 0]
+    assert r["next_cand"][0].tolist() == [7, 1, 0, 3, -1]
+    # one ensemble token: chain 2 -> 4 alone, rankings 0, 2, ... and 1, 3, ...
+    r1 = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=1)
+    assert r1["next_cand"][0].tolist() == [7, 0, 1, 3, -1]
+    assert (oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2)["next_cand"] ==
+            r1["next_cand"]).all()
+    # three ensemble tokens but only two prompt children: state 0
+    r3 = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=3)
+    assert r3["next_state"].tolist() == [0] and r3["next_cand"][0].tolist() == [7, -1, -1, -1, -1]
+
+
+def test_ept_state_is_the_shortest_chain():
+    logits, parent, cand, path, alen, nt, tp, tr = _ept_hand_tree()
+    parent = parent.copy()
+    parent[0, 5] = 0                   # chain 2 loses its second position
+    r = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=2)
+    assert r["next_state"].tolist() == [1]
+    assert r["next_cand"][0].tolist() == [7, 1, -1, -1, -1]
+    assert r["next_parent"][0].tolist() == [-1, 0, 0, 1, 2]
+
+
+@pytest.mark.parametrize("n_ept", [2, 4])
+def test_ept_identical_chains_match_one_chain(n_ept):
+    """With every ensemble chain carrying the same logits, the fp32 average of
+    n_ept = 2^j copies is exact, so the guesses equal those of one chain."""
+    rng = np.random.default_rng(n_ept)
+    w = W.scaled(W.WORKLOADS["tiny"], B=3, V=300, T=16 * (1 + 2 * n_ept), chains=f"ept{n_ept}x2")
+    s = W.make_step_inputs(w, seed=5)
+    logits = s.logits.copy()
+    for b in range(w.B):
+        for i in range(w.T):
+            if s.cand_tokens[b, i] == -1 and s.cand_tokens[b, s.parent[b, i]] != -1:
+                # an ensemble head: copy the first sibling head's chain logits
+                sib = [j for j in range(w.T) if s.parent[b, j] == s.parent[b, i]
+                       and s.cand_tokens[b, j] == -1]
+                first = sib[0]
+                logits[b, i] = logits[b, first]
+                ci = [j for j in range(w.T) if s.parent[b, j] == i]
+                cf = [j for j in range(w.T) if s.parent[b, j] == first]
+                logits[b, ci[0]] = logits[b, cf[0]]
+    acc = oracle.accept_path(oracle.node_argmax(logits), s.cand_tokens, s.parent, s.prefix_len,
+                             w.V, w.S_max)
+    tp, tr = W.make_tree_templates(3, 40, 4, rng, n_ept=n_ept)
+    r = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                         acc["next_token"], tp, tr, 4, n_ept=n_ept)
+    r1 = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                          acc["next_token"], tp, tr, 4, n_ept=1)
+    assert (r["status"] == 0).all()
+    for k in ("next_parent", "next_cand", "next_state"):
+        np.testing.assert_array_equal(r[k], r1[k], err_msg=k)
+
+
+@pytest.mark.parametrize("seed,n_ept", [(0, 2), (1, 3), (2, 2), (3, 5)])
+def test_ept_random_cases_match_independent_restatement(seed, n_ept):
+    rng = np.random.default_rng(100 + seed)
+    c = 1 + seed % 3
+    w = W.scaled(W.WORKLOADS["tiny"], B=4, V=257, T=12 * (1 + n_ept * c), n_cand=12,
+                 chains=f"ept{n_ept}x{c}")
+    s = W.make_step_inputs(w, seed=seed)
+    logits = s.logits.copy()
+    logits[0, :, 3] = np.nan
+    logits[1, :, :5] = -np.inf
+    acc = oracle.accept_path(oracle.node_argmax(logits), s.cand_tokens, s.parent, s.prefix_len,
+                             w.V, w.S_max)
+    n_states, K = 4, 5
+    tp, tr = W.make_tree_templates(n_states, 48, K, rng, n_ept=n_ept)
+    r = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                         acc["next_token"], tp, tr, K, n_ept=n_ept)
+    ref_p, ref_c, ref_s = _independent(logits, s.parent, s.cand_tokens, acc["path"],
+                                       acc["accept_len"], acc["next_token"], tp, tr, K, n_ept)
+    assert (r["status"] == 0).all()
+    np.testing.assert_array_equal(r["next_state"], ref_s)
+    np.testing.assert_array_equal(r["next_parent"], ref_p)
+    np.testing.assert_array_equal(r["next_cand"], ref_c)
 
 
 def test_templates_respect_the_state_depth_rule():
