@@ -64,6 +64,53 @@ def attention_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
+def per_layer_attention(w, t, prefix, parent, out, dev, reps):
+    """Attention as a model runs it: L ppd_tree_attention calls of one layer
+    each, captured in a CUDA graph and replayed `reps` times (CUDA events on the
+    replay stream, median).  With a workspace the library shares each call's
+    key tiles over all SMs when the layer has fewer slices than SMs; without,
+    one whole slice per SM."""
+    import torch
+
+    from paper_2405_18628_gb300 import ppd
+
+    st = torch.zeros(w.B, dtype=torch.int32, device=dev)
+    ws = ppd.workspace(1, w.B, w.H, w.T, w.D, 1, w.S_max, device=dev)
+    res = {}
+    for mode, wsx in (("split", ws), ("unsplit", None)):
+        def layers():
+            for l in range(w.L):
+                ppd.ppd_tree_attention(t["q"][l:l + 1], t["k_cache"][l:l + 1], t["v_cache"][l:l + 1],
+                                       t["k_tree"][l:l + 1], t["v_tree"][l:l + 1], prefix, parent,
+                                       out[l:l + 1], st, workspace=wsx)
+        layers()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream()
+        cap.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(cap):
+            with torch.cuda.graph(g, stream=cap):
+                layers()
+        torch.cuda.current_stream().wait_stream(cap)
+        s = torch.cuda.current_stream()
+        for _ in range(5):
+            g.replay()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for a, b in ev:
+            a.record(s)
+            g.replay()
+            b.record(s)
+        torch.cuda.synchronize()
+        if (st.cpu().numpy() != 0).any():
+            raise SystemExit(f"per-layer attention reported device status {st.cpu().tolist()}")
+        us = statistics.median(a.elapsed_time(b) for a, b in ev) * 1e3
+        res[mode] = {"us_per_step": us, "us_per_layer": us / w.L,
+                     "gbs": attention_bytes(w) / (us * 1e-6) / 1e9}
+        del g
+    return {"graph": True, "layers": w.L, "slices_per_layer": w.B * w.H, **res}
+
+
 def measured_peak_gbs():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -217,6 +264,9 @@ def parse():
     ap.add_argument("--next-tree", action="store_true",
                     help="also time next-step candidate generation (ppd_next_tree, 5 tree "
                          "states, 8 guesses per depth) after each step")
+    ap.add_argument("--per-layer", action="store_true",
+                    help="also time the attention as it runs inside a model: one "
+                         "ppd_tree_attention call per layer, the L calls captured in a CUDA graph")
     ap.add_argument("--layers", type=int, default=0,
                     help="run the workload with this many layers (profiling captures)")
     ap.add_argument("--l2", default="auto", choices=["auto", "flush", "none"],
@@ -479,6 +529,11 @@ def main():
                      "state_histogram": np.bincount(nxt["state"].cpu().numpy(),
                                                     minlength=n_states).tolist()}
 
+    # ---------------------------------------------------------------- per-layer attention
+    per_layer = None
+    if args.per_layer:
+        per_layer = per_layer_attention(w, t, prefix, parent, bufs.out, dev, min(K, 100))
+
     # ---------------------------------------------------------------- tree-size profile
     profile = None
     if args.tree_sizes:
@@ -534,6 +589,8 @@ def main():
             line["tree_size_profile"] = profile
         if next_tree is not None:
             line["next_tree"] = next_tree
+        if per_layer is not None:
+            line["per_layer_attention"] = per_layer
         print(json.dumps(line), flush=True)
     if pg:
         pg.barrier()

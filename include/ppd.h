@@ -74,7 +74,8 @@ typedef enum { PPD_BF16 = 0, PPD_F32 = 1 } ppd_dtype;
  * (device memory, any contents, 256-byte aligned, caller-owned; it may be
  * reused between calls that are ordered on one stream).  Covers the per-split
  * partial maxima (and softmax statistics) of the node argmax, the fused step's
- * per-CTA scratch and, for PPD_F32, the bf16 copies of Q/K/V.
+ * per-CTA scratch, for PPD_F32 the bf16 copies of Q/K/V, and the attention
+ * work split's per-SM records and partial softmax states.
  */
 size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt);
 
@@ -92,7 +93,12 @@ size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, 
  *   PPD_ERR_CAPACITY / PPD_ERR_TIMEOUT; outputs of a failed sequence are
  *   unspecified.  Cache rows at or beyond prefix_len[b] are never used and may
  *   hold anything, NaN included.
- * Workspace: ppd_workspace_bytes(...) bytes (only PPD_F32 uses it).
+ * Workspace: ppd_workspace_bytes(...) bytes.  With it (and B <= 64) the
+ * (layer, sequence, head) slices left over after full rounds of one slice per
+ * SM -- all of them, when there are fewer slices than SMs -- are shared out
+ * over every SM by their key tiles, the slices cut between SMs being merged by
+ * a second, small grid; a bf16 call may pass none (NULL or fewer bytes) and
+ * then runs one whole slice per SM at a time.
  */
 ppd_status ppd_tree_attention(const void *q, const void *k_cache, const void *v_cache,
                               const void *k_tree, const void *v_tree,

@@ -49,10 +49,15 @@ int num_sms()
 
 int argmax_splits(int64_t rows, int V) { return ppd::argmax_split_count(rows, V); }
 
+// Workspace: the argmax partials, the side warp's scratch, the bf16 copies of
+// fp32 operands, then the work split's per-CTA records and partial states.
 struct WsLayout {
-    size_t part_val, part_idx, part_stats, node_lse, node_ent, side, conv, total;
+    size_t part_val, part_idx, part_stats, node_lse, node_ent, side, conv, split_rec, split_part,
+        total;
     int splits;
 };
+
+int split_grid() { return num_sms() < ppd::kSplitMaxGrid ? num_sms() : ppd::kSplitMaxGrid; }
 
 WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt)
 {
@@ -77,6 +82,10 @@ WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, p
         const size_t lbh = (size_t)L * B * H;
         off = align_up(off + lbh * ((size_t)3 * T + 2 * (size_t)S_max) * D * 2);
     }
+    w.split_rec = off;
+    off = align_up(off + (size_t)split_grid() * sizeof(ppd::SplitRecord));
+    w.split_part = off;
+    off = align_up(off + (size_t)2 * split_grid() * ppd::kSplitRows * (D + 2) * sizeof(float));
     w.total = off;
     return w;
 }
@@ -147,11 +156,31 @@ bool attn_dims_ok(int L, int B, int H, int T, int D, int S_max, ppd_dtype dt)
 }
 
 // Enqueue the attention of all L*B*H slices (bf16 operands).
+// Does sharing the launch's key tiles over all SMs (the work split) beat one
+// whole slice per SM?  Only launches with fewer slices than SMs can gain (with
+// more, the last round's idle SMs cost less than the merge; measured on the
+// Vicuna-7B/13B and MobileLlama shapes).  Counted in tiles of 128 keys, with
+// S_max standing in for the (device-side) prefix lengths: one round of whole
+// slices takes t_u tiles; the split takes its share of all tiles plus about
+// kSplitCostTiles for the range planning and the merge grid.
+constexpr long long kSplitCostTiles = 6;
+
+bool split_pays(const AttnParams &p, int sms)
+{
+    if (p.n_units >= sms) return false;
+    const long long t_u = (p.S_max + 127) / 128 + p.n_tt;
+    const long long share = ((long long)p.n_units * t_u + sms - 1) / sms;
+    return share + kSplitCostTiles < t_u;
+}
+
+// With a workspace of the full layout, a batch of at most kSplitMaxB and a
+// launch that gains from it, the key tiles are shared evenly over the CTAs
+// (see ppd_attention_common.cuh).
 ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, const void *kt,
                              const void *vt, const int32_t *prefix_len, const int32_t *parent,
                              int L, int B, int H, int T, int D, int S_max, float scale, float *out,
-                             float *lse, int32_t *dev_status, const ppd::FusedStep *fused,
-                             bool programmatic, cudaStream_t stream)
+                             float *lse, int32_t *dev_status, uint8_t *ws, const WsLayout *wl,
+                             const ppd::FusedStep *fused, bool programmatic, cudaStream_t stream)
 {
     const int T_pad = (T + 31) & ~31;
     const uint64_t lbh = (uint64_t)L * B * H;
@@ -182,9 +211,14 @@ ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, cons
     p.n_units = (int)lbh * p.n_qb;
     const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
     p.scale_log2 = sc * 1.4426950408889634f;
+    if (ws && wl && B <= ppd::kSplitMaxB && split_pays(p, split_grid())) {
+        p.split = 1;
+        p.split_rec = reinterpret_cast<ppd::SplitRecord *>(ws + wl->split_rec);
+        p.split_part = reinterpret_cast<float *>(ws + wl->split_part);
+    }
     p.fused = fused != nullptr;
     if (fused) p.fs = *fused;
-    return cuda_status(ppd::launch_tree_attention(m, p, D, num_sms(), programmatic, stream));
+    return cuda_status(ppd::launch_tree_attention(m, p, D, split_grid(), programmatic, stream));
 }
 
 // fp32 operands: round to bf16 copies in the workspace first.
@@ -199,7 +233,8 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
     // phase, so it may overlap the preceding (argmax) grid.
     if (dt == PPD_BF16)
         return enqueue_attention(q, kc, vc, kt, vt, prefix_len, parent, L, B, H, T, D, S_max, scale,
-                                 out, lse, dev_status, fused, fused != nullptr, stream);
+                                 out, lse, dev_status, ws, ws ? &wl : nullptr, fused,
+                                 fused != nullptr, stream);
     const int64_t lbh = (int64_t)L * B * H;
     const int64_t n_t = lbh * T * D, n_c = lbh * (int64_t)S_max * D;
     uint16_t *bq = reinterpret_cast<uint16_t *>(ws + wl.conv);
@@ -214,7 +249,7 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
         ppd::launch_round_bf16((const float *)vc, bvc, n_c, stream) != cudaSuccess)
         return PPD_ERR_CUDA;
     return enqueue_attention(bq, bkc, bvc, bkt, bvt, prefix_len, parent, L, B, H, T, D, S_max,
-                             scale, out, lse, dev_status, fused, false, stream);
+                             scale, out, lse, dev_status, ws, &wl, fused, false, stream);
 }
 
 }  // namespace
@@ -340,6 +375,7 @@ size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, 
     return workspace_layout(L, B, H, T, D, V, S_max, dt).total;
 }
 
+
 const char *ppd_status_string(ppd_status s)
 {
     switch (s) {
@@ -369,13 +405,14 @@ ppd_status ppd_tree_attention(const void *q, const void *k_cache, const void *v_
         !aligned(v_tree, 16) || !aligned(out, 4) || !aligned(lse, 4))
         return PPD_ERR_INVALID_ARG;
     const WsLayout wl = workspace_layout(L, B, H, T, D, 1, S_max, dt);
-    if (dt == PPD_F32 && (!workspace || ws_bytes < wl.total || !aligned(workspace, kAlign)))
-        return PPD_ERR_INVALID_ARG;
+    const bool ws_ok = workspace && ws_bytes >= wl.total && aligned(workspace, kAlign);
+    if (dt == PPD_F32 && !ws_ok) return PPD_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (cudaMemsetAsync(dev_status, 0, (size_t)B * 4, s) != cudaSuccess) return PPD_ERR_CUDA;
+    // a bf16 call without a full workspace runs unsplit
     return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B, H,
                                  T, D, S_max, dt, scale, out, lse, dev_status,
-                                 static_cast<uint8_t *>(workspace), wl, nullptr, s);
+                                 ws_ok ? static_cast<uint8_t *>(workspace) : nullptr, wl, nullptr, s);
 }
 
 ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *argmax_out,

@@ -29,7 +29,9 @@
 // and their V rows are zeroed in shared memory before the PV product.  O is
 // double-buffered in TMEM and a unit's output is read back only after the
 // next unit's first tile, so the stream of tiles never waits for a unit's
-// last PV product.
+// last PV product.  With the work split (ppd_attention_common.cuh) a CTA's
+// tiles are an equal share of the launch's; a unit cut by a share boundary is
+// done in parts whose partial states the last part merges.
 #include "ppd_attention_common.cuh"
 
 #include <cmath>
@@ -83,13 +85,15 @@ struct AttnLayout {
     static constexpr uint32_t OFF_TMEMPTR = OFF_BAR + NBAR * 8;
     static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
     static constexpr uint32_t OFF_M2 = (OFF_ABORT + 4 + 15) & ~15u;
-    static constexpr uint32_t OFF_LINV = OFF_M2 + TPMAX * 4;      // [OB][TPMAX] 1 / row sums
-    static constexpr uint32_t OFF_UNION = OFF_LINV + OB * TPMAX * 4;
+    static constexpr uint32_t OFF_LINV = OFF_M2 + TPMAX * 4;      // [OB][TPMAX] 1 / row sums (row sums of a partial)
+    static constexpr uint32_t OFF_PMX = OFF_LINV + OB * TPMAX * 4;  // [OB][TPMAX] maxima of a partial
+    static constexpr uint32_t OFF_UNION = OFF_PMX + OB * TPMAX * 4;
     // union: ancestor bitsets [TPMAX][ANC_WORDS] u32, or reduction scratch [2][4][NC_MAX] f32
     static constexpr uint32_t ANC_BYTES = TPMAX * ANC_WORDS * 4;
     static constexpr uint32_t RED_BYTES = 2 * 4 * NC_MAX * 4;
     static constexpr uint32_t UNION_BYTES = ANC_BYTES > RED_BYTES ? ANC_BYTES : RED_BYTES;
-    static constexpr uint32_t SMEM_BYTES = OFF_UNION + UNION_BYTES;
+    static constexpr uint32_t OFF_RANGE = (OFF_UNION + UNION_BYTES + 15) & ~15u;   // WorkRange
+    static constexpr uint32_t SMEM_BYTES = OFF_RANGE + ((sizeof(WorkRange) + 15) & ~15u);
     // TMEM columns: S0 | S1 | O0 (hi | lo) | O1 (hi | lo)
     static constexpr uint32_t T_S = 0, T_O = 2 * TPMAX;
     static constexpr uint32_t TMEM_COLS = 512;
@@ -109,7 +113,7 @@ PPD_DEV uint32_t p_offset(int g)
 }
 
 
-template <int D>
+template <int D, bool SPLIT>
 __global__ void __launch_bounds__(352, 1)
 tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                       const __grid_constant__ CUtensorMap map_kc,
@@ -156,14 +160,26 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         tmem_alloc(tmem_ptr, Lay::TMEM_COLS);
         tmem_relinquish();
     }
+    WorkRange *wr_s = reinterpret_cast<WorkRange *>(smem + Lay::OFF_RANGE);
+    if (warp == 8) {
+        const WorkRange w = plan_range(p, lane);   // whole units round-robin without p.split
+        if (lane == 0) {
+            *wr_s = w;
+            if (SPLIT) p.split_rec[blockIdx.x].u = -1;   // no cut unit recorded yet
+        }
+    }
+    // the merge of cut units (a dependent launch) may be scheduled now; it waits
+    // for this grid to complete
+    if (SPLIT) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_ptr;
+    const WorkRange &wr = *wr_s;
 
     if (warp == 10) {
         // ------------------------------------------------------------ fused-step side work
-        if (p.fused) fused_side_warp(p, lane);
+        if (p.fused) fused_side_warp(p, wr, lane);
     } else if (warp == 8) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
@@ -175,8 +191,10 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             const uint64_t pol = l2_policy_evict_first();
             const uint32_t q_tx = (uint32_t)T_pad * 128u * Lay::DCH;
             int g = 0, k = 0;
-            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
-                const UnitInfo ui = unit_info(p, u);
+            SegIter<SPLIT> it(wr);
+            for (Seg sg; it.next(p, sg); ++k) {
+                const UnitInfo &ui = sg.ui;
+                const int u = sg.u;
                 const int qs = k % Lay::QS;
                 if (k >= Lay::QS)
                     mbar_wait(bars + Lay::B_QEMPTY + qs, ((k / Lay::QS) - 1) & 1, abort_flag);
@@ -187,7 +205,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::Q_GROUP_BYTES,
                                     &map_q, bars + Lay::B_QFULL + qs, c * 64, 0, u, pol);
                 }
-                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                for (int j = sg.j0; j < sg.j1; ++j, ++g) {
                     const bool tree = (j == ui.n_pref);
                     const int row = tree ? 0 : j * Lay::KT;
                     const int ks = g % Lay::KS;
@@ -264,12 +282,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             int prev_g = -1;
             bool prev_first = false;
             uint32_t prev_to = 0;
-            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
-                const UnitInfo ui = unit_info(p, u);
+            SegIter<SPLIT> it(wr);
+            for (Seg sg; it.next(p, sg); ++k) {
                 const int qs = k % Lay::QS;
                 const uint32_t t_o = tmem_base + Lay::T_O + (uint32_t)(k % Lay::OB) * 2 * TPMAX;
                 mbar_wait(bars + Lay::B_QFULL + qs, (k / Lay::QS) & 1, abort_flag);
-                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                for (int j = sg.j0; j < sg.j1; ++j, ++g) {
                     const int ks = g % Lay::KS;
                     const int sb = g & 1;
                     mbar_wait(bars + Lay::B_KFULL + ks, (g / Lay::KS) & 1, abort_flag);
@@ -289,10 +307,10 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     }
                     umma_commit(bars + Lay::B_SFULL + sb);
                     if (!Lay::P_IN_K) umma_commit(bars + Lay::B_KEMPTY + ks);
-                    if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
+                    if (j == sg.j1 - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
                     if (prev_g >= 0) issue_pv(prev_g, prev_first, prev_to);
                     prev_g = g;
-                    prev_first = (j == 0);
+                    prev_first = (j == sg.j0);
                     prev_to = t_o;
                 }
             }
@@ -316,6 +334,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         const float sl2 = p.scale_log2;
         float *red_wg = red + wg * 4 * Lay::NC_MAX;
         float *linv = reinterpret_cast<float *>(smem + Lay::OFF_LINV);   // [OB][TPMAX]
+        float *pmx = reinterpret_cast<float *>(smem + Lay::OFF_PMX);     // [OB][TPMAX]
 
         constexpr int NL = Lay::NC_MAX;
         float lacc[NL];   // this key row's share of every owned query's row sum
@@ -325,9 +344,12 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         int cur_b = -1;
         int g = 0;
         int cur_k = 0;        // this CTA's unit counter (selects the O accumulator)
-        // a finished unit whose output still sits in TMEM
-        bool pend = false;
-        int pend_u = 0, pend_ob = 0, pend_g = 0;
+        // a finished segment whose output still sits in TMEM; a partial one (a
+        // unit cut by the work split) goes to its slot instead of the output
+        // pend_f: bit 0 a segment is pending, bit 1 it is partial, bit 2 it was
+        // the range's first segment, bit 3 its O accumulator
+        int pend_f = 0, pend_u = 0, pend_g = 0;
+
 
         // Probabilities of the 16 query columns [cb, cb+16) of this thread's key row
         // from its raw scores r, against the current running maxima, exponents
@@ -518,9 +540,50 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             tc_fence_before();
         };
 
+        // Partial state of a cut unit into slot `slot`: O (hi + lo) unnormalised,
+        // each query's running maximum and row sum.
+        const size_t slot_floats = split_slot_floats(D);
+        auto write_partial = [&](int slot, int ob, int g_last) {
+            mbar_wait(bars + Lay::B_PFREE + g_last % Lay::PB, (g_last / Lay::PB) & 1, abort_flag);
+            tc_fence_after();
+            float *base = p.split_part + (size_t)slot * slot_floats;
+            if (wq * 32 < D) {
+                const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * 2 * TPMAX;
+#pragma unroll
+                for (int ch = 0; ch < Lay::NC_MAX / 16; ++ch) {
+                    if (ch * 16 < NC) {
+                        uint32_t rh[16], rl[16];
+                        tmem_ld16(t_o + q0 + ch * 16, rh);
+                        tmem_ld16(t_o + T_pad + q0 + ch * 16, rl);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const int q = q0 + ch * 16 + e;
+                            if (q < T) base[(size_t)q * D + t] = __uint_as_float(rh[e]) + __uint_as_float(rl[e]);
+                        }
+                    }
+                }
+            }
+            if (t < NC && q0 + t < T) {
+                base[(size_t)kSplitRows * D + q0 + t] = pmx[ob * TPMAX + q0 + t];
+                base[(size_t)kSplitRows * D + kSplitRows + q0 + t] = linv[ob * TPMAX + q0 + t];
+            }
+            tc_fence_before();
+        };
+
+        // The pending segment: a whole unit's output, or a part's state (counted
+        // in at the end of the range).
+        auto flush_pending = [&]() {
+            const int pend_ob = (pend_f >> 3) & 1;
+            if (!SPLIT || !(pend_f & 2)) read_back(pend_u, pend_ob, pend_g);
+            else write_partial(2 * (int)blockIdx.x + ((pend_f & 4) ? 0 : 1), pend_ob, pend_g);
+        };
+
         int k = 0;
-        for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
-            const UnitInfo ui = unit_info(p, u);
+        SegIter<SPLIT> it(wr);
+        for (Seg sg; it.next(p, sg); ++k) {
+            const UnitInfo &ui = sg.ui;
+            const int u = sg.u;
             cur_k = k;
             const int ob = k % Lay::OB;
             const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)ob * 2 * TPMAX;
@@ -568,7 +631,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                 cur_b = ui.b;
             }
 
-            for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+            for (int j = sg.j0; j < sg.j1; ++j, ++g) {
                 const bool tree = (j == ui.n_pref);
                 const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
                 const bool row_ok = t < n_valid;
@@ -597,7 +660,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     if (gc0 < NC) {
                         const bool two = gc0 + 16 < NC;
                         bool exact;
-                        if (j > 0) {
+                        if (j > sg.j0) {
                             float maxd = -INFINITY;
                             if (kind == kMaskNone) p_group(kind_t<kMaskNone>{}, t_s, gc0, two, row_ok, pbuf, maxd);
                             else if (kind == kMaskRows) p_group(kind_t<kMaskRows>{}, t_s, gc0, two, row_ok, pbuf, maxd);
@@ -608,7 +671,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                             exact = true;
                         }
                         if (exact) {
-                            const bool later = j > 0;
+                            const bool later = j > sg.j0;
                             if (kind == kMaskNone) exact_group(kind_t<kMaskNone>{}, t_s, gc0, two, row_ok, pbuf, later, o_ready);
                             else if (kind == kMaskRows) exact_group(kind_t<kMaskRows>{}, t_s, gc0, two, row_ok, pbuf, later, o_ready);
                             else exact_group(kind_t<kMaskTree>{}, t_s, gc0, two, row_ok, pbuf, later, o_ready);
@@ -637,13 +700,13 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                     mbar_arrive(bars + Lay::B_SFREE + sb);
                 }
 
-                // the previous unit's output, once this unit's first tile is on its way
-                if (j == 0 && pend) {
-                    read_back(pend_u, pend_ob, pend_g);
-                    pend = false;
+                // the previous segment's output, once this segment's first tile is on its way
+                if (j == sg.j0 && pend_f) {
+                    flush_pending();
+                    pend_f = 0;
                 }
 
-                if (j == ui.n_tiles - 1) {
+                if (j == sg.j1 - 1) {
                     // ------------------------------------------ unit end: row sums, LSE
                     named_bar_sync(1 + wg, 128);   // every thread is done reading alpha
 #pragma unroll
@@ -661,23 +724,34 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
                         const float l = red_wg[t] + red_wg[Lay::NC_MAX + t] +
                                         red_wg[2 * Lay::NC_MAX + t] + red_wg[3 * Lay::NC_MAX + t];
                         const int q = q0 + t;
-                        if (p.lse && q < T)
-                            p.lse[(size_t)u * T + q] = (m2[q] + lg2(l)) * 0.69314718055994530942f;
-                        linv[ob * TPMAX + q] = rcp(l);
+                        if (!SPLIT || seg_whole(sg)) {
+                            if (p.lse && q < T)
+                                p.lse[(size_t)u * T + q] = (m2[q] + lg2(l)) * 0.69314718055994530942f;
+                            linv[ob * TPMAX + q] = rcp(l);
+                        } else {
+                            linv[ob * TPMAX + q] = l;
+                            pmx[ob * TPMAX + q] = m2[q];
+                        }
                         m2[q] = -INFINITY;
                     }
 #pragma unroll
                     for (int c = 0; c < NL; ++c) lacc[c] = 0.f;
-                    pend = true;
                     pend_u = u;
-                    pend_ob = ob;
                     pend_g = g;
+                    pend_f = 1 | (ob << 3);
+                    if (SPLIT && !seg_whole(sg)) {
+                        // a part: slot 2c for the tail range's first segment, 2c + 1 for its last
+                        pend_f |= 2 | (sg.u == wr.u_first ? 4 : 0);
+                        // the part holding the unit's first tile records it for the merge
+                        if (sg.j0 == 0 && threadIdx.x == 0)
+                            p.split_rec[blockIdx.x] = SplitRecord{seg_unit_origin(wr, it, sg), wr.n_tail, u, ui.n_tiles};
+                    }
                 }
             }
         }
-        if (pend) {
-            named_bar_sync(1 + wg, 128);   // the reciprocal row sums are in shared memory
-            read_back(pend_u, pend_ob, pend_g);
+        if (pend_f) {
+            named_bar_sync(1 + wg, 128);   // the row sums are in shared memory
+            flush_pending();
         }
     }
 
@@ -693,21 +767,63 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
     if (warp == 9) tmem_dealloc(tmem_base, Lay::TMEM_COLS);
 }
 
+// The merge of the units cut by the work split: blockIdx.x is an attention
+// CTA (gridDim.x = the attention grid), blockIdx.y a block of 256 / (D / 8)
+// rows of the unit that CTA recorded; each thread merges 8 columns of a row,
+// once the attention grid has completed.
+__global__ void __launch_bounds__(256) split_merge_kernel(const AttnParams p, int D)
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const SplitRecord r = p.split_rec[blockIdx.x];
+    if (r.u < 0) return;
+    const int per_row = D / 8;
+    const int rows_per_block = (int)blockDim.x / per_row;
+    const int lbh = r.u / p.n_qb, qb = r.u - lbh * p.n_qb;
+    const int n_rows = min(kSplitRows, p.T - qb * kSplitRows);
+    const int row = (int)blockIdx.y * rows_per_block + (int)threadIdx.x / per_row;
+    if (row >= n_rows) return;
+    const SplitParts sp = split_parts(r.n_tail, r.off, r.n_tiles);
+    split_merge_chunk(p.split_part, p.out, p.lse, sp, r.n_tail, (int)gridDim.x,
+                      (size_t)lbh * p.T + (size_t)qb * kSplitRows, row, ((int)threadIdx.x % per_row) * 8, D);
+}
+
+cudaError_t launch_split_merge(const AttnParams &p, int D, int grid, cudaStream_t stream)
+{
+    const int rows_per_block = 256 / (D / 8);
+    const int rows = p.T < kSplitRows ? p.T : kSplitRows;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid, (unsigned)((rows + rows_per_block - 1) / rows_per_block));
+    cfg.blockDim = dim3(256);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, split_merge_kernel, p, D);
+}
+
 template <int D>
 static cudaError_t launch_tree_attention_t(const AttnMaps &m, const AttnParams &p, int num_sms,
                                            bool programmatic, cudaStream_t stream)
 {
-    static std::atomic<uint64_t> configured{0};
-    return launch_attention_grid(tree_attention_kernel<D>, AttnLayout<D>::SMEM_BYTES, 352, configured, m,
-                                 p, num_sms, programmatic, stream);
+    static std::atomic<uint64_t> configured[2] = {{0}, {0}};
+    if (p.split)
+        return launch_attention_grid(tree_attention_kernel<D, true>, AttnLayout<D>::SMEM_BYTES, 352,
+                                     configured[1], m, p, num_sms, programmatic, stream);
+    return launch_attention_grid(tree_attention_kernel<D, false>, AttnLayout<D>::SMEM_BYTES, 352,
+                                 configured[0], m, p, num_sms, programmatic, stream);
 }
 
 cudaError_t launch_tree_attention(const AttnMaps &m, const AttnParams &p, int D, int num_sms,
                                   bool programmatic, cudaStream_t stream)
 {
-    if (p.T_pad > 64) return launch_tree_attention_rows(m, p, D, num_sms, programmatic, stream);
-    if (D == 128) return launch_tree_attention_t<128>(m, p, num_sms, programmatic, stream);
-    return launch_tree_attention_t<64>(m, p, num_sms, programmatic, stream);
+    cudaError_t e;
+    if (p.T_pad > 64) e = launch_tree_attention_rows(m, p, D, num_sms, programmatic, stream);
+    else if (D == 128) e = launch_tree_attention_t<128>(m, p, num_sms, programmatic, stream);
+    else e = launch_tree_attention_t<64>(m, p, num_sms, programmatic, stream);
+    if (e != cudaSuccess || !p.split) return e;
+    return launch_split_merge(p, D, attention_grid(p, num_sms), stream);
 }
 
 }  // namespace ppd

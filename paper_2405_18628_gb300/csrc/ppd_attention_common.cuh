@@ -1,13 +1,14 @@
 // ppd_attention_common.cuh -- pieces shared by the two tree-attention kernels
 // (ppd_attention.cu for trees of up to 64 tokens, ppd_attention_rows.cu for
-// 65..128): the unit walk, drain waits, mask kinds and the fused step's side
-// warp.
+// 65..512): the work split and unit walk, drain waits, mask kinds and the
+// fused step's side warp.
 #pragma once
 
 #include "ppd_accept.cuh"
 #include "ppd_device.cuh"
 #include "ppd_kernels.h"
 
+#include <algorithm>
 #include <atomic>
 #include <type_traits>
 
@@ -32,6 +33,256 @@ PPD_DEV UnitInfo unit_info(const AttnParams &p, int u)
     ui.n_pref = (ui.P + 127) >> 7;
     ui.n_tiles = ui.n_pref + p.n_tt;
     return ui;
+}
+
+// ------------------------------------------------------------------ work split
+//
+// Without p.split, units are taken round-robin (CTA c: units c, c+G, c+2G,
+// ...), whole.  With p.split (launches with fewer units than CTAs, where whole
+// units would leave SMs idle) all units are shared out by their key tiles: the
+// tiles (unit u's tiles 0..n_tiles(u)-1, units in order) go to the CTAs in
+// equal contiguous ranges (CTA c: tiles [c*N/G, (c+1)*N/G)).  A unit cut by a
+// range boundary is done in parts, one per CTA; each part leaves its partial
+// softmax state (the unnormalised O rows, the running maximum and the row sum
+// of every query) in a slot of its CTA, and the CTA holding the unit's first
+// tile leaves a record of it.  Once the launch is complete a second, small
+// grid merges every recorded unit, so nothing in the attention grid waits
+// for, or counts, other CTAs.
+
+struct WorkRange {
+    int rr_units;            // units taken whole, round-robin (all, or none)
+    int u_first, j_first;    // first unit and tile of this CTA's range (split)
+    int n_tiles;             // tiles in the range (0: none)
+    int u_last;              // last unit the range touches
+    long long x_first;       // index of the range's first tile
+    long long n_tail;        // tiles shared out by the split
+};
+
+// First tail tile of CTA c, and the CTA holding tail tile x.
+PPD_DEV long long split_start(int c, long long N, int G) { return (long long)c * N / G; }
+PPD_DEV int split_cta_of(long long x, long long N, int G) { return (int)(((x + 1) * G + N - 1) / N) - 1; }
+
+// This CTA's work, computed by one whole warp (every lane gets the result).
+// The tiles of one layer's block of sequence b number H * n_qb * (n_pref(b) +
+// n_tt); lanes hold sequences b = lane and lane + 32.
+PPD_DEV WorkRange plan_range(const AttnParams &p, int lane)
+{
+    WorkRange w{};
+    const int G = (int)gridDim.x, c = (int)blockIdx.x;
+    // no tail range unless one is found below
+    w.u_first = p.n_units;
+    w.u_last = -1;
+    w.n_tiles = 0;
+    w.rr_units = p.split ? 0 : p.n_units;   // units taken whole, round-robin
+    if (!p.split) return w;
+    const unsigned full = 0xffffffffu;
+    const int per_b = p.H * p.n_qb;
+    auto nt_of = [&](int b) {
+        const int P = min(max(__ldg(p.prefix_len + b), 0), p.S_max);
+        return ((P + 127) >> 7) + p.n_tt;
+    };
+    const int w0 = lane < p.B ? per_b * nt_of(lane) : 0;
+    const int w1 = lane + 32 < p.B ? per_b * nt_of(lane + 32) : 0;
+    int s0 = w0, s1 = w1;   // inclusive prefix sums over b
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int a = __shfl_up_sync(full, s0, o);
+        const int x = __shfl_up_sync(full, s1, o);
+        if (lane >= o) {
+            s0 += a;
+            s1 += x;
+        }
+    }
+    s1 += __shfl_sync(full, s0, 31);
+    const long long per_layer = __shfl_sync(full, s1, 31);
+    const long long N = per_layer * p.L;
+    // global tile index of unit u's tile 0
+    auto origin = [&](int u) {
+        const int l = u / (p.B * per_b);
+        const int rem = u - l * p.B * per_b;
+        const int b = rem / per_b, idx = rem - b * per_b;
+        const int incl = b < 32 ? __shfl_sync(full, s0, b & 31) : __shfl_sync(full, s1, b & 31);
+        const int wt = b < 32 ? __shfl_sync(full, w0, b & 31) : __shfl_sync(full, w1, b & 31);
+        return (long long)l * per_layer + (incl - wt) + (long long)idx * (wt / per_b);
+    };
+    // unit and tile of global tile x (0 <= x < N)
+    auto locate = [&](long long x, int &u, int &j) {
+        const int l = (int)(x / per_layer);
+        const int r = (int)(x - (long long)l * per_layer);
+        const unsigned m0 = __ballot_sync(full, lane < p.B && s0 > r);
+        int b, incl, wt;
+        if (m0) {
+            b = __ffs(m0) - 1;
+            incl = __shfl_sync(full, s0, b);
+            wt = __shfl_sync(full, w0, b);
+        } else {
+            const unsigned m1 = __ballot_sync(full, lane + 32 < p.B && s1 > r);
+            const int bl = m1 ? __ffs(m1) - 1 : 0;
+            b = bl + 32;
+            incl = __shfl_sync(full, s1, bl);
+            wt = __shfl_sync(full, w1, bl);
+        }
+        const int rb = r - (incl - wt);   // tile offset within the block of sequence b
+        const int nt = wt / per_b;
+        const int idx = rb / nt;
+        j = rb - idx * nt;
+        u = (l * p.B + b) * per_b + idx;
+    };
+    const long long base = origin(w.rr_units);
+    w.n_tail = N - base;
+    const long long gs = split_start(c, w.n_tail, G), ge = split_start(c + 1, w.n_tail, G);
+    w.x_first = gs;
+    w.n_tiles = (int)(ge - gs);
+    if (ge > gs) {
+        int jl;
+        locate(base + gs, w.u_first, w.j_first);
+        locate(base + ge - 1, w.u_last, jl);
+    }
+    return w;
+}
+
+// One stretch of a unit's tiles [j0, j1) processed by this CTA.
+struct Seg {
+    UnitInfo ui;
+    int u, j0, j1;
+};
+
+// Walks this CTA's segments in order (every role of the CTA walks the same
+// sequence): whole units round-robin, or (SPLIT) its range of tiles, `left`
+// counting the range's tiles not yet handed out.
+template <bool SPLIT>
+struct SegIter {
+    int u, j0, left;
+    PPD_DEV explicit SegIter(const WorkRange &w)
+    {
+        u = SPLIT ? w.u_first : (int)blockIdx.x;
+        j0 = SPLIT ? w.j_first : 0;
+        left = SPLIT ? w.n_tiles : 0;
+    }
+    PPD_DEV bool next(const AttnParams &p, Seg &s)
+    {
+        if (!SPLIT) {
+            if (u >= p.n_units) return false;
+            s.ui = unit_info(p, u);
+            s.u = u;
+            s.j0 = 0;
+            s.j1 = s.ui.n_tiles;
+            u += (int)gridDim.x;
+            return true;
+        }
+        if (left <= 0 || u >= p.n_units) return false;
+        s.ui = unit_info(p, u);
+        s.u = u;
+        s.j0 = j0;
+        s.j1 = min(s.ui.n_tiles, j0 + left);
+        if (s.j1 <= j0) {   // cannot happen with a consistent plan; never loop on it
+            left = 0;
+            return false;
+        }
+        left -= s.j1 - j0;
+        ++u;
+        j0 = 0;
+        return true;
+    }
+};
+
+// Does the CTA process all of the segment's unit?
+PPD_DEV bool seg_whole(const Seg &s) { return s.j0 == 0 && s.j1 == s.ui.n_tiles; }
+
+// Tail-relative index of the segment's unit's tile 0, given the iterator
+// right after it handed the (tail) segment out.
+template <bool SPLIT>
+PPD_DEV long long seg_unit_origin(const WorkRange &w, const SegIter<SPLIT> &it, const Seg &s)
+{
+    return w.x_first + (w.n_tiles - it.left) - s.j1;
+}
+
+// The parts of a cut unit: the CTAs c_a..c_b whose ranges are not empty (a
+// launch with fewer tiles than CTAs leaves some ranges empty).  Part c's slot
+// is 2c for the first segment of its range and 2c + 1 for the last (only c_a
+// can hold the unit in its last segment).
+struct SplitParts {
+    int c_a, c_b, slot_a, n_parts;
+};
+
+PPD_DEV bool split_nonempty(int c, long long N, int G) { return split_start(c + 1, N, G) > split_start(c, N, G); }
+
+PPD_DEV SplitParts split_parts(long long N, long long off, int n_tiles)
+{
+    SplitParts sp;
+    const int G = (int)gridDim.x;
+    sp.c_a = split_cta_of(off, N, G);
+    sp.c_b = split_cta_of(off + n_tiles - 1, N, G);
+    sp.slot_a = 2 * sp.c_a + (split_start(sp.c_a, N, G) < off ? 1 : 0);
+    sp.n_parts = 0;
+    for (int c = sp.c_a; c <= sp.c_b; ++c) sp.n_parts += split_nonempty(c, N, G) ? 1 : 0;
+    return sp;
+}
+
+PPD_DEV int split_slot(const SplitParts &sp, int c) { return c == sp.c_a ? sp.slot_a : 2 * c; }
+
+// Floats of one partial-state slot: kSplitRows rows of D, their maxima, their sums.
+PPD_DEV size_t split_slot_floats(int D) { return (size_t)kSplitRows * (D + 2); }
+
+// Merge the partial states of a cut unit whose parts have all arrived: slot
+// row r (output row out_row0 + r), columns [c0, c0 + 8), by one thread.  One
+// pass over the parts with a running maximum M: part c enters with weight
+// 2^(m_c - M), earlier sums are rescaled when M grows; the output is the
+// weighted sum of the parts' O rows over the weighted sum of their row sums.
+// The parts are read eight at a time, every load of a batch issued before any
+// is used, so a batch costs one round trip to L2.
+static __device__ __forceinline__ void split_merge_chunk(const float *split_part, float *out, float *lse,
+                                                         const SplitParts &sp, long long N, int G,
+                                                         size_t out_row0, int r, int c0, int D)
+{
+    constexpr int PB = 8;   // parts per batch
+    const size_t sf = split_slot_floats(D);
+    const bool dense = N >= G;   // no empty ranges
+    float M = -INFINITY, Ls = 0.f;
+    float acc[8];
+#pragma unroll
+    for (int x = 0; x < 8; ++x) acc[x] = 0.f;
+    for (int cb = sp.c_a; cb <= sp.c_b; cb += PB) {
+        float mc[PB], lc[PB];
+        float4 v[PB][2];
+#pragma unroll
+        for (int y = 0; y < PB; ++y) {
+            const int c = cb + y;
+            const bool live = c <= sp.c_b && (dense || split_nonempty(c, N, G));
+            const float *b_ = split_part + (size_t)split_slot(sp, live ? c : sp.c_a) * sf;
+            mc[y] = live ? __ldcg(b_ + (size_t)kSplitRows * D + r) : -INFINITY;
+            lc[y] = live ? __ldcg(b_ + (size_t)kSplitRows * D + kSplitRows + r) : 0.f;
+            const float4 *o4 = reinterpret_cast<const float4 *>(b_ + (size_t)r * D + c0);
+            v[y][0] = live ? __ldcg(o4) : make_float4(0.f, 0.f, 0.f, 0.f);
+            v[y][1] = live ? __ldcg(o4 + 1) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int y = 0; y < PB; ++y) {
+            if (mc[y] == -INFINITY) continue;   // absent, or the part saw no key of this row
+            const float Mn = fmaxf(M, mc[y]);
+            const float so = ex2(M - Mn);       // 0 while M = -inf
+            const float w = ex2(mc[y] - Mn);
+            Ls = fmaf(Ls, so, w * lc[y]);
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                acc[4 * x] = fmaf(acc[4 * x], so, w * v[y][x].x);
+                acc[4 * x + 1] = fmaf(acc[4 * x + 1], so, w * v[y][x].y);
+                acc[4 * x + 2] = fmaf(acc[4 * x + 2], so, w * v[y][x].z);
+                acc[4 * x + 3] = fmaf(acc[4 * x + 3], so, w * v[y][x].w);
+            }
+            M = Mn;
+        }
+    }
+    const float inv = 1.f / Ls;
+    float *dst = out + (out_row0 + r) * D + c0;
+    if ((reinterpret_cast<uintptr_t>(out) & 15u) == 0) {
+        reinterpret_cast<float4 *>(dst)[0] = make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
+        reinterpret_cast<float4 *>(dst)[1] = make_float4(acc[4] * inv, acc[5] * inv, acc[6] * inv, acc[7] * inv);
+    } else {
+#pragma unroll
+        for (int x = 0; x < 8; ++x) dst[x] = acc[x] * inv;
+    }
+    if (c0 == 0 && lse) lse[out_row0 + r] = (M + lg2(Ls)) * 0.69314718055994530942f;
 }
 
 PPD_DEV void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
@@ -67,9 +318,18 @@ enum : int { kMaskNone = 0, kMaskRows = 1, kMaskTree = 2 };
 // (layer, sequence, head) slices into the cache.  Attention only reads cache
 // rows below each prefix, so the copies never race with it.  Scratch (parent
 // copies, top-1 tokens, path) lives in a per-CTA slice of the workspace.
-PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
+PPD_DEV void fused_side_warp(const AttnParams &p, const WorkRange &wr, int lane)
 {
     asm volatile("griddepcontrol.wait;" ::: "memory");
+    // the units whose first tile this CTA streams (its round-robin units and the
+    // tail units starting in its range) compact their slices here
+    const int t_lo = wr.u_first + (wr.j_first > 0 ? 1 : 0), t_hi = wr.n_tiles > 0 ? wr.u_last : -1;
+    auto owns_first_tile = [&](auto f) {
+        for (int u = (int)blockIdx.x; u < wr.rr_units; u += (int)gridDim.x)
+            if (f(u)) return;
+        for (int u = t_lo; u <= t_hi; ++u)
+            if (f(u)) return;
+    };
     const FusedStep &f = p.fs;
     const int T = p.T, B = p.B, S = f.splits;
     int *s_par = f.scratch + (size_t)blockIdx.x * kSideScratchInts;
@@ -81,8 +341,10 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
     for (int b = 0; b < B; ++b) {
         const bool designated = (b % (int)gridDim.x) == (int)blockIdx.x;
         bool has_unit = false;
-        for (int u = blockIdx.x; u < p.n_units && !has_unit; u += gridDim.x)
+        owns_first_tile([&](int u) {
             has_unit = ((u / p.n_qb / p.H) % B) == b && u % p.n_qb == 0;
+            return has_unit;
+        });
         if (!designated && !has_unit) continue;
         for (int r = lane; r < T; r += 32) {
             const size_t base = ((size_t)b * T + r) * S;
@@ -118,10 +380,10 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
             // cache rows [P_b, P_b + n_acc) <- the accepted tree rows
             const int P = __ldg(p.prefix_len + b);
             const int n = res.n_acc;
-            // each slice once: by the CTA holding its first query block
-            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
+            // each slice once: by the CTA holding the first tile of its first query block
+            owns_first_tile([&](int u) {
                 const int lbh = u / p.n_qb;
-                if (u % p.n_qb != 0 || ((lbh / p.H) % B) != b) continue;
+                if (u % p.n_qb != 0 || ((lbh / p.H) % B) != b) return false;
                 for (int w = lane; w < n * chunks; w += 32) {
                     const int j = w / chunks, c = w - j * chunks;
                     const int src = path[j];
@@ -132,15 +394,18 @@ PPD_DEV void fused_side_warp(const AttnParams &p, int lane)
                     *reinterpret_cast<uint4 *>(f.k_cache + dof) = kx;
                     *reinterpret_cast<uint4 *>(f.v_cache + dof) = vx;
                 }
-            }
+                return false;
+            });
         }
         __syncwarp();
     }
 }
 
 // Launch one of the persistent attention kernels: one CTA per SM (at most one
-// per unit) of `threads` threads, `smem` bytes of dynamic shared memory, with programmatic stream
-// serialization when asked.  The shared-memory opt-in is set once per device.
+// per unit, or with the work split at most one per tile and kSplitMaxGrid) of
+// `threads` threads, `smem` bytes of dynamic shared memory, with programmatic
+// stream serialization when asked.  The shared-memory opt-in is set once per
+// device.
 template <class Kern>
 cudaError_t launch_attention_grid(Kern kern, uint32_t smem, int threads,
                                   std::atomic<uint64_t> &configured,
@@ -157,7 +422,7 @@ cudaError_t launch_attention_grid(Kern kern, uint32_t smem, int threads,
         configured.fetch_or(bit, std::memory_order_acq_rel);
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(p.n_units < num_sms ? p.n_units : num_sms));
+    cfg.gridDim = dim3((unsigned)attention_grid(p, num_sms));
     cfg.blockDim = dim3((unsigned)threads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;

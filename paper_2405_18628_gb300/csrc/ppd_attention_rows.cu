@@ -25,8 +25,9 @@
 // products and the next S product queue in the tensor pipe; the single O
 // accumulator of a finished unit is read back after the next unit's first
 // tile, and that unit's first PV product waits for the readback.  The unit
-// walk and the fused step's side warp are those of the kernel for trees of up
-// to 64 tokens (ppd_attention.cu); the warp roles (384 threads) differ in one
+// walk (with the work split), the fused step's side warp and the merge of a
+// cut unit's partial states are those of the kernel for trees of up to 64
+// tokens (ppd_attention.cu); the warp roles (384 threads) differ in one
 // point: warp 8 loads Q and K, warp 11 loads V.
 #include "ppd_attention_common.cuh"
 
@@ -70,7 +71,8 @@ struct RowsLayout {
     static constexpr uint32_t OFF_ABORT = OFF_TMEMPTR + 4;
     static constexpr uint32_t OFF_XM = (OFF_ABORT + 4 + 15) & ~15u;   // [2][M] partial row maxima
     static constexpr uint32_t OFF_XL = OFF_XM + 2 * M * 4;            // [2][M] partial row sums
-    static constexpr uint32_t SMEM_BYTES = OFF_XL + 2 * M * 4;
+    static constexpr uint32_t OFF_RANGE = OFF_XL + 2 * M * 4;        // WorkRange
+    static constexpr uint32_t SMEM_BYTES = OFF_RANGE + ((sizeof(WorkRange) + 15) & ~15u);
     // TMEM columns: S0 | S1 | S2 (128 each; P is written over S) | O (D)
     static constexpr uint32_t T_S = 0, T_O = NSB * 128, TMEM_COLS = 512;
     static_assert(NSB * 128 + D <= 512, "TMEM budget");
@@ -79,7 +81,7 @@ struct RowsLayout {
     static_assert((OFF_K | OFF_V | Q_BYTES) % 1024 == 0, "1024-byte aligned operand tiles");
 };
 
-template <int D>
+template <int D, bool SPLIT>
 __global__ void __launch_bounds__(384, 1)
 tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                            const __grid_constant__ CUtensorMap map_kc,
@@ -116,14 +118,26 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
         tmem_alloc(tmem_ptr, Lay::TMEM_COLS);
         tmem_relinquish();
     }
+    WorkRange *wr_s = reinterpret_cast<WorkRange *>(smem + Lay::OFF_RANGE);
+    if (warp == 8) {
+        const WorkRange w = plan_range(p, lane);   // whole units round-robin without p.split
+        if (lane == 0) {
+            *wr_s = w;
+            if (SPLIT) p.split_rec[blockIdx.x].u = -1;   // no cut unit recorded yet
+        }
+    }
+    // the merge of cut units (a dependent launch) may be scheduled now; it waits
+    // for this grid to complete
+    if (SPLIT) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_ptr;
+    const WorkRange &wr = *wr_s;
 
     if (warp == 10) {
         // ------------------------------------------------------------ fused-step side work
-        if (p.fused) fused_side_warp(p, lane);
+        if (p.fused) fused_side_warp(p, wr, lane);
     } else if (warp == 8 || warp == 11) {
         // ------------------------------------------------------------ TMA producers
         // warp 8 loads Q and the K tiles, warp 11 the V tiles: a V slot is released
@@ -140,8 +154,9 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             }
             const uint64_t pol = l2_policy_evict_first();
             int g = 0, k = 0;
-            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
-                const UnitInfo ui = unit_info(p, u);
+            SegIter<SPLIT> it(wr);
+            for (Seg sg; it.next(p, sg); ++k) {
+                const UnitInfo &ui = sg.ui;
                 const int qs = k % Lay::QS;
                 if (kq) {
                     if (k >= Lay::QS)
@@ -156,7 +171,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                                         ui.lbh, pol);
                     }
                 }
-                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                for (int j = sg.j0; j < sg.j1; ++j, ++g) {
                     const bool tree = (j >= ui.n_pref);
                     const int row = (tree ? j - ui.n_pref : j) * Lay::KT;
                     if (kq) {
@@ -244,11 +259,11 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             int g = 0, k = 0;
             int lag_g[2] = {-1, -1}, lag_k[2] = {0, 0};   // tiles g-2 and g-1 awaiting PV
             bool lag_first[2] = {false, false};
-            for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
-                const UnitInfo ui = unit_info(p, u);
+            SegIter<SPLIT> it(wr);
+            for (Seg sg; it.next(p, sg); ++k) {
                 const int qs = k % Lay::QS;
                 mbar_wait(bars + Lay::B_QFULL + qs, (k / Lay::QS) & 1, abort_flag);
-                for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+                for (int j = sg.j0; j < sg.j1; ++j, ++g) {
                     const int ks = g % Lay::KS;
                     const int sb = g % Lay::NSB;
                     mbar_wait(bars + Lay::B_KFULL + ks, (g / Lay::KS) & 1, abort_flag);
@@ -269,13 +284,13 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                     }
                     umma_commit(bars + Lay::B_SFULL + sb);
                     umma_commit(bars + Lay::B_KEMPTY + ks);
-                    if (j == ui.n_tiles - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
+                    if (j == sg.j1 - 1) umma_commit(bars + Lay::B_QEMPTY + qs);
                     if (lag_g[0] >= 0) issue_pv(lag_g[0], lag_first[0], lag_k[0]);
                     lag_g[0] = lag_g[1];
                     lag_first[0] = lag_first[1];
                     lag_k[0] = lag_k[1];
                     lag_g[1] = g;
-                    lag_first[1] = (j == 0);
+                    lag_first[1] = (j == sg.j0);
                     lag_k[1] = k;
                 }
             }
@@ -301,9 +316,13 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
         uint64_t tmask = 0;
         int cur_key = -1;
         int g = 0;
-        bool pend = false;      // a finished unit whose output still sits in TMEM
-        int pend_lbh = 0, pend_qb = 0, pend_g = 0;
-        float pend_linv = 0.f;
+        // a finished segment whose output still sits in TMEM; a partial one (a
+        // unit cut by the work split) goes to its slot instead of the output
+        // pend_f: bit 0 a segment is pending, bit 1 it is partial, bit 2 it was
+        // the range's first segment; pend_m, pend_l its row's maximum and sum
+        int pend_f = 0, pend_u = 0, pend_g = 0;
+        float pend_m = 0.f, pend_l = 0.f;
+
 
         // Probabilities of this thread's 64 keys from its raw scores s against the
         // maximum mx (exponents clamped at 64), split into bf16 hi + lo and stored
@@ -391,9 +410,51 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             if (lane == 0) mbar_arrive(bars + Lay::B_OFREE);
         };
 
+        // Partial state of a cut unit into slot `slot`: this thread's half of the
+        // row of O unnormalised, and (h == 0) the row's maximum and sum; then O
+        // is free.
+        const size_t slot_floats = split_slot_floats(D);
+        auto write_partial = [&](int slot, int qb_out, int g_last, float rm, float rl) {
+            mbar_wait(bars + Lay::B_PDONE + g_last % Lay::NSB, (g_last / Lay::NSB) & 1, abort_flag);
+            tc_fence_after();
+            const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)h * (D / 2);
+            float *base = p.split_part + (size_t)slot * slot_floats;
+            float *orow = base + (size_t)q * D + h * (D / 2);
+            const bool live = qb_out * Lay::M + q < T;
+#pragma unroll
+            for (int ch = 0; ch < D / 32; ++ch) {
+                uint32_t r[16];
+                tmem_ld16(t_o + ch * 16, r);
+                tmem_wait_ld();
+                if (live) {
+#pragma unroll
+                    for (int e = 0; e < 16; e += 4)
+                        *reinterpret_cast<float4 *>(orow + ch * 16 + e) =
+                            make_float4(__uint_as_float(r[e]), __uint_as_float(r[e + 1]),
+                                        __uint_as_float(r[e + 2]), __uint_as_float(r[e + 3]));
+                }
+            }
+            if (h == 0 && live) {
+                base[(size_t)kSplitRows * D + q] = rm;
+                base[(size_t)kSplitRows * D + kSplitRows + q] = rl;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bars + Lay::B_OFREE);
+        };
+
+        // The pending segment: a whole unit's output, or a part's state (counted
+        // in at the end of the range).
+        auto flush_pending = [&]() {
+            const int lbh_o = pend_u / p.n_qb, qb_o = pend_u - lbh_o * p.n_qb;
+            if (!SPLIT || !(pend_f & 2)) read_back(lbh_o, qb_o, pend_g, rcp(pend_l));
+            else write_partial(2 * (int)blockIdx.x + ((pend_f & 4) ? 0 : 1), qb_o, pend_g, pend_m, pend_l);
+        };
+
         int k = 0;
-        for (int u = blockIdx.x; u < p.n_units; u += gridDim.x, ++k) {
-            const UnitInfo ui = unit_info(p, u);
+        SegIter<SPLIT> it(wr);
+        for (Seg sg; it.next(p, sg); ++k) {
+            const UnitInfo &ui = sg.ui;
             const int qg = ui.qb * Lay::M + q;   // this thread's tree token
             if (ui.b * p.n_qb + ui.qb != cur_key) {
                 // ancestors of node qg among tree nodes 128t + [64h, 64h + 64)
@@ -426,7 +487,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 cur_key = ui.b * p.n_qb + ui.qb;
             }
 
-            for (int j = 0; j < ui.n_tiles; ++j, ++g) {
+            for (int j = sg.j0; j < sg.j1; ++j, ++g) {
                 const bool tree = (j >= ui.n_pref);
                 const int n_valid = tree ? T : min(Lay::KT, ui.P - j * Lay::KT);
                 if (tree) {
@@ -446,7 +507,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 tmem_wait_ld();
 
                 float lt = 0.f;
-                bool exact = (j == 0);
+                bool exact = (j == sg.j0);
                 if (!exact) {
                     // optimistic pass against the current maximum
                     float maxd = -INFINITY;
@@ -464,7 +525,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                     named_bar_sync(1, 256);
                     const float mn = fmaxf(m, fmaxf(xm[q], xm[Lay::M + q]));
                     const float alpha = (mn == m) ? 1.f : ex2(m - mn);
-                    if (j > 0) {
+                    if (j > sg.j0) {
                         if (__any_sync(0xffffffffu, alpha != 1.f)) {
                             // rescale this thread's half of the row of O once the PV
                             // product of the previous tile has landed
@@ -513,30 +574,37 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bars + Lay::B_PFULL + sb);
 
-                // the previous unit's output, once this unit's first tile is on its way
-                if (j == 0 && pend) {
-                    read_back(pend_lbh, pend_qb, pend_g, pend_linv);
-                    pend = false;
+                // the previous segment's output, once this segment's first tile is on its way
+                if (j == sg.j0 && pend_f) {
+                    flush_pending();
+                    pend_f = 0;
                 }
 
-                if (j == ui.n_tiles - 1) {
-                    // ------------------------------------------ unit end: row sum, LSE
+                if (j == sg.j1 - 1) {
+                    // ------------------------------------------ segment end: row sum, LSE
                     xl[h * Lay::M + q] = l;
                     named_bar_sync(1, 256);
                     const float L = xl[q] + xl[Lay::M + q];
-                    if (h == 0 && qg < T && p.lse)
+                    if ((!SPLIT || seg_whole(sg)) && h == 0 && qg < T && p.lse)
                         p.lse[(size_t)ui.lbh * T + qg] = (m + lg2(L)) * 0.69314718055994530942f;
-                    pend = true;
-                    pend_lbh = ui.lbh;
-                    pend_qb = ui.qb;
+                    pend_u = sg.u;
                     pend_g = g;
-                    pend_linv = rcp(L);
+                    pend_m = m;
+                    pend_l = L;
+                    pend_f = 1;
+                    if (SPLIT && !seg_whole(sg)) {
+                        // a part: slot 2c for the tail range's first segment, 2c + 1 for its last
+                        pend_f |= 2 | (sg.u == wr.u_first ? 4 : 0);
+                        // the part holding the unit's first tile records it for the merge
+                        if (sg.j0 == 0 && threadIdx.x == 0)
+                            p.split_rec[blockIdx.x] = SplitRecord{seg_unit_origin(wr, it, sg), wr.n_tail, sg.u, ui.n_tiles};
+                    }
                     m = -INFINITY;
                     l = 0.f;
                 }
             }
         }
-        if (pend) read_back(pend_lbh, pend_qb, pend_g, pend_linv);
+        if (pend_f) flush_pending();
     }
 
     tc_fence_before();
@@ -555,9 +623,12 @@ template <int D>
 static cudaError_t launch_rows_t(const AttnMaps &m, const AttnParams &p, int num_sms,
                                  bool programmatic, cudaStream_t stream)
 {
-    static std::atomic<uint64_t> configured{0};
-    return launch_attention_grid(tree_attention_rows_kernel<D>, RowsLayout<D>::SMEM_BYTES, 384,
-                                 configured, m, p, num_sms, programmatic, stream);
+    static std::atomic<uint64_t> configured[2] = {{0}, {0}};
+    if (p.split)
+        return launch_attention_grid(tree_attention_rows_kernel<D, true>, RowsLayout<D>::SMEM_BYTES, 384,
+                                     configured[1], m, p, num_sms, programmatic, stream);
+    return launch_attention_grid(tree_attention_rows_kernel<D, false>, RowsLayout<D>::SMEM_BYTES, 384,
+                                 configured[0], m, p, num_sms, programmatic, stream);
 }
 
 cudaError_t launch_tree_attention_rows(const AttnMaps &m, const AttnParams &p, int D, int num_sms,

@@ -61,9 +61,49 @@ struct AttnParams {
     int n_qb;                   // query blocks of 128 per (layer, sequence, head) slice
     int n_tt;                   // tree-key tiles of 128 per slice
     float scale_log2;           // softmax scale * log2(e)
+    // Work split: split != 0 shares the units left after the full round-robin
+    // rounds out by their key tiles (B <= kSplitMaxB); units cut by a range
+    // boundary leave partial softmax states in split_part, merged afterwards by
+    // launch_split_merge from the per-CTA records in split_rec.
+    int split;
+    float *split_part;          // [2 * grid][kSplitRows * (D + 2)] partial states
+    struct SplitRecord *split_rec;   // [grid]
     int fused;                  // run the end phase below
     FusedStep fs;
 };
+
+// Work split limits: batch size (the per-CTA range search holds the batch in
+// two warp-wide registers), CTAs, and query rows of a partial state.
+constexpr int kSplitMaxB = 64;
+constexpr int kSplitMaxGrid = 256;
+constexpr int kSplitRows = 128;
+
+// The unit a CTA has to have merged: it holds the unit's first tile and its
+// range ends inside the unit (u = -1: none).  off: the unit's tile 0 among
+// the tail's tiles; n_tail: the tail's tile count.
+struct SplitRecord {
+    long long off, n_tail;
+    int u, n_tiles;
+};
+
+// CTAs of an attention launch: one per SM, at most one per unit (with the
+// work split: at most one per tile, and kSplitMaxGrid).
+inline int attention_grid(const AttnParams &p, int num_sms)
+{
+    long long grid = num_sms;
+    if (p.split) {
+        const long long max_tiles = (long long)p.n_units * ((p.S_max + 127) / 128 + p.n_tt);
+        grid = grid < kSplitMaxGrid ? grid : kSplitMaxGrid;
+        grid = grid < max_tiles ? grid : max_tiles;
+    } else {
+        grid = grid < p.n_units ? grid : p.n_units;
+    }
+    return (int)grid;
+}
+
+// Merge the partial states of every cut unit of the attention launch just
+// enqueued (one CTA per attention CTA, `grid` of them), after it completes.
+cudaError_t launch_split_merge(const AttnParams &p, int D, int grid, cudaStream_t stream);
 
 // Batches up to this size run the fused two-grid step.
 constexpr int kFusedMaxB = 64;
