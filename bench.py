@@ -48,10 +48,10 @@ L2_BYTES = 129 * 1000 * 1000
 # same shapes with 19 layers (608 / 760 units: whole rounds of 152 CTAs) and
 # are scaled to the full layer count, since traffic grows with the units.
 MEASURED_TRAFFIC = {
-    # 675,516,672 B at 19 layers x 32/19
-    "vicuna7b": {"bytes_per_launch": 1_137_712_289, "src": "9eeadeae524caf7d"},
-    # 1,659,153,664 B at 19 layers x 40/19
-    "vicuna13b": {"bytes_per_launch": 3_492_955_082, "src": "9eeadeae524caf7d"},
+    # 675,317,760 B at 19 layers x 32/19
+    "vicuna7b": {"bytes_per_launch": 1_137_377_280, "src": "5160a2839377052c"},
+    # 1,659,191,040 B at 19 layers x 40/19
+    "vicuna13b": {"bytes_per_launch": 3_493_033_768, "src": "5160a2839377052c"},
 }
 
 
