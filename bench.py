@@ -580,7 +580,8 @@ def main():
                          "bytes_per_launch": att_bytes, "peak_kind": peak_kind,
                          "frac_of_8000": achieved / NOMINAL_HBM_GBS},
             "e2e": e2e,
-            "gpu_launches": (2 if w.B <= 64 else 5) * K,
+            "gpu_launches": ppd.ppd_verify_step_launches(
+                w.L, w.B, w.H, w.T, w.D, w.V, w.S_max, typical=args.accept == "typical") * K,
             "clocks": clk,
             "cpu_baseline": cpu,
             "wall_s_timed": wall,

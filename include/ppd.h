@@ -146,16 +146,25 @@ ppd_status ppd_kv_compact(void *k_cache, void *v_cache, const void *k_tree, cons
                           int S_max, ppd_dtype dt, void *stream);
 
 /*
- * The whole verification step: node argmax and acceptance, tree-masked
- * attention over all L layers, and compaction of the accepted rows, enqueued
- * on `stream` with no host synchronisation.  For B <= 64 this is two grids:
- * the argmax partial maxima, then the attention grid (allowed to start while
- * the first still runs), whose end phase combines the argmax, decides
- * acceptance and compacts; larger batches run the steps as separate grids.  Arguments as in the four entry
- * points above; `out`/`lse` as in ppd_tree_attention, `argmax_out` as in
- * ppd_node_argmax.  Attention reads only prefix rows [0, prefix_len[b]) and
- * compaction writes only rows [prefix_len[b], new_prefix_len[b]), so the
- * result equals running the four steps one after another.
+ * The whole verification step (Section 3 steps (1)-(3)): node argmax and
+ * acceptance, tree-masked attention over all L layers, and compaction of the
+ * accepted rows, enqueued on `stream` with no host synchronisation.  For
+ * B <= 64 the attention grid does the other steps with one spare warp per CTA
+ * while its other warps stream K/V: that warp combines the argmax, decides
+ * acceptance and compacts.  When the logits are at most 1/64 of the K/V bytes
+ * (counted over S_max + T rows), those warps also compute the argmax partial
+ * maxima themselves and the step is a single cooperative grid (the CTAs
+ * exchange flags in the workspace, tagged with a per-call epoch that the
+ * workspace also holds, so its contents still do not matter); otherwise an
+ * argmax grid runs first and the attention grid may start while it runs.
+ * If the cooperative launch cannot have every CTA resident, the step falls
+ * back to the two-grid form.  Larger batches run the steps as separate grids.
+ * Arguments as in the four entry points above; `out`/`lse` as in
+ * ppd_tree_attention, `argmax_out` as in ppd_node_argmax.  Attention reads
+ * only prefix rows [0, prefix_len[b]) and compaction writes only rows
+ * [prefix_len[b], new_prefix_len[b]), so the result equals running the four
+ * steps one after another.  After a call that reported PPD_ERR_TIMEOUT, fill
+ * the workspace with zeros before reusing it.
  */
 ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
                            const void *k_tree, const void *v_tree,
@@ -282,6 +291,16 @@ ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32
  */
 ppd_status ppd_node_argmax_noalloc(const float *logits, int B, int T, int V, int32_t *argmax_out,
                                    void *stream);
+
+/*
+ * Kernel launches one ppd_verify_step call (typical == 0) or
+ * ppd_verify_step_typical call (typical != 0) enqueues for these sizes, with
+ * a workspace of ppd_workspace_bytes(...) bytes and the whole GPU available.
+ * No paper counterpart: it lets a caller or benchmark count the kernels of a
+ * step without a profiler.  Returns -1 for sizes the step rejects.
+ */
+int ppd_verify_step_launches(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt,
+                             int typical);
 
 /* Human-readable name of a status code (static string). */
 const char *ppd_status_string(ppd_status s);

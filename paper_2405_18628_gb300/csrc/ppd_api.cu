@@ -52,12 +52,40 @@ int argmax_splits(int64_t rows, int V) { return ppd::argmax_split_count(rows, V)
 // Workspace: the argmax partials, the side warp's scratch, the bf16 copies of
 // fp32 operands, then the work split's per-CTA records and partial states.
 struct WsLayout {
-    size_t part_val, part_idx, part_stats, node_lse, node_ent, side, conv, split_rec, split_part,
-        total;
+    size_t part_val, part_idx, part_stats, node_lse, node_ent, side, sync, conv, split_rec,
+        split_part, total;
     int splits;
 };
 
 int split_grid() { return num_sms() < ppd::kSplitMaxGrid ? num_sms() : ppd::kSplitMaxGrid; }
+
+// Logits per (row, split) chunk of the argmax (a multiple of 4), and whether
+// the rows can be read with 16-byte loads; as launch_argmax_partials does.
+int argmax_chunk(int V, int splits) { return (((V + splits - 1) / splits) + 3) & ~3; }
+int argmax_vec(const float *logits, int V)
+{
+    return (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
+}
+
+// The fused step computes the node argmax inside the attention grid (one
+// side warp per CTA, while the other warps stream K/V) when the logits are a
+// small share of the bytes the attention streams.  A side warp keeps 2 KB in
+// flight (deeper bursts slow the attention more than they gain) and, with the
+// HBM saturated by the K/V stream, reads about 1 GB/s against its CTA's
+// ~42 GB/s of K/V.  Measured at Vicuna-7B shapes with a growing vocabulary:
+// in-grid beats the two-grid form while the logits are at most 1/70 of the
+// K/V bytes, and the side warps become the bottleneck at 1/35.  Otherwise a
+// separate argmax grid runs first.  S_max bounds the prefix lengths, which
+// only the device knows.
+#ifndef PPD_IN_GRID_MIN_RATIO
+#define PPD_IN_GRID_MIN_RATIO 64
+#endif
+bool in_grid_argmax_pays(int L, int B, int H, int T, int D, int V, int S_max)
+{
+    const double kv = 4.0 * L * B * H * ((double)S_max + T) * D;
+    const double logits = 4.0 * B * (double)T * V;
+    return logits * PPD_IN_GRID_MIN_RATIO <= kv;
+}
 
 WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt)
 {
@@ -77,6 +105,8 @@ WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, p
     off = align_up(off + (size_t)rows * 4);
     w.side = off;
     off = align_up(off + (size_t)num_sms() * ppd::kSideScratchInts * 4);
+    w.sync = off;   // the in-grid argmax's epoch and all-ready words, per-CTA flags
+    off = align_up(off + (size_t)(2 + ppd::kSplitMaxGrid) * 8);
     w.conv = off;
     if (dt == PPD_F32) {
         const size_t lbh = (size_t)L * B * H;
@@ -173,9 +203,23 @@ bool split_pays(const AttnParams &p, int sms)
     return share + kSplitCostTiles < t_u;
 }
 
-// With a workspace of the full layout, a batch of at most kSplitMaxB and a
-// launch that gains from it, the key tiles are shared evenly over the CTAs
-// (see ppd_attention_common.cuh).
+// Whether an attention launch of these sizes, given a workspace, shares its key
+// tiles out (the work split): a batch of at most kSplitMaxB and a launch that
+// gains from it.
+bool attention_splits(int L, int B, int H, int T, int S_max)
+{
+    if (B > ppd::kSplitMaxB) return false;
+    AttnParams p{};
+    const int T_pad = (T + 31) & ~31;
+    p.S_max = S_max;
+    p.n_qb = T_pad > 64 ? (T + 127) / 128 : 1;
+    p.n_tt = p.n_qb;
+    p.n_units = (int)((long long)L * B * H) * p.n_qb;
+    return split_pays(p, split_grid());
+}
+
+// With a workspace of the full layout and attention_splits(...), the key tiles
+// are shared evenly over the CTAs (see ppd_attention_common.cuh).
 ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, const void *kt,
                              const void *vt, const int32_t *prefix_len, const int32_t *parent,
                              int L, int B, int H, int T, int D, int S_max, float scale, float *out,
@@ -211,7 +255,7 @@ ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, cons
     p.n_units = (int)lbh * p.n_qb;
     const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
     p.scale_log2 = sc * 1.4426950408889634f;
-    if (ws && wl && B <= ppd::kSplitMaxB && split_pays(p, split_grid())) {
+    if (ws && wl && attention_splits(L, B, H, T, S_max)) {
         p.split = 1;
         p.split_rec = reinterpret_cast<ppd::SplitRecord *>(ws + wl->split_rec);
         p.split_part = reinterpret_cast<float *>(ws + wl->split_part);
@@ -230,11 +274,11 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
                                  cudaStream_t stream)
 {
     // With bf16 operands the attention grid only reads caller inputs before its end
-    // phase, so it may overlap the preceding (argmax) grid.
+    // phase, so it may overlap the preceding (argmax) grid -- when there is one.
     if (dt == PPD_BF16)
         return enqueue_attention(q, kc, vc, kt, vt, prefix_len, parent, L, B, H, T, D, S_max, scale,
                                  out, lse, dev_status, ws, ws ? &wl : nullptr, fused,
-                                 fused != nullptr, stream);
+                                 fused != nullptr && !fused->in_grid, stream);
     const int64_t lbh = (int64_t)L * B * H;
     const int64_t n_t = lbh * T * D, n_c = lbh * (int64_t)S_max * D;
     uint16_t *bq = reinterpret_cast<uint16_t *>(ws + wl.conv);
@@ -298,40 +342,59 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
     const int64_t rows = (int64_t)B * T;
 
     if (B <= ppd::kFusedMaxB) {
-        // 1. partial maxima (and statistics) of every node's logits; also zeroes dev_status
-        if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temp, dev_status, B,
-                                        s) != cudaSuccess)
-            return PPD_ERR_CUDA;
-        // 2. attention over every layer, overlapping step 1; its end phase combines
-        //    the argmax, decides acceptance and compacts the accepted rows
-        ppd::FusedStep f{};
-        f.part_val = pv;
-        f.part_idx = pi;
-        f.splits = wl.splits;
-        f.cand_tokens = cand_tokens;
-        f.argmax_out = argmax_out;
-        f.accept_len = accept_len;
-        f.path = path;
-        f.next_token = next_token;
-        f.new_prefix_len = new_prefix_len;
-        f.status = dev_status;
-        f.k_cache = static_cast<uint8_t *>(k_cache);
-        f.v_cache = static_cast<uint8_t *>(v_cache);
-        f.k_tree = static_cast<const uint8_t *>(k_tree);
-        f.v_tree = static_cast<const uint8_t *>(v_tree);
-        f.row_bytes = D * eb;
-        f.V = V;
-        f.scratch = reinterpret_cast<int *>(ws + wl.side);
-        if (typ) {
-            f.typical = 1;
-            f.part_stats = pst;
+        bool in_grid = in_grid_argmax_pays(L, B, H, T, D, V, S_max);
+        while (true) {
+            // 1. partial maxima (and statistics) of every node's logits; also zeroes
+            //    dev_status.  In-grid: the attention grid's side warps do this instead.
+            if (!in_grid && ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst,
+                                                        temp, dev_status, B, s) != cudaSuccess)
+                return PPD_ERR_CUDA;
+            // 2. attention over every layer, overlapping step 1; its side warps combine
+            //    the argmax, decide acceptance and compact the accepted rows
+            ppd::FusedStep f{};
+            f.part_val = pv;
+            f.part_idx = pi;
+            f.splits = wl.splits;
+            f.cand_tokens = cand_tokens;
+            f.argmax_out = argmax_out;
+            f.accept_len = accept_len;
+            f.path = path;
+            f.next_token = next_token;
+            f.new_prefix_len = new_prefix_len;
+            f.status = dev_status;
+            f.k_cache = static_cast<uint8_t *>(k_cache);
+            f.v_cache = static_cast<uint8_t *>(v_cache);
+            f.k_tree = static_cast<const uint8_t *>(k_tree);
+            f.v_tree = static_cast<const uint8_t *>(v_tree);
+            f.row_bytes = D * eb;
+            f.V = V;
+            f.scratch = reinterpret_cast<int *>(ws + wl.side);
             f.logits = logits;
-            f.inv_temp = 1.f / typ->temperature;
-            f.epsilon = typ->epsilon;
-            f.delta = typ->delta;
+            if (in_grid) {
+                f.in_grid = 1;
+                f.chunk = argmax_chunk(V, wl.splits);
+                f.vec = argmax_vec(logits, V);
+                f.stat_k = 1.4426950408889634f / temp;
+                f.epoch = reinterpret_cast<unsigned long long *>(ws + wl.sync);
+                f.all_ready = f.epoch + 1;
+                f.ready = f.epoch + 2;
+            }
+            if (typ) {
+                f.typical = 1;
+                f.part_stats = pst;
+                f.inv_temp = 1.f / typ->temperature;
+                f.epsilon = typ->epsilon;
+                f.delta = typ->delta;
+            }
+            const ppd_status st = enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree,
+                                                        prefix_len, parent, L, B, H, T, D, S_max,
+                                                        dt, scale, out, lse, nullptr, ws, wl, &f, s);
+            if (st == PPD_OK || !in_grid) return st;
+            // the cooperative launch could not have every CTA resident (SMs taken by
+            // other work): clear its error and run the argmax as its own grid
+            if (cudaGetLastError() != cudaErrorCooperativeLaunchTooLarge) return st;
+            in_grid = false;
         }
-        return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B,
-                                     H, T, D, S_max, dt, scale, out, lse, nullptr, ws, wl, &f, s);
     }
 
     // large batches: the same steps as separate grids
@@ -359,6 +422,18 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
     if (st != PPD_OK) return st;
     return cuda_status(ppd::launch_kv_compact(k_cache, v_cache, k_tree, v_tree, path, accept_len,
                                               prefix_len, L, B, H, T, D, S_max, eb, s));
+}
+
+int ppd_verify_step_launches(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt,
+                             int typical)
+{
+    (void)typical;   // both acceptance rules launch the same number of kernels
+    if (!attn_dims_ok(L, B, H, T, D, S_max, dt) || V < 1) return -1;
+    const int round = dt == PPD_F32 ? 5 : 0;   // fp32 -> bf16 copies of Q, K/V tree, K/V cache
+    const int attn = attention_splits(L, B, H, T, S_max) ? 2 : 1;   // + the merge grid
+    if (B <= ppd::kFusedMaxB) return (in_grid_argmax_pays(L, B, H, T, D, V, S_max) ? 0 : 1) + round + attn;
+    // partial maxima, combine (or statistics), acceptance, attention, compaction
+    return 3 + round + attn + 1;
 }
 
 static bool typical_params_ok(float temperature, float epsilon, float delta)

@@ -309,28 +309,164 @@ using kind_t = std::integral_constant<int, K>;
 // visible (the last, partial prefix tile), or the tree-ancestor mask.
 enum : int { kMaskNone = 0, kMaskRows = 1, kMaskTree = 2 };
 
-// Side work of the fused verification step, done by one extra warp of every CTA
-// while the other warps stream attention.  Once the preceding argmax grid has
-// completed (griddepcontrol.wait), for every sequence b this CTA touches -- or
-// is designated to report (b mod grid) -- the warp combines the node argmax
-// from the partial maxima, decides acceptance, writes the sequence's outputs
-// if designated, and copies the accepted tree K/V rows of this CTA's own
-// (layer, sequence, head) slices into the cache.  Attention only reads cache
-// rows below each prefix, so the copies never race with it.  Scratch (parent
-// copies, top-1 tokens, path) lives in a per-CTA slice of the workspace.
-PPD_DEV void fused_side_warp(const AttnParams &p, const WorkRange &wr, int lane)
+// One warp's partial top-1 of columns [lo, hi) of the logits row x, and with
+// kStats the softmax statistics of the same columns at scale stat_k; lane 0
+// holds the result.  Four 16-byte loads per lane (2 KB per warp) are in
+// flight at a time: deeper bursts of loads from this warp slow the softmax
+// warps that share its SM sub-partition more than they gain.
+template <bool kStats>
+PPD_DEV void warp_logit_partial(const float *x, int lo, int hi, bool vec, float stat_k, int lane,
+                                float &bv, int &bi, SoftStats &st)
 {
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+    bv = -INFINITY;
+    bi = INT_MAX;
+    st = SoftStats{};
+    auto take4 = [&](const float4 &f, int base) {
+        consider(f.x, base, bv, bi);
+        consider(f.y, base + 1, bv, bi);
+        consider(f.z, base + 2, bv, bi);
+        consider(f.w, base + 3, bv, bi);
+        if (kStats) stats_add4(st, f.x * stat_k, f.y * stat_k, f.z * stat_k, f.w * stat_k);
+    };
+    if (vec) {
+        const float4 *x4 = reinterpret_cast<const float4 *>(x);
+        const int n4_hi = hi >> 2;
+        int i = (lo >> 2) + lane;
+        for (; i + 3 * 32 < n4_hi; i += 4 * 32) {
+            float4 f[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) f[k] = __ldcs(x4 + i + k * 32);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) take4(f[k], 4 * (i + k * 32));
+        }
+        for (; i < n4_hi; i += 32) take4(__ldcs(x4 + i), 4 * i);
+    } else {
+        for (int i = lo + lane; i < hi; i += 32) {
+            const float v = __ldcs(x + i);
+            consider(v, i, bv, bi);
+            if (kStats) stats_add4(st, v * stat_k, -INFINITY, -INFINITY, -INFINITY);
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float ov = __shfl_down_sync(0xffffffffu, bv, off);
+        const int oi = __shfl_down_sync(0xffffffffu, bi, off);
+        consider(ov, oi, bv, bi);
+        if (kStats) {
+            SoftStats o;
+            o.m = __shfl_down_sync(0xffffffffu, st.m, off);
+            o.s = __shfl_down_sync(0xffffffffu, st.s, off);
+            o.t = __shfl_down_sync(0xffffffffu, st.t, off);
+            stats_merge(st, o);
+        }
+    }
+}
+
+// In-grid argmax of the fused step: this CTA's chunks of the [B*T][splits]
+// partial grid (chunk c by CTA c mod grid), then its flag.  Each lane fences
+// its own writes before the warp barrier, so lane 0's release covers them all.
+PPD_DEV void side_argmax_chunks(const AttnParams &p, unsigned long long tag, int lane)
+{
+    const FusedStep &f = p.fs;
+    const int S = f.splits;
+    const long long n_chunks = (long long)p.B * p.T * S;
+    for (long long c = blockIdx.x; c < n_chunks; c += gridDim.x) {
+        const long long row = c / S;
+        const int lo = (int)(c - row * S) * f.chunk;
+        const int hi = min(f.V, lo + f.chunk);
+        const float *x = f.logits + row * (long long)f.V;
+        float bv;
+        int bi;
+        SoftStats st;
+        if (f.typical) warp_logit_partial<true>(x, lo, hi, f.vec != 0, f.stat_k, lane, bv, bi, st);
+        else warp_logit_partial<false>(x, lo, hi, f.vec != 0, 0.f, lane, bv, bi, st);
+        if (lane == 0) {
+            f.part_val[c] = bv;
+            f.part_idx[c] = bi;
+            if (f.typical) {
+                float *ps = f.part_stats + 3 * c;
+                ps[0] = st.m;
+                ps[1] = st.s;
+                ps[2] = st.t;
+            }
+        }
+    }
+    __threadfence();
+    __syncwarp();
+    if (lane == 0) st_release_gpu(f.ready + blockIdx.x, tag);
+}
+
+// Wait until every CTA of the grid has published `tag` (bounded: raises the
+// CTA's abort flag and returns false after kWaitLimitNs, or at once when the
+// flag is already up).  Only CTA 0 reads the per-CTA flags; once all are up
+// it advances the epoch for the next call and publishes `tag` in all_ready,
+// the one word the other CTAs poll (from one lane, with a backoff), so the
+// waits add little to the L2 traffic of the attention stream.
+PPD_DEV bool side_wait_all(const AttnParams &p, unsigned long long tag, int lane,
+                           volatile int *abort_flag)
+{
+    const FusedStep &f = p.fs;
+    const int G = (int)gridDim.x;
+    const uint64_t t0 = global_timer();
+    bool done = false;
+    while (true) {
+        if (blockIdx.x == 0) {
+            bool ok = true;
+            for (int c = lane; c < G; c += 32) ok = ok && ld_acquire_gpu(f.ready + c) == tag;
+            done = __all_sync(0xffffffffu, ok);
+        } else {
+            done = __shfl_sync(0xffffffffu, lane == 0 && ld_acquire_gpu(f.all_ready) == tag, 0);
+        }
+        if (done) break;
+        if (*abort_flag || global_timer() - t0 > kWaitLimitNs) {
+            *abort_flag = 1;
+            return false;
+        }
+        __nanosleep(blockIdx.x == 0 ? 200 : 1000);
+    }
+    __syncwarp();
+    __threadfence();
+    if (blockIdx.x == 0 && lane == 0) {
+        st_relaxed_gpu(f.epoch, tag);
+        st_release_gpu(f.all_ready, tag);
+    }
+    return true;
+}
+
+// Side work of the fused verification step, done by one extra warp of every CTA
+// while the other warps stream attention.  Once the argmax partials are
+// complete -- the preceding grid's (griddepcontrol.wait), or with in_grid the
+// ones the side warps of all CTAs compute first (side_argmax_chunks, then
+// side_wait_all) -- for every sequence b this CTA touches, or is designated to
+// report (b mod grid), the warp combines the node argmax from the partial
+// maxima, decides acceptance, writes the sequence's outputs if designated, and
+// copies the accepted tree K/V rows of this CTA's own (layer, sequence, head)
+// slices into the cache.  Attention only reads cache rows below each prefix,
+// so the copies never race with it.  Scratch (parent copies, top-1 tokens,
+// path) lives in a per-CTA slice of the workspace.  Kept out of line so that
+// its code does not reshape the register allocation of the attention loops.
+static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const WorkRange &wr, int lane,
+                                                    volatile int *abort_flag)
+{
+    const FusedStep &f = p.fs;
+    unsigned long long tag = 0;
+    bool have_all = false;
+    if (f.in_grid) {
+        tag = __shfl_sync(0xffffffffu, lane == 0 ? ld_relaxed_gpu(f.epoch) + 1ull : 0ull, 0);
+        side_argmax_chunks(p, tag, lane);
+    } else {
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        have_all = true;
+    }
     // the units whose first tile this CTA streams (its round-robin units and the
     // tail units starting in its range) compact their slices here
     const int t_lo = wr.u_first + (wr.j_first > 0 ? 1 : 0), t_hi = wr.n_tiles > 0 ? wr.u_last : -1;
-    auto owns_first_tile = [&](auto f) {
+    auto owns_first_tile = [&](auto fn) {
         for (int u = (int)blockIdx.x; u < wr.rr_units; u += (int)gridDim.x)
-            if (f(u)) return;
+            if (fn(u)) return;
         for (int u = t_lo; u <= t_hi; ++u)
-            if (f(u)) return;
+            if (fn(u)) return;
     };
-    const FusedStep &f = p.fs;
     const int T = p.T, B = p.B, S = f.splits;
     int *s_par = f.scratch + (size_t)blockIdx.x * kSideScratchInts;
     int *top = s_par + kAcceptScratchInts;
@@ -346,6 +482,10 @@ PPD_DEV void fused_side_warp(const AttnParams &p, const WorkRange &wr, int lane)
             return has_unit;
         });
         if (!designated && !has_unit) continue;
+        if (!have_all) {
+            if (!side_wait_all(p, tag, lane, abort_flag)) return;
+            have_all = true;
+        }
         for (int r = lane; r < T; r += 32) {
             const size_t base = ((size_t)b * T + r) * S;
             float bv = __ldcg(f.part_val + base);
@@ -373,7 +513,8 @@ PPD_DEV void fused_side_warp(const AttnParams &p, const WorkRange &wr, int lane)
                 f.accept_len[b] = res.n_acc;
                 f.next_token[b] = res.next_token;
                 f.new_prefix_len[b] = res.new_prefix_len;
-                atomicMax(f.status + b, res.status);
+                if (f.in_grid) f.status[b] = res.status;
+                else atomicMax(f.status + b, res.status);
             }
         }
         if (has_unit && res.n_acc > 0) {
@@ -404,7 +545,9 @@ PPD_DEV void fused_side_warp(const AttnParams &p, const WorkRange &wr, int lane)
 // Launch one of the persistent attention kernels: one CTA per SM (at most one
 // per unit, or with the work split at most one per tile and kSplitMaxGrid) of
 // `threads` threads, `smem` bytes of dynamic shared memory, with programmatic
-// stream serialization when asked.  The shared-memory opt-in is set once per
+// stream serialization when asked, and as a cooperative launch (all CTAs
+// resident at once, or the launch fails) when the fused step's side warps
+// compute the argmax in-grid.  The shared-memory opt-in is set once per
 // device.
 template <class Kern>
 cudaError_t launch_attention_grid(Kern kern, uint32_t smem, int threads,
@@ -426,11 +569,21 @@ cudaError_t launch_attention_grid(Kern kern, uint32_t smem, int threads,
     cfg.blockDim = dim3((unsigned)threads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute attr[2];
+    unsigned n_attr = 0;
+    if (programmatic) {
+        attr[n_attr].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n_attr].val.programmaticStreamSerializationAllowed = 1;
+        ++n_attr;
+    }
+    if (p.fused && p.fs.in_grid) {
+        // the side warps wait for one another's flags: every CTA must be resident
+        attr[n_attr].id = cudaLaunchAttributeCooperative;
+        attr[n_attr].val.cooperative = 1;
+        ++n_attr;
+    }
     cfg.attrs = attr;
-    cfg.numAttrs = programmatic ? 1 : 0;
+    cfg.numAttrs = n_attr;
     return cudaLaunchKernelEx(&cfg, kern, m.q, m.kc, m.vc, m.kt, m.vt, p);
 }
 

@@ -137,7 +137,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
     if (warp == 10) {
         // ------------------------------------------------------------ fused-step side work
-        if (p.fused) fused_side_warp(p, wr, lane);
+        if (p.fused) fused_side_warp(p, wr, lane, abort_flag);
     } else if (warp == 8 || warp == 11) {
         // ------------------------------------------------------------ TMA producers
         // warp 8 loads Q and the K tiles, warp 11 the V tiles: a V slot is released

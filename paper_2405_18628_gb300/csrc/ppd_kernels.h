@@ -15,20 +15,35 @@ struct AttnMaps {
     CUtensorMap q, kc, vc, kt, vt;
 };
 
-// The fused verification step's side work (see ppd_attention.cu): argmax
-// partials from the preceding grid, acceptance, and compaction of the CTA's
-// own (layer, sequence, head) slices.
+// The fused verification step's side work (see ppd_attention_common.cuh):
+// argmax partials (from the preceding grid, or with in_grid computed by the
+// side warps themselves), acceptance, and compaction of the CTA's own
+// (layer, sequence, head) slices.
 struct FusedStep {
-    const float *part_val;       // [B*T*splits] partial maxima
-    const int32_t *part_idx;
+    float *part_val;             // [B*T*splits] partial maxima
+    int32_t *part_idx;
     int splits;
+    // in_grid != 0: no preceding grid.  Chunk c of the [B*T][splits] partial
+    // grid is computed by CTA c mod grid; a CTA publishes ready[cta] = tag once
+    // its chunks are written, where tag = *epoch + 1 read at its start.  CTA 0
+    // waits until every flag equals tag, then sets *epoch = tag and
+    // *all_ready = tag; the other CTAs read partials once *all_ready equals
+    // their tag.  Every call has a fresh tag, so no flag needs zeroing.
+    int in_grid;
+    int chunk;                   // logits per chunk (multiple of 4 when vec)
+    int vec;                     // 16-byte loads of the logits
+    float stat_k;                // log2(e) / temperature (typical acceptance)
+    unsigned long long *epoch;   // [1]
+    unsigned long long *all_ready;   // [1]
+    unsigned long long *ready;   // [grid]
     const int32_t *cand_tokens;  // [B,T]
     int32_t *argmax_out;         // [B,T]
     int32_t *accept_len;         // [B]
     int32_t *path;               // [B,T]
     int32_t *next_token;         // [B]
     int32_t *new_prefix_len;     // [B]
-    int32_t *status;             // [B], zeroed by the argmax grid, raised with atomicMax
+    int32_t *status;             // [B]: zeroed by the argmax grid and raised with atomicMax;
+                                 // with in_grid written by the sequence's designated CTA
     uint8_t *k_cache, *v_cache;  // raw cache storage
     const uint8_t *k_tree, *v_tree;
     int row_bytes;               // D * element size
@@ -37,7 +52,7 @@ struct FusedStep {
     // typical acceptance (typical != 0): partial softmax statistics from the
     // preceding grid, the logits for p(token), and the rule's parameters
     int typical;
-    const float *part_stats;     // [B*T*splits][3]
+    float *part_stats;           // [B*T*splits][3]
     const float *logits;         // [B,T,V]
     float inv_temp, epsilon, delta;
 };

@@ -42,6 +42,7 @@ def load() -> ctypes.CDLL:
                                  ctypes.c_size_t)
         sig = {
             "ppd_workspace_bytes": ([i32] * 7 + [i32], sz),
+            "ppd_verify_step_launches": ([i32] * 7 + [i32, i32], i32),
             "ppd_status_string": ([i32], ctypes.c_char_p),
             "ppd_tree_attention": ([vp] * 7 + [i32] * 7 + [f32, vp, vp, vp, vp, sz, vp], i32),
             "ppd_node_argmax": ([vp, i32, i32, i32, vp, vp, sz, vp], i32),
@@ -101,6 +102,11 @@ def _check(status: int, where: str):
 
 def ppd_workspace_bytes(L, B, H, T, D, V, S_max, dtype=PPD_BF16) -> int:
     return int(load().ppd_workspace_bytes(L, B, H, T, D, V, S_max, dtype))
+
+
+def ppd_verify_step_launches(L, B, H, T, D, V, S_max, dtype=PPD_BF16, typical=False) -> int:
+    """Kernels one ppd_verify_step (or ppd_verify_step_typical) call enqueues."""
+    return int(load().ppd_verify_step_launches(L, B, H, T, D, V, S_max, dtype, int(typical)))
 
 
 def workspace(L, B, H, T, D, V, S_max, dtype=PPD_BF16, device="cuda") -> torch.Tensor:

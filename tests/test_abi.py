@@ -51,6 +51,22 @@ def test_workspace_bytes(lib):
     assert ppd.ppd_workspace_bytes(0, 1, 1, 1, 64, 1, 1) == 0
 
 
+def test_verify_step_launch_counts(lib):
+    """Kernels per verification step: one grid when the argmax runs inside the
+    attention grid (Vicuna-7B shapes: 8 MB of logits against 1.1 GB of K/V), an
+    argmax grid first when the logits weigh more (48 x 1024 logits against a
+    128-token prefix), five grids above 64 sequences, five fp32 rounding grids
+    in front for fp32 operands, and -1 for sizes the step rejects."""
+    from paper_2405_18628_gb300 import ppd
+    assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112) == 1
+    assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112, typical=True) == 1
+    assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 1024, 176) == 2
+    assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 1024, 176, ppd.PPD_F32) == 7
+    assert ppd.ppd_verify_step_launches(1, 65, 2, 16, 64, 300, 56) == 5
+    assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 96, 1024, 176) == -1
+    assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 0, 176) == -1
+
+
 def test_host_argument_checks(lib):
     """Invalid sizes and null pointers are rejected with PPD_ERR_INVALID_ARG
     (or UNSUPPORTED) without launching anything."""
