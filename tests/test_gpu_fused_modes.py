@@ -194,6 +194,36 @@ def test_in_grid_graph_replays(cuda_device):
         _check(w, s2, t, g, bufs, _ref(s2, t), f"replay seed {seed}")
 
 
+def test_in_grid_argmax_ties_nans_and_chunk_edges(cuda_device):
+    """The side warps' argmax follows the library's ranking rule (first NaN,
+    then the largest value, then the lowest index; -0 == +0) across the
+    chunk boundaries of the in-grid partial grid (V = 8192: 4 chunks of 2048
+    per row): bit for bit against the oracle, and the step's acceptance with it."""
+    w = _wl("f", 506, L=4, B=2, H=32, D=64, P=2000, T=16, V=8192, n_cand=8, chains="every1")
+    assert in_grid(w)
+    s, t = _inputs(w, [2000, 1234])
+    x = s.logits
+    x[0, 1, :] = -1.0
+    x[0, 1, 2047] = x[0, 1, 2048] = 5.0            # tie straddling chunks 0 and 1
+    x[0, 2, 5000] = np.nan
+    x[0, 2, 7000] = np.nan                          # first NaN wins, in a later chunk
+    x[0, 3, :] = -np.inf                            # all -inf: index 0
+    x[0, 4, 6000] = x[0, 4, 6001] = np.inf          # +inf tie inside one chunk
+    x[0, 5, :] = 0.25                               # constant row: index 0
+    x[0, 6, :] = -3.0
+    x[0, 6, 4096] = -0.0
+    x[0, 6, 4095] = 0.0                             # -0 == +0: the lower index
+    x[1, 0, :] = -2.0
+    x[1, 0, 8191] = 7.0                             # the very last logit
+    x[1, 1, :] = np.nan                             # all NaN: index 0
+    ref = _ref(s, t)
+    assert ref["argmax"][0, 1] == 2047 and ref["argmax"][0, 2] == 5000
+    assert ref["argmax"][0, 6] == 4095 and ref["argmax"][1, 0] == 8191
+    g, bufs = _run(w, s, t, cuda_device)
+    np.testing.assert_array_equal(bufs.argmax.cpu().numpy(), ref["argmax"])
+    _check(w, s, t, g, bufs, ref, "ties and NaNs")
+
+
 def test_in_grid_reports_bad_sequences(cuda_device):
     """Per-sequence status in the in-grid mode, written by each sequence's
     designated CTA: a malformed tree and a prefix with no room left."""
