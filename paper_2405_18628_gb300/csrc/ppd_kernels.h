@@ -120,7 +120,8 @@ inline int attention_grid(const AttnParams &p, int num_sms)
 // enqueued (one CTA per attention CTA, `grid` of them), after it completes.
 cudaError_t launch_split_merge(const AttnParams &p, int D, int grid, cudaStream_t stream);
 
-// Batches up to this size run the fused two-grid step.
+// Batches up to this size run the fused step (one grid, or an argmax grid then
+// the attention grid).
 constexpr int kFusedMaxB = 64;
 
 // Dispatches on the padded tree size: up to 64 tokens the key-row kernel

@@ -372,7 +372,8 @@ def test_verify_step_is_repeatable(cuda_device):
 
 @pytest.mark.parametrize("B", [64, 65])
 def test_verify_step_batch_paths(cuda_device, B):
-    """B <= 64 runs the fused two-grid step; larger batches run separate grids."""
+    """B <= 64 runs the fused step (here with an argmax grid first: the logits
+    outweigh the short prefixes); larger batches run separate grids."""
     w = W.Workload("batch", L=1, B=B, H=2, D=64, P=40, T=16, V=300, n_cand=8, max_depth=3,
                    chains="every1", match_rate=0.8, seed=B)
     rng = np.random.default_rng(B)
