@@ -49,10 +49,10 @@ L2_BYTES = 129 * 1000 * 1000
 # are scaled to the full layer count, since traffic grows with the units
 # (the logits, read once per step, are not scaled).
 MEASURED_TRAFFIC = {
-    # whole fused step: 685,501,696 B at 19 layers; slices x 32/19, logits once
-    "vicuna7b": {"bytes_per_launch": 1_148_924_120, "src": "c8ef1d632065f989"},
-    # whole fused step: 1,673,020,160 B at 19 layers; slices x 40/19, logits once
-    "vicuna13b": {"bytes_per_launch": 3_508_566_232, "src": "c8ef1d632065f989"},
+    # whole fused step: 685,382,912 B at 19 layers; slices x 32/19, logits once
+    "vicuna7b": {"bytes_per_launch": 1_148_724_062, "src": "34ce1a8dc4edf4e2"},
+    # whole fused step: 1,672,942,592 B at 19 layers; slices x 40/19, logits once
+    "vicuna13b": {"bytes_per_launch": 3_508_402_931, "src": "34ce1a8dc4edf4e2"},
 }
 
 

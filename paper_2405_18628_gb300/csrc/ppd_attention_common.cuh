@@ -398,7 +398,8 @@ PPD_DEV void side_argmax_chunks(const AttnParams &p, unsigned long long tag, int
 
 // Wait until every CTA of the grid has published `tag` (bounded: raises the
 // CTA's abort flag and returns false after kWaitLimitNs, or at once when the
-// flag is already up).  Only CTA 0 reads the per-CTA flags; once all are up
+// flag is already up; lane 0 takes that decision for the whole warp, so no
+// lane leaves while others still shuffle).  Only CTA 0 reads the per-CTA flags; once all are up
 // it advances the epoch for the next call and publishes `tag` in all_ready,
 // the one word the other CTAs poll (from one lane, with a backoff), so the
 // waits add little to the L2 traffic of the attention stream.
@@ -418,8 +419,10 @@ PPD_DEV bool side_wait_all(const AttnParams &p, unsigned long long tag, int lane
             done = __shfl_sync(0xffffffffu, lane == 0 && ld_acquire_gpu(f.all_ready) == tag, 0);
         }
         if (done) break;
-        if (*abort_flag || global_timer() - t0 > kWaitLimitNs) {
-            *abort_flag = 1;
+        const bool give_up = __shfl_sync(
+            0xffffffffu, lane == 0 && (*abort_flag || global_timer() - t0 > kWaitLimitNs), 0);
+        if (give_up) {
+            if (lane == 0) *abort_flag = 1;
             return false;
         }
         __nanosleep(blockIdx.x == 0 ? 200 : 1000);
