@@ -125,7 +125,7 @@ def measured_peak_gbs():
 def packed(specs, device):
     """One uint8 buffer holding several tensors, each at a 256-byte aligned
     offset: specs {name: (shape, dtype)} -> (buffer, {name: view}).  Host
-    buffers are pinned."""
+    buffers are pinned when a GPU is present."""
     import torch
     offs, off = {}, 0
     for k, (shape, dt) in specs.items():
@@ -133,7 +133,7 @@ def packed(specs, device):
         offs[k] = (off, n)
         off += (n + 255) // 256 * 256
     buf = torch.empty(off, dtype=torch.uint8, device=device,
-                      pin_memory=(str(device) == "cpu"))
+                      pin_memory=(str(device) == "cpu" and torch.cuda.is_available()))
     views = {k: buf[o:o + n].view(specs[k][1]).view(specs[k][0]) for k, (o, n) in offs.items()}
     return buf, views
 

@@ -1,5 +1,6 @@
-"""Host logic of bench.py's multi-rank runs (one replica per GPU, timing is
-the slowest rank's): checked with two gloo ranks on the CPU."""
+"""Host logic of bench.py: multi-rank runs (one replica per GPU, timing is the
+slowest rank's), checked with two gloo ranks on the CPU, and the packed
+buffers of the end-to-end leg."""
 import os
 import socket
 import sys
@@ -56,3 +57,20 @@ def test_single_process_defaults():
     assert bench.dist_setup({"WORLD_SIZE": "4", "RANK": "2", "LOCAL_RANK": "2"}) == (4, 2, 2)
     assert bench.max_over_ranks(3.5) == 3.5
     assert bench.aggregate_rate(10, 1, 1000.0) == pytest.approx(10.0)
+
+
+def test_packed_buffer_layout():
+    """The end-to-end leg's one-copy buffers: every member at a 256-byte aligned
+    offset, contiguous, with its own shape and dtype, and writable in place."""
+    import torch
+    sys.path.insert(0, ROOT)
+    import bench
+    buf, v = bench.packed({"q": ((2, 3, 5, 7), torch.bfloat16), "logits": ((3, 11), torch.float32),
+                           "parent": ((4,), torch.int32)}, "cpu")
+    for x in v.values():
+        assert x.is_contiguous() and (x.data_ptr() - buf.data_ptr()) % 256 == 0
+    assert v["q"].shape == (2, 3, 5, 7) and v["q"].dtype == torch.bfloat16
+    assert v["logits"].dtype == torch.float32 and v["parent"].dtype == torch.int32
+    assert buf.numel() == 512 + 256 + 256
+    v["parent"].copy_(torch.arange(4, dtype=torch.int32))
+    assert buf[768:784].view(torch.int32).tolist() == [0, 1, 2, 3]
