@@ -4,7 +4,7 @@ node argmax, acceptance, KV compaction) through libppd's C ABI.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl reference]
 
-Prints one JSON line.  The default workload is the Vicuna-7B-shaped cache
+Prints one JSON line.  The headline workload is the Vicuna-7B-shaped cache
 (32 layers, 32 heads x 128, bf16 K/V, batch 1, prefix 2048, 64-token tree,
 vocab 32000).  Inputs are seeded synthetic tensors resident in HBM.  When a
 step's inputs are at least four times the 129 MB L2 (every Vicuna-shaped
@@ -12,15 +12,27 @@ workload: 1.17 GB per step at Vicuna-7B), steps run back to back and no step
 can find the previous one's data in L2; smaller workloads flush L2 (a 256 MiB
 write) before every timed step, outside the step's events.
 
-Under torchrun (N > 1) each rank runs an independent replica of the workload
-on its own GPU (weak scaling: the sequences of different ranks are
+On one GPU the default run also times, each with its own K steps, the other
+workloads of the paper's evaluation models (MobileLlama-, Vicuna-13B-shaped,
+and the batch-8 / prefix-16384 tree-size sweep) under "workloads", the
+attention as a model calls it (one call per layer) under
+"per_layer_attention", and the step latency against the tree size (the
+hardware half of the paper's hardware-aware tree size) under
+"tree_size_profile".  GPU clocks are sampled from before the first warm-up
+step to after the last timed loop; "clocks" summarises the samples taken
+inside timed loops.
+
+Under torchrun (N > 1) each rank runs an independent replica of the headline
+workload on its own GPU (weak scaling: the sequences of different ranks are
 independent, no data-path collective); the step time is the maximum over
 ranks.  `--impl reference` times the fp64 CPU oracle on the host cores
-instead (rank 0 only), on a bounded sample of the same workload.
+instead (rank 0 only), on whole steps of the same workload when they fit a
+few minutes, else on a bounded sample of each step.
 """
 from __future__ import annotations
 
 import argparse
+import datetime
 import hashlib
 import json
 import os
@@ -41,13 +53,22 @@ FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 256 << 20
 TYPICAL = (0.7, 0.09, 0.3)   # temperature, epsilon, delta of --accept typical
 L2_BYTES = 129 * 1000 * 1000
+# the other workloads of the paper's evaluation models, timed after the headline one
+EXTRA_WORKLOADS = ("mobilellama", "vicuna13b", "sweep_t16", "sweep_t32", "sweep_t64", "sweep_t128")
+# tree sizes of the latency profile L_fp(n) (Vicuna-7B shapes)
+PROFILE_SIZES = (16, 32, 48, 64, 96, 128, 192, 256, 384, 512)
+# seconds of oracle work the reference arm may spend in total before it falls
+# back from whole steps to a bounded sample of each step
+REFERENCE_BUDGET_S = 180.0
 
 # DRAM traffic of one launch of the roofline kernel (dram__bytes_read.sum +
 # dram__bytes_write.sum), keyed by workload, with the hash of the attention
 # sources it was taken on: a stale entry reports null.  The captures ran the
 # same shapes with 19 layers (608 / 760 units: whole rounds of 152 CTAs) and
 # are scaled to the full layer count, since traffic grows with the units
-# (the logits, read once per step, are not scaled).
+# (the logits, read once per step, are not scaled).  Writes still held in L2
+# when the kernel ends are not in the count, so this is the reads plus the
+# part of the writes that reached DRAM during the launch.
 MEASURED_TRAFFIC = {
     # whole fused step: 685,382,912 B at 19 layers; slices x 32/19, logits once
     "vicuna7b": {"bytes_per_launch": 1_148_724_062, "src": "34ce1a8dc4edf4e2"},
@@ -63,53 +84,6 @@ def attention_source_hash() -> str:
         with open(os.path.join(ROOT, "paper_2405_18628_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
-
-
-def per_layer_attention(w, t, prefix, parent, out, dev, reps):
-    """Attention as a model runs it: L ppd_tree_attention calls of one layer
-    each, captured in a CUDA graph and replayed `reps` times (CUDA events on the
-    replay stream, median).  With a workspace the library shares each call's
-    key tiles over all SMs when the layer has fewer slices than SMs; without,
-    one whole slice per SM."""
-    import torch
-
-    from paper_2405_18628_gb300 import ppd
-
-    st = torch.zeros(w.B, dtype=torch.int32, device=dev)
-    ws = ppd.workspace(1, w.B, w.H, w.T, w.D, 1, w.S_max, device=dev)
-    res = {}
-    for mode, wsx in (("split", ws), ("unsplit", None)):
-        def layers():
-            for l in range(w.L):
-                ppd.ppd_tree_attention(t["q"][l:l + 1], t["k_cache"][l:l + 1], t["v_cache"][l:l + 1],
-                                       t["k_tree"][l:l + 1], t["v_tree"][l:l + 1], prefix, parent,
-                                       out[l:l + 1], st, workspace=wsx)
-        layers()
-        torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
-        cap = torch.cuda.Stream()
-        cap.wait_stream(torch.cuda.current_stream())
-        with torch.cuda.stream(cap):
-            with torch.cuda.graph(g, stream=cap):
-                layers()
-        torch.cuda.current_stream().wait_stream(cap)
-        s = torch.cuda.current_stream()
-        for _ in range(5):
-            g.replay()
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(reps)]
-        for a, b in ev:
-            a.record(s)
-            g.replay()
-            b.record(s)
-        torch.cuda.synchronize()
-        if (st.cpu().numpy() != 0).any():
-            raise SystemExit(f"per-layer attention reported device status {st.cpu().tolist()}")
-        us = statistics.median(a.elapsed_time(b) for a, b in ev) * 1e3
-        res[mode] = {"us_per_step": us, "us_per_layer": us / w.L,
-                     "gbs": attention_bytes(w) / (us * 1e-6) / 1e9}
-        del g
-    return {"graph": True, "layers": w.L, "slices_per_layer": w.B * w.H, **res}
 
 
 def measured_peak_gbs():
@@ -148,67 +122,114 @@ def attention_bytes(w) -> int:
 
 def step_bytes(w, n_acc_total: int) -> int:
     """Algorithmic bytes of one verification step: attention, the fp32 logits,
-    the compacted K/V rows (read from the tree, written to the cache) and the
-    small integer arrays."""
+    the compacted K/V rows written into the cache (bf16 K and V: 4*D bytes per
+    layer, head and accepted node; the tree rows they copy are already counted
+    in the attention's reads) and the small integer arrays (parent, candidate
+    ids, argmax and path per node; prefix, accepted length, next token, new
+    prefix, status per sequence)."""
     ints = 4 * w.B * w.T * 4 + 4 * w.B * 6
     return (attention_bytes(w) + 4 * w.B * w.T * w.V +
-            2 * 4 * w.L * w.H * w.D * n_acc_total + ints)
+            4 * w.L * w.H * w.D * n_acc_total + ints)
 
 
 # ----------------------------------------------------------------------------- clocks
 
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi sampling every 50 ms into a file, with the sample timestamps;
+    `summary(windows)` keeps the samples inside the given (start, end)
+    datetime windows (the timed loops)."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
 
     def __init__(self, index: int):
         self.index = index
         self.proc = None
         self.path = None
 
-    def __enter__(self):
+    def start(self, wait_s: float = 5.0):
         fd, self.path = tempfile.mkstemp(suffix=".csv")
         os.close(fd)
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
+            return self
+        t0 = time.perf_counter()
+        while time.perf_counter() - t0 < wait_s and not self._rows():
+            time.sleep(0.05)
         return self
 
-    def __exit__(self, *exc):
+    def stop(self):
         if self.proc is not None:
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
             except Exception:
                 self.proc.kill()
+            self.proc = None
 
-    def summary(self):
+    @staticmethod
+    def _num(x):
+        try:
+            return float(x)
+        except ValueError:
+            return None
+
+    def _rows(self):
         rows = []
         try:
             with open(self.path) as f:
                 for line in f:
                     parts = [p.strip() for p in line.split(",")]
-                    if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
-                        rows.append(parts)
+                    if len(parts) < 10 or self._num(parts[2]) is None:
+                        continue
+                    try:
+                        ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f")
+                    except ValueError:
+                        continue
+                    rows.append((ts, parts))
         except Exception:
             pass
-        finally:
-            if self.path and os.path.exists(self.path):
-                os.unlink(self.path)
+        return rows
+
+    def summary(self, windows):
+        rows = self._rows()
+        if self.path and os.path.exists(self.path):
+            os.unlink(self.path)
+        inside = [r for ts, r in rows if any(a <= ts <= b for a, b in windows)]
         if not rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k].lower() == "active"})
-        return {"sm_mhz": statistics.median(float(r[1]) for r in rows),
-                "sm_max_mhz": max(float(r[2]) for r in rows),
-                "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())
-                if any(r[3].replace(".", "").isdigit() for r in rows) else None,
-                "reasons": reasons, "samples": len(rows)}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "samples_in_timed_loops": 0}
+        use = inside if inside else [r for _, r in rows]
+        pw = [self._num(r[4]) for r in use if self._num(r[4]) is not None]
+        reasons = sorted({self.REASONS[k] for r in use for k in range(4)
+                          if r[6 + k].lower() == "active"})
+        return {"sm_mhz": statistics.median(self._num(r[2]) for r in use),
+                "sm_max_mhz": max(self._num(r[3]) for r in use),
+                "power_w_max": max(pw) if pw else None,
+                "reasons": reasons, "samples": len(rows),
+                "samples_in_timed_loops": len(inside),
+                "basis": ("samples inside the timed loops" if inside else
+                          "every sample of the run (none fell inside a timed loop)")}
+
+
+class Windows:
+    """Wall-clock windows of the timed loops (for the clock summary)."""
+
+    def __init__(self):
+        self.spans = []
+
+    def __enter__(self):
+        self._t0 = datetime.datetime.now()
+        return self
+
+    def __exit__(self, *exc):
+        self.spans.append((self._t0, datetime.datetime.now()))
 
 
 # ----------------------------------------------------------------------------- CPU oracle
@@ -218,7 +239,8 @@ def oracle_step_seconds(w, host, s, units, n_threads: int) -> float:
     the whole step.  `host` holds the first few layers of Q/K/V on the host;
     attention runs on `units` of them (None: all), compaction on all of them,
     argmax and acceptance once, as in a full step.  Attention and compaction
-    times are scaled by the fraction of the workload the sample covers."""
+    times are scaled by the fraction of the workload the sample covers (1 for
+    a whole step)."""
     import oracle
     L_h = host["q"].shape[0]
     n_sample = len(units) if units is not None else L_h * w.B * w.H
@@ -238,10 +260,16 @@ def oracle_step_seconds(w, host, s, units, n_threads: int) -> float:
     return t_att * (w.L * w.B * w.H) / n_sample + t_acc + t_cmp * w.L / L_h
 
 
+def one_thread_seconds(w, host, s) -> float:
+    """The oracle step on one host thread: the attention of the first layer
+    (all sequences and heads) scaled by L, argmax and acceptance in full."""
+    one = {k: v[:1] for k, v in host.items()}
+    return oracle_step_seconds(w, one, s, None, 1)
+
+
 def cpu_baseline(w, t_dev, s, budget_s: float):
     """Oracle on the first `nl` layers, `nl` chosen from a one-layer calibration
     so the sample takes about `budget_s` seconds of host time."""
-    import oracle
     n_threads = os.cpu_count() or 1
     one = {k: v[:1].cpu() for k, v in t_dev.items()}
     t0 = time.perf_counter()
@@ -251,14 +279,16 @@ def cpu_baseline(w, t_dev, s, budget_s: float):
     host = one if nl == 1 else {k: v[:nl].cpu() for k, v in t_dev.items()}
     sec = oracle_step_seconds(w, host, s, None, n_threads)
     return {"value": 1.0 / sec, "unit": "steps/s", "cores": n_threads, "kind": "oracle",
-            "sample": f"fp64 oracle verification step on the first {nl} of {w.L} layers "
-                      f"(all heads; attention and compaction time scaled by {w.L}/{nl}; "
-                      f"full argmax and acceptance)"}
+            "sample": (f"fp64 oracle verification step on all {w.L} layers (whole step)"
+                       if nl == w.L else
+                       f"fp64 oracle verification step on the first {nl} of {w.L} layers "
+                       f"(all heads; attention and compaction time scaled by {w.L}/{nl}; "
+                       f"full argmax and acceptance)")}
 
 
 # ----------------------------------------------------------------------------- main
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
@@ -269,26 +299,28 @@ def parse():
                     help="seconds of oracle work in the CPU baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="time the headline workload only (no other workloads, per-layer "
+                         "attention or tree-size profile)")
     ap.add_argument("--accept", default="exact", choices=["exact", "typical"],
                     help="verification rule: exact matching, or typical acceptance at "
                          "temperature 0.7, epsilon 0.09, delta 0.3")
-    ap.add_argument("--tree-sizes", default="",
-                    help="comma-separated tree sizes: also report the step latency of each "
-                         "(the hardware half of the paper's hardware-aware tree size)")
+    ap.add_argument("--tree-sizes", default=None,
+                    help="comma-separated tree sizes of the latency profile (the hardware "
+                         "half of the paper's hardware-aware tree size); '' for none")
     ap.add_argument("--tau", default="",
-                    help="JSON file {tree size: acceptance length}: with --tree-sizes, also "
-                         "report Speedup(n) = tau(n) / latency(n) and the best size")
+                    help="JSON file {tree size: acceptance length}: also report "
+                         "Speedup(n) = tau(n) / latency(n) and the best size")
     ap.add_argument("--next-tree", action="store_true",
                     help="also time next-step candidate generation (ppd_next_tree, 5 tree "
                          "states, 8 guesses per depth) after each step")
     ap.add_argument("--per-layer", action="store_true",
-                    help="also time the attention as it runs inside a model: one "
-                         "ppd_tree_attention call per layer, the L calls captured in a CUDA graph")
+                    help="time the per-layer attention even when extras are off")
     ap.add_argument("--layers", type=int, default=0,
                     help="run the workload with this many layers (profiling captures)")
     ap.add_argument("--l2", default="auto", choices=["auto", "flush", "none"],
                     help="auto: flush L2 before each step unless the step's inputs exceed 4x L2")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def dist_setup(env=None):
@@ -315,53 +347,239 @@ def aggregate_rate(steps_per_rank: int, world: int, slowest_ms: float) -> float:
     return world * steps_per_rank / (slowest_ms / 1e3)
 
 
+def resolve_workload(args):
+    from paper_2405_18628_gb300 import workloads as W
+    w = W.WORKLOADS[args.config]
+    if args.layers:
+        # fewer layers of the same shapes: small cases for profiler captures
+        w = W.scaled(w, L=args.layers)
+    return w
+
+
+def flushes_l2(w, mode: str) -> bool:
+    """Whether L2 is flushed before each timed step: always with "flush", never
+    with "none", and with "auto" when a step's inputs are below 4x L2."""
+    return mode == "flush" or (mode == "auto" and step_bytes(w, 0) < 4 * L2_BYTES)
+
+
+def config_of(w, args, world: int) -> dict:
+    """The `config` object of the JSON line (the same for both arms)."""
+    footprint = step_bytes(w, 0)
+    return {"workload": w.name + (f" ({w.L} layers)" if args.layers else ""),
+            "layers": w.L, "batch": w.B, "heads": w.H, "head_dim": w.D, "prefix": w.P,
+            "tree_tokens": w.T, "vocab": w.V, "S_max": w.S_max,
+            "l2": ("flushed before every step (256 MiB write, outside the step events)"
+                   if flushes_l2(w, args.l2) else
+                   f"not flushed: inputs larger than L2 ({footprint / 1e6:.0f} MB "
+                   f"streamed per step, L2 {L2_BYTES / 1e6:.0f} MB)"),
+            "parallelism": f"replicas x{world}",
+            "accept": ("exact matching" if args.accept == "exact" else
+                       "typical acceptance (temperature %g, epsilon %g, delta %g)" % TYPICAL)}
+
+
 def run_reference(args, w, world, rank):
-    """The CPU oracle as the reference arm.  Each step is a bounded sample: a
-    few attention slices of layer 0 (scaled to all slices), the full argmax and
-    acceptance, and layer 0's compaction (scaled to all layers)."""
+    """The CPU oracle as the reference arm: whole verification steps of the
+    workload (attention of every layer, argmax, acceptance, compaction of every
+    layer) when W + K of them fit REFERENCE_BUDGET_S, else each step a bounded
+    sample (a few attention slices of layer 0 scaled to all slices, the full
+    argmax and acceptance, layer-0 compaction scaled to all layers).  Also a
+    one-thread timing of the step (first layer scaled by L)."""
     if rank != 0:
         return
     from paper_2405_18628_gb300 import workloads as W
 
     s = W.make_step_inputs(w)
     n_threads = os.cpu_count() or 1
-    host = W.make_tensors(W.scaled(w, L=1), device="cpu")
-    n_all = w.B * w.H
-    cal = list(range(min(n_threads, n_all)))
+    host = W.make_tensors(w, device="cpu")
     t0 = time.perf_counter()
-    oracle_step_seconds(w, host, s, cal, n_threads)
-    t_cal = time.perf_counter() - t0
-    per_step_budget = max(0.01, 150.0 / max(1, args.steps + args.warmup))
-    n_units = int(max(1, min(n_all, len(cal) * per_step_budget / max(t_cal, 1e-9))))
-    units = list(range(n_units))
-    for _ in range(args.warmup):
+    oracle_step_seconds(w, host, s, None, n_threads)          # calibration (= warm-up 1)
+    t_full = time.perf_counter() - t0
+    whole = (args.warmup + args.steps) * t_full <= REFERENCE_BUDGET_S
+    if whole:
+        units = None
+        sample = (f"whole steps: attention of all {w.L * w.B * w.H} slices, full argmax and "
+                  f"acceptance, compaction of all {w.L} layers")
+    else:
+        per_step = max(0.01, REFERENCE_BUDGET_S / max(1, args.steps + args.warmup))
+        n_all = w.L * w.B * w.H
+        n_units = int(max(1, min(n_all, n_all * per_step / max(t_full, 1e-9))))
+        units = list(range(n_units))
+        sample = (f"{n_units} of {n_all} attention slices per step, scaled to all slices; "
+                  f"full argmax and acceptance; compaction of all layers")
+    for _ in range(max(0, args.warmup - 1)):
         oracle_step_seconds(w, host, s, units, n_threads)
     secs = [oracle_step_seconds(w, host, s, units, n_threads) for _ in range(args.steps)]
     sec_per_step = statistics.mean(secs)
     value = 1.0 / sec_per_step
-    sample = (f"{n_units} of {w.L * w.B * w.H} attention slices (layer 0) per step, scaled to all "
-              f"slices; full argmax and acceptance; layer-0 compaction scaled to {w.L} layers")
+    t1 = one_thread_seconds(w, host, s)
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": sec_per_step * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name},
+        "config": config_of(w, args, world),
         "cpu_baseline": {"value": value, "unit": "steps/s", "cores": n_threads, "kind": "oracle",
                          "sample": sample},
+        "one_thread": {"value": 1.0 / t1, "unit": "steps/s", "cores": 1, "kind": "oracle",
+                       "sample": f"attention of layer 0 (all heads) scaled by {w.L}; full argmax "
+                                 f"and acceptance; compaction of layer 0 scaled by {w.L}"},
         "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }), flush=True)
 
 
-def main():
-    args = parse()
-    world, rank, local = dist_setup()
+class Step:
+    """Device inputs and outputs of one workload and its step call."""
+
+    def __init__(self, w, dev, seed, accept="exact"):
+        import torch
+
+        from paper_2405_18628_gb300 import ppd
+        from paper_2405_18628_gb300 import workloads as W
+        self.w, self.dev, self.accept = w, dev, accept
+        self.s = W.make_step_inputs(w, seed=seed)
+        self.t = W.make_tensors(w, device=dev, seed=seed)
+        i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
+        self.parent, self.cand, self.prefix = (i32(self.s.parent), i32(self.s.cand_tokens),
+                                               i32(self.s.prefix_len))
+        self.logits = torch.from_numpy(self.s.logits).to(dev)
+        self.bufs = ppd.StepBuffers(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max, device=dev)
+
+    def __call__(self, stream):
+        from paper_2405_18628_gb300 import ppd
+        t, b = self.t, self.bufs
+        if self.accept == "typical":
+            ppd.ppd_verify_step_typical(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
+                                        self.prefix, self.parent, self.cand, self.logits, *TYPICAL,
+                                        b.out, b.argmax, b.accept_len, b.path, b.next_token,
+                                        b.new_prefix_len, b.dev_status, b.workspace, stream=stream)
+        else:
+            ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
+                                self.prefix, self.parent, self.cand, self.logits, b.out, b.argmax,
+                                b.accept_len, b.path, b.next_token, b.new_prefix_len,
+                                b.dev_status, b.workspace, stream=stream)
+
+    def check(self):
+        status = self.bufs.dev_status.cpu().numpy()
+        n_acc = int(self.bufs.accept_len.sum().item())
+        if (status != 0).any() or n_acc < self.w.B:
+            raise SystemExit(f"{self.w.name}: verification step reported device status "
+                             f"{status.tolist()}")
+        return n_acc
+
+
+def time_loop(fn, K, warmup, stream, flush, windows):
+    """W untimed calls, then K calls each between CUDA events on `stream`
+    (L2 flushed before each when `flush` is a buffer).  Returns the K times in
+    ms and the wall-clock seconds of the timed loop."""
+    import torch
+    for _ in range(max(3, warmup)):
+        if flush is not None:
+            flush.zero_()
+        fn()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    with windows:
+        t0 = time.perf_counter()
+        for a, b in ev:
+            if flush is not None:
+                flush.zero_()
+            a.record(stream)
+            fn()
+            b.record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    return [a.elapsed_time(b) for a, b in ev], wall
+
+
+def per_layer_attention(w, t, prefix, parent, out, dev, reps, windows):
+    """Attention as a model runs it: L ppd_tree_attention calls of one layer
+    each, captured in a CUDA graph and replayed `reps` times (CUDA events on the
+    replay stream, median).  With a workspace the library shares each call's
+    key tiles over all SMs when the layer has fewer slices than SMs; without,
+    one whole slice per SM."""
+    import torch
+
+    from paper_2405_18628_gb300 import ppd
+
+    st = torch.zeros(w.B, dtype=torch.int32, device=dev)
+    ws = ppd.workspace(1, w.B, w.H, w.T, w.D, 1, w.S_max, device=dev)
+    res = {}
+    for mode, wsx in (("split", ws), ("unsplit", None)):
+        def layers():
+            for l in range(w.L):
+                ppd.ppd_tree_attention(t["q"][l:l + 1], t["k_cache"][l:l + 1], t["v_cache"][l:l + 1],
+                                       t["k_tree"][l:l + 1], t["v_tree"][l:l + 1], prefix, parent,
+                                       out[l:l + 1], st, workspace=wsx)
+        layers()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream()
+        cap.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(cap):
+            with torch.cuda.graph(g, stream=cap):
+                layers()
+        torch.cuda.current_stream().wait_stream(cap)
+        s = torch.cuda.current_stream()
+        ms, _ = time_loop(g.replay, reps, 5, s, None, windows)
+        if (st.cpu().numpy() != 0).any():
+            raise SystemExit(f"per-layer attention reported device status {st.cpu().tolist()}")
+        us = statistics.median(ms) * 1e3
+        res[mode] = {"us_per_step": us, "us_per_layer": us / w.L,
+                     "gbs": attention_bytes(w) / (us * 1e-6) / 1e9}
+        del g
+    return {"graph": True, "layers": w.L, "slices_per_layer": w.B * w.H, **res}
+
+
+def summarize(w, ms, n_acc, peak, launches):
+    q10, q50, q90 = np.percentile(ms, [10, 50, 90])
+    mean = float(np.mean(ms))
+    sb = step_bytes(w, n_acc)
+    return {"ms_per_step": mean, "ms_per_step_p10_p50_p90": [float(q10), float(q50), float(q90)],
+            "steps_per_s": 1e3 / mean, "step_bytes": sb, "step_gbs": sb / (mean * 1e-3) / 1e9,
+            "frac": sb / (mean * 1e-3) / 1e9 / peak,
+            "frac_of_8000": sb / (mean * 1e-3) / 1e9 / NOMINAL_HBM_GBS, "launches": launches}
+
+
+def bench_extra_workload(name, K, warmup, dev, stream, peak, windows, accept, with_per_layer):
+    """One of the other workloads: its own inputs, K timed steps (L2 flushed
+    before each when the inputs are below 4x L2), freed afterwards."""
+    import torch
+
+    from paper_2405_18628_gb300 import ppd
     from paper_2405_18628_gb300 import workloads as W
-    w = W.WORKLOADS[args.config]
-    if args.layers:
-        # fewer layers of the same shapes: small cases for profiler captures
-        w = W.scaled(w, L=args.layers)
+    w = W.WORKLOADS[name]
+    need = 2 * w.L * w.B * w.H * (w.S_max + 2 * w.T) * w.D * 2
+    torch.cuda.empty_cache()
+    free, _ = torch.cuda.mem_get_info()
+    if need * 1.3 > free:
+        return {"skipped": f"needs {need / 2**30:.0f} GiB of device memory"}
+    st = Step(w, dev, w.seed, accept)
+    flush = (torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+             if flushes_l2(w, "auto") else None)
+    st(stream)
+    torch.cuda.synchronize()
+    n_acc = st.check()
+    ms, _ = time_loop(lambda: st(stream), K, warmup, stream, flush, windows)
+    n_launch = ppd.ppd_verify_step_launches(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max,
+                                            typical=accept == "typical")
+    res = summarize(w, ms, n_acc, peak, n_launch)
+    res["l2"] = "flushed before every step" if flush is not None else "not flushed"
+    res["shape"] = {"layers": w.L, "batch": w.B, "heads": w.H, "head_dim": w.D,
+                    "prefix": w.P, "tree_tokens": w.T, "vocab": w.V}
+    if with_per_layer:
+        res["per_layer_attention"] = per_layer_attention(w, st.t, st.prefix, st.parent,
+                                                         st.bufs.out, dev, min(K, 100), windows)
+    del st, flush
+    torch.cuda.empty_cache()
+    return res
+
+
+def main(argv=None):
+    args = parse(argv)
+    world, rank, local = dist_setup()
+    w = resolve_workload(args)
     if args.impl == "reference":
         run_reference(args, w, world, rank)
         return
@@ -377,58 +595,43 @@ def main():
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
     ppd.load()
+    extras = world == 1 and not args.no_extras and not args.layers
+    clocks = ClockSampler(local).start()
+    windows = Windows()
+    peak, peak_kind = measured_peak_gbs()
 
     # ---------------------------------------------------------------- inputs (resident in HBM)
-    s = W.make_step_inputs(w, seed=w.seed + 1000 * rank)
-    t = W.make_tensors(w, device=dev, seed=w.seed + 1000 * rank)
-    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
-    parent, cand, prefix = i32(s.parent), i32(s.cand_tokens), i32(s.prefix_len)
-    logits = torch.from_numpy(s.logits).to(dev)
-    bufs = ppd.StepBuffers(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max, device=dev)
+    seed = w.seed + 1000 * rank
+    st = Step(w, dev, seed, args.accept)
+    t, s, bufs, logits = st.t, st.s, st.bufs, st.logits
+    parent, cand, prefix = st.parent, st.cand, st.prefix
     stream = torch.cuda.current_stream()
-    footprint = step_bytes(w, 0)
-    do_flush = args.l2 == "flush" or (args.l2 == "auto" and footprint < 4 * L2_BYTES)
+    do_flush = flushes_l2(w, args.l2)
     flush = torch.empty(L2_FLUSH_BYTES if do_flush else 0, dtype=torch.uint8, device=dev)
 
     def maybe_flush():
         if do_flush:
             flush.zero_()
 
-    def step():
-        if args.accept == "typical":
-            ppd.ppd_verify_step_typical(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
-                                        prefix, parent, cand, logits, *TYPICAL, bufs.out,
-                                        bufs.argmax, bufs.accept_len, bufs.path, bufs.next_token,
-                                        bufs.new_prefix_len, bufs.dev_status, bufs.workspace,
-                                        stream=stream)
-        else:
-            ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
-                                parent, cand, logits, bufs.out, bufs.argmax, bufs.accept_len,
-                                bufs.path, bufs.next_token, bufs.new_prefix_len, bufs.dev_status,
-                                bufs.workspace, stream=stream)
-
     for _ in range(max(3, args.warmup)):
         maybe_flush()
-        step()
+        st(stream)
     torch.cuda.synchronize()
-    status = bufs.dev_status.cpu().numpy()
-    n_acc = int(bufs.accept_len.sum().item())
-    if (status != 0).any() or n_acc < w.B:
-        raise SystemExit(f"verification step reported device status {status.tolist()}")
+    n_acc = st.check()
 
     # ---------------------------------------------------------------- timed region
     K = args.steps
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(K)]
-    with ClockSampler(local) as clocks:
-        if pg:
-            pg.barrier()
-        torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    with windows:
         wall0 = time.perf_counter()
         for k in range(K):
             maybe_flush()
             ev[k][0].record(stream)
-            step()
+            st(stream)
             ev[k][1].record(stream)
         torch.cuda.synchronize()
         if pg:
@@ -439,25 +642,15 @@ def main():
     total_ms = max_over_ranks(sum(step_ms), pg, dev)
     ms_per_step = total_ms / K
     value = aggregate_rate(K, world, total_ms)
-    clk = clocks.summary()
 
     # ---------------------------------------------------------------- dominant kernel alone
-    K2 = min(K, 300)
-    ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(K2)]
     st_att = torch.empty(w.B, dtype=torch.int32, device=dev)
-    for k in range(K2 + 3):
-        maybe_flush()
-        if k >= 3:
-            ev2[k - 3][0].record(stream)
-        ppd.ppd_tree_attention(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"], prefix,
-                               parent, bufs.out, st_att, stream=stream)
-        if k >= 3:
-            ev2[k - 3][1].record(stream)
-    torch.cuda.synchronize()
-    att_ms = statistics.mean(a.elapsed_time(b) for a, b in ev2)
+    att, _ = time_loop(lambda: ppd.ppd_tree_attention(t["q"], t["k_cache"], t["v_cache"],
+                                                      t["k_tree"], t["v_tree"], prefix, parent,
+                                                      bufs.out, st_att, stream=stream),
+                       min(K, 300), 3, stream, flush if do_flush else None, windows)
+    att_ms = statistics.mean(att)
     att_bytes = attention_bytes(w)
-    peak, peak_kind = measured_peak_gbs()
     achieved = att_bytes / (att_ms * 1e-3) / 1e9
     tr = None if args.layers else MEASURED_TRAFFIC.get(w.name)
     traffic = tr["bytes_per_launch"] if tr and tr.get("src") == attention_source_hash() else None
@@ -512,17 +705,14 @@ def main():
                        "index arrays copied in from one pinned host buffer, every output "
                        "copied back into one (256-byte aligned members, one copy each way)"}
 
-    # ---------------------------------------------------------------- CPU baseline (oracle)
-    cpu = None
-    if world == 1 and rank == 0 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w, t, s, args.cpu_budget)
-
     # ---------------------------------------------------------------- next-step candidates
     next_tree = None
     if args.next_tree:
+        from paper_2405_18628_gb300 import workloads as W
+        i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
         n_states, K_guess = 5, 8
-        tp, tr = W.make_tree_templates(n_states, w.T, K_guess, np.random.default_rng(w.seed))
-        tp_d, tr_d = i32(tp), i32(tr)
+        tp, trk = W.make_tree_templates(n_states, w.T, K_guess, np.random.default_rng(w.seed))
+        tp_d, tr_d = i32(tp), i32(trk)
         nxt = {k: torch.empty(shape, dtype=torch.int32, device=dev) for k, shape in
                (("parent", (w.B, w.T)), ("cand", (w.B, w.T)), ("state", (w.B,)), ("status", (w.B,)))}
         ws_nt = torch.empty(max(256, ppd.load().ppd_next_tree_workspace_bytes(w.B, n_states, K_guess)),
@@ -537,7 +727,7 @@ def main():
         ev4 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                for _ in range(K4)]
         for k in range(K4 + 3):
-            step()
+            st(stream)
             if k >= 3:
                 ev4[k - 3][0].record(stream)
             next_step()
@@ -553,29 +743,51 @@ def main():
 
     # ---------------------------------------------------------------- per-layer attention
     per_layer = None
-    if args.per_layer:
-        per_layer = per_layer_attention(w, t, prefix, parent, bufs.out, dev, min(K, 100))
+    if extras or args.per_layer:
+        per_layer = per_layer_attention(w, t, prefix, parent, bufs.out, dev, min(K, 100), windows)
 
-    # ---------------------------------------------------------------- tree-size profile
-    profile = None
-    if args.tree_sizes:
-        from paper_2405_18628_gb300 import tree_profile
-        del t, bufs, logits
-        torch.cuda.empty_cache()
-        sizes = [int(x) for x in args.tree_sizes.split(",") if x.strip()]
-        lat = tree_profile.latency_profile(w, sizes, steps=min(K, 50), warmup=3, device=dev,
-                                           flush_bytes=L2_FLUSH_BYTES if do_flush else 0)
-        profile = {"latency": [{"T": n, "ms_per_step": ms} for n, ms in lat]}
-        if args.tau:
-            with open(args.tau) as f:
-                tau = {int(k): float(v) for k, v in json.load(f).items()}
-            rows, best = tree_profile.speedup_table(tau, lat)
-            profile["speedup"] = rows
-            profile["best_tree_size"] = best
+    # ---------------------------------------------------------------- CPU baseline (oracle)
+    cpu = None
+    if world == 1 and rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, t, s, args.cpu_budget)
 
     sb = step_bytes(w, n_acc)
     n_launch = ppd.ppd_verify_step_launches(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max,
                                             typical=args.accept == "typical")
+    del st, t, bufs, logits, flush
+    torch.cuda.empty_cache()
+
+    # ---------------------------------------------------------------- the other workloads
+    others = None
+    if extras:
+        others = {}
+        for name in EXTRA_WORKLOADS:
+            others[name] = bench_extra_workload(name, K, args.warmup, dev, stream, peak, windows,
+                                                args.accept, name in ("mobilellama", "vicuna13b"))
+
+    # ---------------------------------------------------------------- tree-size profile
+    profile = None
+    sizes_arg = args.tree_sizes if args.tree_sizes is not None else (
+        ",".join(str(n) for n in PROFILE_SIZES) if extras else "")
+    if sizes_arg:
+        from paper_2405_18628_gb300 import tree_profile
+        sizes = [int(x) for x in sizes_arg.split(",") if x.strip()]
+        lat = tree_profile.latency_profile(w, sizes, steps=max(K, 20), warmup=3, device=dev,
+                                           flush_bytes=L2_FLUSH_BYTES if do_flush else 0,
+                                           timed=windows)
+        profile = {"base": w.name, "steps_each": max(K, 20),
+                   "latency": [{"T": n, "ms_per_step": ms} for n, ms in lat]}
+        if args.tau:
+            from paper_2405_18628_gb300 import tree_profile as tp_
+            with open(args.tau) as f:
+                tau = {int(k): float(v) for k, v in json.load(f).items()}
+            rows, best = tp_.speedup_table(tau, lat)
+            profile["speedup"] = rows
+            profile["best_tree_size"] = best
+
+    clocks.stop()
+    clk = clocks.summary(windows.spans)
+
     kernel = "tree_attention_kernel" if w.T <= 64 else "tree_attention_rows_kernel"
     alone = {"kernel": kernel, "launch_us": att_ms * 1e3, "bytes_per_launch": att_bytes,
              "achieved": achieved, "frac": achieved / peak}
@@ -593,23 +805,16 @@ def main():
     roof["frac"] = roof["achieved"] / peak
     roof["peak_kind"] = peak_kind
     roof["frac_of_8000"] = roof["achieved"] / NOMINAL_HBM_GBS
+    if traffic is not None:
+        roof["traffic_note"] = ("ncu dram__bytes_read.sum + dram__bytes_write.sum of a 19-layer "
+                                "capture scaled to all layers; output writes still in L2 at "
+                                "kernel end are not counted")
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": w.name + (f" ({w.L} layers)" if args.layers else ""),
-                       "layers": w.L, "batch": w.B, "heads": w.H,
-                       "head_dim": w.D, "prefix": w.P, "tree_tokens": w.T, "vocab": w.V,
-                       "S_max": w.S_max,
-                       "l2": ("flushed before every step (256 MiB write, outside the step events)"
-                              if do_flush else
-                              f"not flushed: inputs larger than L2 ({footprint / 1e6:.0f} MB "
-                              f"streamed per step, L2 {L2_BYTES / 1e6:.0f} MB)"),
-                       "parallelism": f"replicas x{world}",
-                       "accept": ("exact matching" if args.accept == "exact" else
-                                  "typical acceptance (temperature %g, epsilon %g, delta %g)"
-                                  % TYPICAL)},
+            "config": config_of(w, args, world),
             "ms_per_step_p10_p50_p90": [float(q10), float(q50), float(q90)],
             "step_gbs": sb / (ms_per_step * 1e-3) / 1e9,
             "step_frac_of_8tbs": sb / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
@@ -622,12 +827,14 @@ def main():
             "cpu_baseline": cpu,
             "wall_s_timed": wall,
         }
+        if others is not None:
+            line["workloads"] = others
+        if per_layer is not None:
+            line["per_layer_attention"] = per_layer
         if profile is not None:
             line["tree_size_profile"] = profile
         if next_tree is not None:
             line["next_tree"] = next_tree
-        if per_layer is not None:
-            line["per_layer_attention"] = per_layer
         print(json.dumps(line), flush=True)
     if pg:
         pg.barrier()

@@ -9,13 +9,13 @@
  *
  *   1. tree-masked attention: every tree token attends to the KV-cache prefix,
  *      its tree ancestors and itself (Section 3, step (1), tree attention;
- *      Section 4.1, the attention mask over the tree-structured input);
+ *      Section 4.1, the tree attention mask);
  *   2. node argmax: the model's top-1 token after every tree node (the greedy
- *      "exact matching" check of Section 3, step (2));
+ *      exact-matching check of Section 3, step (2));
  *   3. acceptance: the longest root-to-node path whose every candidate equals
  *      the top-1 token at its parent (Section 3, steps (2)-(3));
  *   4. compaction: the accepted nodes' K/V rows enter the cache (Section 3,
- *      step (3), "KV cache is updated accordingly").
+ *      step (3): the accepted rows are appended to the cache).
  *
  * Conventions shared by every entry point
  * ---------------------------------------
@@ -163,8 +163,11 @@ ppd_status ppd_kv_compact(void *k_cache, void *v_cache, const void *k_tree, cons
  * ppd_tree_attention, `argmax_out` as in ppd_node_argmax.  Attention reads
  * only prefix rows [0, prefix_len[b]) and compaction writes only rows
  * [prefix_len[b], new_prefix_len[b]), so the result equals running the four
- * steps one after another.  After a call that reported PPD_ERR_TIMEOUT, fill
- * the workspace with zeros before reusing it.
+ * steps one after another.  The epoch word and the flags sit in the first
+ * 2,064 bytes of the workspace at the same place for every size, so a
+ * workspace may be reused across sizes (a flag only ever holds the tag of an
+ * earlier call, below the next call's).  After a call that reported
+ * PPD_ERR_TIMEOUT, fill the workspace with zeros before reusing it.
  */
 ppd_status ppd_verify_step(const void *q, void *k_cache, void *v_cache,
                            const void *k_tree, const void *v_tree,

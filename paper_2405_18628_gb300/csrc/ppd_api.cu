@@ -49,8 +49,9 @@ int num_sms()
 
 int argmax_splits(int64_t rows, int V) { return ppd::argmax_split_count(rows, V); }
 
-// Workspace: the argmax partials, the side warp's scratch, the bf16 copies of
-// fp32 operands, then the work split's per-CTA records and partial states.
+// Workspace: the in-grid argmax's sync words, the argmax partials, the side
+// warp's scratch, the bf16 copies of fp32 operands, then the work split's
+// per-CTA records and partial states.
 struct WsLayout {
     size_t part_val, part_idx, part_stats, node_lse, node_ent, side, sync, conv, split_rec,
         split_part, total;
@@ -93,6 +94,11 @@ WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, p
     const int64_t rows = (int64_t)B * T;
     w.splits = argmax_splits(rows, V);
     size_t off = 0;
+    // the in-grid argmax's epoch and all-ready words and per-CTA flags first, at
+    // the same offset for every size: a workspace reused for another shape
+    // keeps them in place, so its flags only ever hold tags of earlier calls
+    w.sync = off;
+    off = align_up(off + (size_t)(2 + ppd::kSplitMaxGrid) * 8);
     w.part_val = off;
     off = align_up(off + (size_t)rows * w.splits * 4);
     w.part_idx = off;
@@ -105,8 +111,6 @@ WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, p
     off = align_up(off + (size_t)rows * 4);
     w.side = off;
     off = align_up(off + (size_t)num_sms() * ppd::kSideScratchInts * 4);
-    w.sync = off;   // the in-grid argmax's epoch and all-ready words, per-CTA flags
-    off = align_up(off + (size_t)(2 + ppd::kSplitMaxGrid) * 8);
     w.conv = off;
     if (dt == PPD_F32) {
         const size_t lbh = (size_t)L * B * H;

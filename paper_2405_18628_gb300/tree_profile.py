@@ -33,10 +33,13 @@ def tree_size_workload(base: W.Workload, n: int) -> W.Workload:
 
 
 def measure_step_latency(w: W.Workload, steps: int = 30, warmup: int = 5, device="cuda",
-                         flush_bytes: int = 0) -> float:
+                         flush_bytes: int = 0, timed=None) -> float:
     """Median device time (ms) of ppd_verify_step on workload `w`, CUDA events
     on the current stream, `warmup` untimed steps first.  With flush_bytes > 0
-    a buffer of that size is written before every step (outside the events)."""
+    a buffer of that size is written before every step (outside the events).
+    `timed`, when given, is a context manager entered around the timed loop."""
+    import contextlib
+
     import torch
 
     from . import ppd
@@ -63,13 +66,15 @@ def measure_step_latency(w: W.Workload, steps: int = 30, warmup: int = 5, device
         step()
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(steps)]
-    for a, b in ev:
-        if flush is not None:
-            flush.zero_()
-        a.record(stream)
-        step()
-        b.record(stream)
     torch.cuda.synchronize()
+    with (timed if timed is not None else contextlib.nullcontext()):
+        for a, b in ev:
+            if flush is not None:
+                flush.zero_()
+            a.record(stream)
+            step()
+            b.record(stream)
+        torch.cuda.synchronize()
     status = bufs.dev_status.cpu().numpy()
     if (status != 0).any():
         raise RuntimeError(f"verification step reported device status {status.tolist()}")
@@ -80,11 +85,11 @@ def measure_step_latency(w: W.Workload, steps: int = 30, warmup: int = 5, device
 
 
 def latency_profile(base: W.Workload, sizes: Iterable[int], steps: int = 30, warmup: int = 5,
-                    device="cuda", flush_bytes: int = 0) -> List[Tuple[int, float]]:
+                    device="cuda", flush_bytes: int = 0, timed=None) -> List[Tuple[int, float]]:
     """L_fp(n) of the verification step on this GPU for each tree size n, as
     (n, median ms per step) pairs in the order given."""
     return [(int(n), measure_step_latency(tree_size_workload(base, int(n)), steps, warmup,
-                                          device, flush_bytes))
+                                          device, flush_bytes, timed))
             for n in sizes]
 
 

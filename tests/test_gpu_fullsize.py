@@ -93,3 +93,74 @@ def test_full_size_step(cuda_device, name):
         r2 += float(np.sum(ref ** 2))
     rel = np.sqrt(d2 / r2)
     assert err <= ATOL and rel <= RTOL_L2, (layers, err, rel)
+
+
+def _plant_ties(logits, chunk):
+    """Rows of one sequence's logits rewritten with ties, NaNs, infinities and
+    signed zeros, many of them straddling the boundaries of the argmax's
+    per-row chunks (columns k*chunk - 1 | k*chunk)."""
+    T, V = logits.shape
+    n_b = max(1, (V - 1) // chunk)
+    for r in range(min(T, 7)):                           # max tied across a boundary
+        k = 1 + r % n_b
+        m = logits[r].max() + 1.0
+        logits[r, [k * chunk, k * chunk - 1]] = m
+    for r in range(7, min(T, 14)):                       # two NaNs either side of a boundary
+        k = 1 + r % n_b
+        logits[r, [k * chunk, k * chunk - 1]] = np.nan
+    for r in range(14, min(T, 21)):                      # +inf in two chunks
+        k = 1 + r % n_b
+        logits[r, [k * chunk + 3, (k - 1) * chunk + 1]] = np.inf
+    if T > 21:
+        logits[21, :] = -np.inf                          # all equal: index 0
+    if T > 22:
+        logits[22, :] = -2.0
+        logits[22, [chunk, chunk - 1]] = [0.0, -0.0]     # -0 == +0
+    if T > 23:
+        logits[23, V - 1] = np.nan                       # the only NaN, last column
+    if T > 24:
+        m = logits[24].max() + 0.5
+        logits[24, [V - 1, 2 * chunk, chunk]] = m        # three-way tie
+
+
+@pytest.mark.parametrize("name", ["mobilellama", "vicuna7b"])
+def test_full_size_step_argmax_ties(cuda_device, name):
+    """The fused step at full size (its in-grid side-warp argmax at Vicuna-7B
+    shapes, the argmax grid at MobileLlama shapes) with ties, NaNs, +-inf and
+    signed zeros planted across the per-row argmax chunks: every index output
+    and the compacted cache rows bit for bit against the oracle."""
+    w = W.WORKLOADS[name]
+    s = W.make_step_inputs(w)
+    lg = s.logits.copy()
+    for b in range(w.B):
+        _plant_ties(lg[b], 4000)
+    am = oracle.node_argmax(lg)
+    # candidates that copied their parent's planted top token now copy the new argmax
+    cand = s.cand_tokens.copy()
+    for b in range(w.B):
+        for i in range(1, w.T):
+            pa = s.parent[b, i]
+            if cand[b, i] >= 0 and cand[b, i] == s.top[b, pa]:
+                cand[b, i] = am[b, pa]
+    t = W.make_tensors(w, device=cuda_device)
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(cuda_device)
+    bufs = ppd.StepBuffers(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max, device=cuda_device)
+    ppd.ppd_verify_step(t["q"], t["k_cache"], t["v_cache"], t["k_tree"], t["v_tree"],
+                        i32(s.prefix_len), i32(s.parent), i32(cand),
+                        torch.from_numpy(lg).to(cuda_device), bufs.out, bufs.argmax,
+                        bufs.accept_len, bufs.path, bufs.next_token, bufs.new_prefix_len,
+                        bufs.dev_status, bufs.workspace)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(bufs.argmax.cpu().numpy(), am)
+    acc = oracle.accept_path(am, cand, s.parent, s.prefix_len, w.V, w.S_max)
+    for k in ("accept_len", "path", "next_token", "new_prefix_len"):
+        np.testing.assert_array_equal(getattr(bufs, k).cpu().numpy(), acc[k], err_msg=k)
+    np.testing.assert_array_equal(bufs.dev_status.cpu().numpy(), acc["status"])
+    assert (acc["accept_len"] > 1).any()          # the rewritten rows still accept paths
+    for b in range(w.B):
+        n, P = int(acc["accept_len"][b]), int(s.prefix_len[b])
+        src = torch.from_numpy(acc["path"][b, :n].astype(np.int64)).to(cuda_device)
+        for k, kt in (("k_cache", "k_tree"), ("v_cache", "v_tree")):
+            got = t[k][:, b, :, P:P + n].view(torch.int16)
+            want = t[kt][:, b, :, :][:, :, src].view(torch.int16)
+            assert torch.equal(got, want), (k, b)

@@ -134,6 +134,21 @@ def test_in_grid_junk_workspace(cuda_device):
             _check(w, s, t, g, bufs, ref, f"fill {fill} call {rep}")
 
 
+def test_in_grid_workspace_reused_across_shapes(cuda_device):
+    """One workspace (sized for the largest) serving in-grid steps of different
+    shapes in turn: the epoch word and flags stay at the workspace's start for
+    every shape, so no call sees stale flags of another shape's layout."""
+    names = ["rows_t285", "keyrow_roundrobin", "batch64", "keyrow_split_v301", "rows_t285"]
+    n = max(ppd.ppd_workspace_bytes(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max)
+            for w, _ in (CASES[k] for k in names))
+    ws = torch.zeros(n, dtype=torch.uint8, device=cuda_device)
+    for i, name in enumerate(names):
+        w, pl = CASES[name]
+        s, t = _inputs(w, pl)
+        g, bufs = _run(w, s, t, cuda_device, ws=ws)
+        _check(w, s, t, g, bufs, _ref(s, t), f"{name} (call {i})")
+
+
 def test_in_grid_calls_back_to_back(cuda_device):
     """Different steps through one workspace, enqueued without host syncs in
     between: each sees only its own argmax partials."""
