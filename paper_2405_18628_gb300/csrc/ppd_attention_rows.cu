@@ -27,8 +27,9 @@
 // tile, and that unit's first PV product waits for the readback.  The unit
 // walk (with the work split), the fused step's side warp and the merge of a
 // cut unit's partial states are those of the kernel for trees of up to 64
-// tokens (ppd_attention.cu); the warp roles (384 threads) differ in one
-// point: warp 8 loads Q and K, warp 11 loads V.
+// tokens (ppd_attention.cu), and so are the warp roles (352 threads), except
+// that the producer queues each V tile two tiles behind its K tile, the order
+// in which the MMA issuer consumes them.
 #include "ppd_attention_common.cuh"
 
 #include <cmath>
@@ -82,7 +83,7 @@ struct RowsLayout {
 };
 
 template <int D, bool SPLIT>
-__global__ void __launch_bounds__(384, 1)
+__global__ void __launch_bounds__(352, 1)
 tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
                            const __grid_constant__ CUtensorMap map_kc,
                            const __grid_constant__ CUtensorMap map_vc,
@@ -138,80 +139,84 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
     if (warp == 10) {
         // ------------------------------------------------------------ fused-step side work
         if (p.fused) fused_side_warp(p, wr, lane, abort_flag);
-    } else if (warp == 8 || warp == 11) {
-        // ------------------------------------------------------------ TMA producers
-        // warp 8 loads Q and the K tiles, warp 11 the V tiles: a V slot is released
-        // only by its PV product, so the K stream never queues behind it.
+    } else if (warp == 8) {
+        // ------------------------------------------------------------ TMA producer
+        // One queue of copies in the order the MMA issuer consumes them -- S(g)
+        // then PV(g - 2) -- so each tile's V follows the K tile two tiles later:
+        // Q(unit), K(g), V(g - 2), K(g + 1), V(g - 1), ...  An SM's copies land
+        // roughly in issue order, so a V tile queued ahead of its turn would
+        // hold back the K tile the next score product waits for, and vice versa.
         if (lane == 0) {
-            const bool kq = (warp == 8);
-            if (kq) {
-                tma_prefetch_map(&map_q);
-                tma_prefetch_map(&map_kc);
-                tma_prefetch_map(&map_kt);
-            } else {
-                tma_prefetch_map(&map_vc);
-                tma_prefetch_map(&map_vt);
-            }
+            tma_prefetch_map(&map_q);
+            tma_prefetch_map(&map_kc);
+            tma_prefetch_map(&map_kt);
+            tma_prefetch_map(&map_vc);
+            tma_prefetch_map(&map_vt);
             const uint64_t pol = l2_policy_evict_first();
-            int g = 0, k = 0;
+            constexpr int LAG = 2;
+            int v_row[LAG + 1], v_lbh[LAG + 1];
+            bool v_tree[LAG + 1];
+            int g = 0, gv = 0, k = 0;
+            auto load_v = [&]() {   // V tile gv (its coordinates queued when K(gv) was loaded)
+                const int i = gv % (LAG + 1);
+                const int vs = gv % Lay::VS;
+                if (gv >= Lay::VS)
+                    mbar_wait(bars + Lay::B_VEMPTY + vs, ((gv / Lay::VS) - 1) & 1, abort_flag);
+                if (!*abort_flag) {
+                    mbar_arrive_expect_tx(bars + Lay::B_VFULL + vs, Lay::TILE_BYTES);
+#pragma unroll
+                    for (int c = 0; c < Lay::DCH; ++c)
+                        tma_load_3d(smem + Lay::OFF_V + vs * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                    v_tree[i] ? &map_vt : &map_vc, bars + Lay::B_VFULL + vs, c * 64,
+                                    v_row[i], v_lbh[i], pol);
+                }
+                ++gv;
+            };
             SegIter<SPLIT> it(wr);
             for (Seg sg; it.next(p, sg); ++k) {
                 const UnitInfo &ui = sg.ui;
                 const int qs = k % Lay::QS;
-                if (kq) {
-                    if (k >= Lay::QS)
-                        mbar_wait(bars + Lay::B_QEMPTY + qs, ((k / Lay::QS) - 1) & 1, abort_flag);
-                    if (!*abort_flag) {
-                        // rows T..127 of the box lie beyond the tensor and arrive as zeros
-                        mbar_arrive_expect_tx(bars + Lay::B_QFULL + qs, Lay::Q_BYTES);
+                if (k >= Lay::QS)
+                    mbar_wait(bars + Lay::B_QEMPTY + qs, ((k / Lay::QS) - 1) & 1, abort_flag);
+                if (!*abort_flag) {
+                    // rows T..127 of the box lie beyond the tensor and arrive as zeros
+                    mbar_arrive_expect_tx(bars + Lay::B_QFULL + qs, Lay::Q_BYTES);
 #pragma unroll
-                        for (int c = 0; c < Lay::DCH; ++c)
-                            tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::GROUP_BYTES,
-                                        &map_q, bars + Lay::B_QFULL + qs, c * 64, ui.qb * Lay::M,
-                                        ui.lbh, pol);
-                    }
+                    for (int c = 0; c < Lay::DCH; ++c)
+                        tma_load_3d(smem + Lay::OFF_Q + qs * Lay::Q_BYTES + c * Lay::GROUP_BYTES,
+                                    &map_q, bars + Lay::B_QFULL + qs, c * 64, ui.qb * Lay::M,
+                                    ui.lbh, pol);
                 }
                 for (int j = sg.j0; j < sg.j1; ++j, ++g) {
                     const bool tree = (j >= ui.n_pref);
                     const int row = (tree ? j - ui.n_pref : j) * Lay::KT;
-                    if (kq) {
-                        const int ks = g % Lay::KS;
-                        if (g >= Lay::KS)
-                            mbar_wait(bars + Lay::B_KEMPTY + ks, ((g / Lay::KS) - 1) & 1, abort_flag);
-                        if (!*abort_flag) {
-                            mbar_arrive_expect_tx(bars + Lay::B_KFULL + ks, Lay::TILE_BYTES);
+                    const int ks = g % Lay::KS;
+                    if (g >= Lay::KS)
+                        mbar_wait(bars + Lay::B_KEMPTY + ks, ((g / Lay::KS) - 1) & 1, abort_flag);
+                    if (!*abort_flag) {
+                        mbar_arrive_expect_tx(bars + Lay::B_KFULL + ks, Lay::TILE_BYTES);
 #pragma unroll
-                            for (int c = 0; c < Lay::DCH; ++c)
-                                tma_load_3d(smem + Lay::OFF_K + ks * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
-                                            tree ? &map_kt : &map_kc, bars + Lay::B_KFULL + ks, c * 64,
-                                            row, ui.lbh, pol);
-                        }
-                    } else {
-                        const int vs = g % Lay::VS;
-                        if (g >= Lay::VS)
-                            mbar_wait(bars + Lay::B_VEMPTY + vs, ((g / Lay::VS) - 1) & 1, abort_flag);
-                        if (!*abort_flag) {
-                            mbar_arrive_expect_tx(bars + Lay::B_VFULL + vs, Lay::TILE_BYTES);
-#pragma unroll
-                            for (int c = 0; c < Lay::DCH; ++c)
-                                tma_load_3d(smem + Lay::OFF_V + vs * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
-                                            tree ? &map_vt : &map_vc, bars + Lay::B_VFULL + vs, c * 64,
-                                            row, ui.lbh, pol);
-                        }
+                        for (int c = 0; c < Lay::DCH; ++c)
+                            tma_load_3d(smem + Lay::OFF_K + ks * Lay::TILE_BYTES + c * Lay::GROUP_BYTES,
+                                        tree ? &map_kt : &map_kc, bars + Lay::B_KFULL + ks, c * 64,
+                                        row, ui.lbh, pol);
                     }
+                    const int i = g % (LAG + 1);
+                    v_row[i] = row;
+                    v_lbh[i] = ui.lbh;
+                    v_tree[i] = tree;
+                    if (g >= LAG) load_v();
                 }
             }
+            while (gv < g) load_v();
             if (*abort_flag) {
                 // let every copy already issued land before the CTA can exit
-                if (kq) {
-                    for (int i = max(0, g - Lay::KS); i < g; ++i)
-                        mbar_wait_drain(bars + Lay::B_KFULL + i % Lay::KS, (i / Lay::KS) & 1);
-                    for (int i = max(0, k - Lay::QS); i < k; ++i)
-                        mbar_wait_drain(bars + Lay::B_QFULL + i % Lay::QS, (i / Lay::QS) & 1);
-                } else {
-                    for (int i = max(0, g - Lay::VS); i < g; ++i)
-                        mbar_wait_drain(bars + Lay::B_VFULL + i % Lay::VS, (i / Lay::VS) & 1);
-                }
+                for (int i = max(0, g - Lay::KS); i < g; ++i)
+                    mbar_wait_drain(bars + Lay::B_KFULL + i % Lay::KS, (i / Lay::KS) & 1);
+                for (int i = max(0, k - Lay::QS); i < k; ++i)
+                    mbar_wait_drain(bars + Lay::B_QFULL + i % Lay::QS, (i / Lay::QS) & 1);
+                for (int i = max(0, gv - Lay::VS); i < gv; ++i)
+                    mbar_wait_drain(bars + Lay::B_VFULL + i % Lay::VS, (i / Lay::VS) & 1);
             }
         }
     } else if (warp == 9) {
@@ -307,6 +312,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
         const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
         const float sl2 = p.scale_log2;
         const bool vec_out = (reinterpret_cast<uintptr_t>(p.out) & 15u) == 0;
+        const bool out32 = (reinterpret_cast<uintptr_t>(p.out) & 31u) == 0;
 
         float m = -INFINITY;    // running maximum of the row (log2 units), same in both threads
         float l = 0.f;          // this thread's share of the row sum
@@ -386,22 +392,30 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             const uint32_t t_o = tmem_base + lane_off + Lay::T_O + (uint32_t)h * (D / 2);
             const int qg = qb_out * Lay::M + q;
             float *orow = p.out + ((size_t)lbh_out * T + qg) * D + h * (D / 2);
+            // the half row in two round trips to TMEM, then full-sector stores
+            uint32_t r[2][16];
 #pragma unroll
-            for (int ch = 0; ch < D / 32; ++ch) {
-                uint32_t r[16];
-                tmem_ld16(t_o + ch * 16, r);
+            for (int c2 = 0; c2 < D / 32; c2 += 2) {
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch) tmem_ld16(t_o + (c2 + ch) * 16, r[ch]);
                 tmem_wait_ld();
-                if (qg < T) {
-                    if (vec_out) {
+                if (qg >= T) continue;
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch) {
+                    if (out32) {
+#pragma unroll
+                        for (int e = 0; e < 16; e += 8)
+                            st_global_v8(orow + (c2 + ch) * 16 + e, r[ch] + e, linv);
+                    } else if (vec_out) {
 #pragma unroll
                         for (int e = 0; e < 16; e += 4)
-                            *reinterpret_cast<float4 *>(orow + ch * 16 + e) =
-                                make_float4(__uint_as_float(r[e]) * linv, __uint_as_float(r[e + 1]) * linv,
-                                            __uint_as_float(r[e + 2]) * linv,
-                                            __uint_as_float(r[e + 3]) * linv);
+                            *reinterpret_cast<float4 *>(orow + (c2 + ch) * 16 + e) =
+                                make_float4(__uint_as_float(r[ch][e]) * linv, __uint_as_float(r[ch][e + 1]) * linv,
+                                            __uint_as_float(r[ch][e + 2]) * linv,
+                                            __uint_as_float(r[ch][e + 3]) * linv);
                     } else {
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) orow[ch * 16 + e] = __uint_as_float(r[e]) * linv;
+                        for (int e = 0; e < 16; ++e) orow[(c2 + ch) * 16 + e] = __uint_as_float(r[ch][e]) * linv;
                     }
                 }
             }
@@ -412,7 +426,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
         // Partial state of a cut unit into slot `slot`: this thread's half of the
         // row of O unnormalised, and (h == 0) the row's maximum and sum; then O
-        // is free.
+        // is free.  Slots are 256-byte aligned rows of D floats.
         const size_t slot_floats = split_slot_floats(D);
         auto write_partial = [&](int slot, int qb_out, int g_last, float rm, float rl) {
             mbar_wait(bars + Lay::B_PDONE + g_last % Lay::NSB, (g_last / Lay::NSB) & 1, abort_flag);
@@ -421,17 +435,18 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             float *base = p.split_part + (size_t)slot * slot_floats;
             float *orow = base + (size_t)q * D + h * (D / 2);
             const bool live = qb_out * Lay::M + q < T;
+            uint32_t r[2][16];
 #pragma unroll
-            for (int ch = 0; ch < D / 32; ++ch) {
-                uint32_t r[16];
-                tmem_ld16(t_o + ch * 16, r);
+            for (int c2 = 0; c2 < D / 32; c2 += 2) {
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch) tmem_ld16(t_o + (c2 + ch) * 16, r[ch]);
                 tmem_wait_ld();
                 if (live) {
 #pragma unroll
-                    for (int e = 0; e < 16; e += 4)
-                        *reinterpret_cast<float4 *>(orow + ch * 16 + e) =
-                            make_float4(__uint_as_float(r[e]), __uint_as_float(r[e + 1]),
-                                        __uint_as_float(r[e + 2]), __uint_as_float(r[e + 3]));
+                    for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                        for (int e = 0; e < 16; e += 8)
+                            st_global_v8(orow + (c2 + ch) * 16 + e, r[ch] + e, 1.f);
                 }
             }
             if (h == 0 && live) {
@@ -625,9 +640,9 @@ static cudaError_t launch_rows_t(const AttnMaps &m, const AttnParams &p, int num
 {
     static std::atomic<uint64_t> configured[2] = {{0}, {0}};
     if (p.split)
-        return launch_attention_grid(tree_attention_rows_kernel<D, true>, RowsLayout<D>::SMEM_BYTES, 384,
+        return launch_attention_grid(tree_attention_rows_kernel<D, true>, RowsLayout<D>::SMEM_BYTES, 352,
                                      configured[1], m, p, num_sms, programmatic, stream);
-    return launch_attention_grid(tree_attention_rows_kernel<D, false>, RowsLayout<D>::SMEM_BYTES, 384,
+    return launch_attention_grid(tree_attention_rows_kernel<D, false>, RowsLayout<D>::SMEM_BYTES, 352,
                                  configured[0], m, p, num_sms, programmatic, stream);
 }
 

@@ -149,6 +149,18 @@ PPD_DEV void st_relaxed_gpu(unsigned long long *p, unsigned long long v)
 PPD_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 PPD_DEV void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
+// 32-byte store of eight fp32 values (bit patterns v[0..7]) times `scale` to a
+// 32-byte aligned global address: one full sector per thread.
+PPD_DEV void st_global_v8(float *dst, const uint32_t *v, float scale)
+{
+    asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst),
+                 "f"(__uint_as_float(v[0]) * scale), "f"(__uint_as_float(v[1]) * scale),
+                 "f"(__uint_as_float(v[2]) * scale), "f"(__uint_as_float(v[3]) * scale),
+                 "f"(__uint_as_float(v[4]) * scale), "f"(__uint_as_float(v[5]) * scale),
+                 "f"(__uint_as_float(v[6]) * scale), "f"(__uint_as_float(v[7]) * scale)
+                 : "memory");
+}
+
 // ---------------------------------------------------------------- TMA
 
 PPD_DEV void tma_prefetch_map(const CUtensorMap *map)
