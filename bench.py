@@ -318,6 +318,9 @@ def parse(argv=None):
                     help="time the per-layer attention even when extras are off")
     ap.add_argument("--layers", type=int, default=0,
                     help="run the workload with this many layers (profiling captures)")
+    ap.add_argument("--form", type=int, default=None, choices=[1, 2, 3],
+                    help="force the fused step's form (1: argmax grid first; 2: argmax in the "
+                         "side warps; 3: argmax in the softmax warps before their first tile)")
     ap.add_argument("--l2", default="auto", choices=["auto", "flush", "none"],
                     help="auto: flush L2 before each step unless the step's inputs exceed 4x L2")
     return ap.parse_args(argv)
@@ -595,6 +598,8 @@ def main(argv=None):
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
     ppd.load()
+    if args.form is not None:
+        ppd.ppd_set_verify_step_form(args.form)
     extras = world == 1 and not args.no_extras and not args.layers
     clocks = ClockSampler(local).start()
     windows = Windows()
@@ -823,6 +828,7 @@ def main(argv=None):
             "attention_alone": alone,
             "e2e": e2e,
             "gpu_launches": n_launch * K,
+            "form": ppd.ppd_verify_step_form(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max),
             "clocks": clk,
             "cpu_baseline": cpu,
             "wall_s_timed": wall,

@@ -305,6 +305,34 @@ ppd_status ppd_node_argmax_noalloc(const float *logits, int B, int T, int V, int
 int ppd_verify_step_launches(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt,
                              int typical);
 
+/*
+ * The form a ppd_verify_step (or _typical) call takes for these sizes, with a
+ * workspace of ppd_workspace_bytes(...) bytes and the whole GPU available
+ * (no paper counterpart; for tests and benchmarks):
+ *   0  B > 64: argmax, acceptance, attention and compaction as separate grids;
+ *   1  an argmax grid, then the attention grid (which accepts and compacts);
+ *   2  one attention grid whose spare warp per CTA also computes the argmax
+ *      partial maxima while the K/V stream runs (chosen when the logits are
+ *      at most 1/64 of the K/V bytes and form 3 does not fit);
+ *   3  one attention grid whose softmax warps compute the argmax partial
+ *      maxima before their first tile (chosen when the logits are at most
+ *      128 KB per CTA of the attention grid).
+ * Forms 2 and 3 fall back to form 1 when the cooperative launch cannot have
+ * every CTA resident.  Returns -1 for sizes the step rejects.
+ */
+int ppd_verify_step_form(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt);
+
+/*
+ * Force the form of every later fused step of this process (B <= 64): 1, 2
+ * or 3 as above, or -1 to return to the automatic choice.  The forms compute
+ * the same results; this exists so that tests can cover each one at any size
+ * and benchmarks can compare them (no paper counterpart).  Returns the
+ * previous setting, or -2 (and changes nothing) for any other value.  Not
+ * synchronised with steps already enqueued; set it while none is being
+ * enqueued from another thread.
+ */
+int ppd_set_verify_step_form(int form);
+
 /* Human-readable name of a status code (static string). */
 const char *ppd_status_string(ppd_status s);
 

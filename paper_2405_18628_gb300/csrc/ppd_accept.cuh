@@ -247,4 +247,69 @@ PPD_DEV AcceptResult accept_warp_typical(TopLoad top, const float *x, Lse lse, E
         par, tok, P, T, V, S_max, lane, s_par, path);
 }
 
+// ------------------------------------------------------------------ logits scan
+
+// Top-1 (and with kStats the softmax statistics) of columns [lo, hi) of the
+// logits row x by one warp, with kDepth 16-byte loads per lane issued before
+// any is used (predicated at the end of the span, so a span of n float4 takes
+// ceil(n / (32 kDepth)) round trips); lane 0 holds the result.
+template <bool kStats, int kDepth>
+PPD_DEV void warp_logit_span(const float *x, int lo, int hi, bool vec, float stat_k, int lane,
+                             float &bv, int &bi, SoftStats &st)
+{
+    bv = -INFINITY;
+    bi = INT_MAX;
+    st = SoftStats{};
+    if (vec) {
+        const float4 *x4 = reinterpret_cast<const float4 *>(x);
+        const int n4_hi = hi >> 2;
+        for (int i = (lo >> 2) + lane; i < n4_hi; i += kDepth * 32) {
+            float4 f[kDepth];
+#pragma unroll
+            for (int k = 0; k < kDepth; ++k)
+                if (i + k * 32 < n4_hi) f[k] = __ldcs(x4 + i + k * 32);
+#pragma unroll
+            for (int k = 0; k < kDepth; ++k) {
+                if (i + k * 32 < n4_hi) {
+                    const int base = 4 * (i + k * 32);
+                    consider(f[k].x, base, bv, bi);
+                    consider(f[k].y, base + 1, bv, bi);
+                    consider(f[k].z, base + 2, bv, bi);
+                    consider(f[k].w, base + 3, bv, bi);
+                    if (kStats)
+                        stats_add4(st, f[k].x * stat_k, f[k].y * stat_k, f[k].z * stat_k,
+                                   f[k].w * stat_k);
+                }
+            }
+        }
+    } else {
+        for (int i = lo + lane; i < hi; i += kDepth * 32) {
+            float v[kDepth];
+#pragma unroll
+            for (int k = 0; k < kDepth; ++k)
+                if (i + k * 32 < hi) v[k] = __ldcs(x + i + k * 32);
+#pragma unroll
+            for (int k = 0; k < kDepth; ++k) {
+                if (i + k * 32 < hi) {
+                    consider(v[k], i + k * 32, bv, bi);
+                    if (kStats) stats_add4(st, v[k] * stat_k, -INFINITY, -INFINITY, -INFINITY);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float ov = __shfl_down_sync(0xffffffffu, bv, off);
+        const int oi = __shfl_down_sync(0xffffffffu, bi, off);
+        consider(ov, oi, bv, bi);
+        if (kStats) {
+            SoftStats o;
+            o.m = __shfl_down_sync(0xffffffffu, st.m, off);
+            o.s = __shfl_down_sync(0xffffffffu, st.s, off);
+            o.t = __shfl_down_sync(0xffffffffu, st.t, off);
+            stats_merge(st, o);
+        }
+    }
+}
+
 }  // namespace ppd

@@ -10,6 +10,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <atomic>
 #include <cstring>
 #include <mutex>
 
@@ -88,6 +89,30 @@ bool in_grid_argmax_pays(int L, int B, int H, int T, int D, int V, int S_max)
     return logits * PPD_IN_GRID_MIN_RATIO <= kv;
 }
 
+// Forms of the fused step (ppd_verify_step_form): separate grids for large
+// batches; an argmax grid then the attention grid; one grid whose side warps
+// compute the argmax partials while the K/V stream runs.
+enum FusedForm { kFormGrids = 0, kFormTwoGrids = 1, kFormSide = 2 };
+
+// A form forced by ppd_set_verify_step_form (-1: chosen by the rules below).
+std::atomic<int> g_forced_form{-1};
+
+int narrow_argmax_grid(int L, int B, int H, int T, int D, int V, int S_max);
+
+// The form of a fused step (B <= kFusedMaxB) of these sizes: an argmax grid
+// first when it fits on the idle SMs of the attention grid's last, partial
+// round (measured at Vicuna-7B shapes: 181.9 us against 183.2 us with the
+// side warps; equal at Vicuna-13B and on the batch-8 sweep), else the side
+// warps when the logits are a small enough share of the K/V bytes, else an
+// argmax grid over every SM.
+int choose_form(int L, int B, int H, int T, int D, int V, int S_max)
+{
+    const int forced = g_forced_form.load(std::memory_order_relaxed);
+    if (forced >= kFormTwoGrids) return forced;
+    if (narrow_argmax_grid(L, B, H, T, D, V, S_max) > 0) return kFormTwoGrids;
+    return in_grid_argmax_pays(L, B, H, T, D, V, S_max) ? kFormSide : kFormTwoGrids;
+}
+
 WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt)
 {
     WsLayout w{};
@@ -99,12 +124,13 @@ WsLayout workspace_layout(int L, int B, int H, int T, int D, int V, int S_max, p
     // keeps them in place, so its flags only ever hold tags of earlier calls
     w.sync = off;
     off = align_up(off + (size_t)(2 + ppd::kSplitMaxGrid) * 8);
+    const size_t cap = (size_t)rows * (size_t)w.splits;
     w.part_val = off;
-    off = align_up(off + (size_t)rows * w.splits * 4);
+    off = align_up(off + cap * 4);
     w.part_idx = off;
-    off = align_up(off + (size_t)rows * w.splits * 4);
+    off = align_up(off + cap * 4);
     w.part_stats = off;   // softmax statistics partials (typical acceptance)
-    off = align_up(off + (size_t)rows * w.splits * 12);
+    off = align_up(off + cap * 12);
     w.node_lse = off;
     off = align_up(off + (size_t)rows * 4);
     w.node_ent = off;
@@ -300,6 +326,32 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
                              scale, out, lse, dev_status, ws, &wl, fused, false, stream);
 }
 
+// Blocks of the fused step's narrow argmax grid (0: use the wide grid).  When
+// the attention grid's slices do not fill whole rounds, the CTAs of the last,
+// partial round that hold one slice fewer -- grid - (n_units mod grid) of
+// them -- have a slice's time to spare; the argmax blocks take as many SMs
+// (at most half of them), the CTAs dispatched last, which are those, wait for
+// them, and nothing on the critical path does.  Each block's share of the
+// logits must then be at most half a slice's K/V bytes (S_max standing in for
+// the device-side prefix lengths).  The work split (fewer slices than SMs)
+// leaves no CTA with time to spare.
+int narrow_argmax_grid(int L, int B, int H, int T, int D, int V, int S_max)
+{
+    if (attention_splits(L, B, H, T, S_max)) return 0;
+    const int T_pad = (T + 31) & ~31;
+    const long long n_qb = T_pad > 64 ? (T + 127) / 128 : 1;
+    const long long n_units = (long long)L * B * H * n_qb;
+    const long long grid = n_units < split_grid() ? n_units : split_grid();
+    const long long r = n_units % grid;
+    if (r == 0) return 0;
+    long long g = grid - r;
+    if (g > num_sms() / 2) g = num_sms() / 2;
+    if (g < 8) return 0;
+    const double logits = 4.0 * B * (double)T * V;
+    const double slice = 4.0 * ((double)S_max + T) * D;
+    return logits / (double)g <= slice / 2 ? (int)g : 0;
+}
+
 }  // namespace
 
 // Parameters of typical acceptance (null: exact matching).
@@ -346,13 +398,19 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
     const int64_t rows = (int64_t)B * T;
 
     if (B <= ppd::kFusedMaxB) {
-        bool in_grid = in_grid_argmax_pays(L, B, H, T, D, V, S_max);
+        bool in_grid = choose_form(L, B, H, T, D, V, S_max) == kFormSide;
         while (true) {
             // 1. partial maxima (and statistics) of every node's logits; also zeroes
             //    dev_status.  In-grid: the attention grid's side warps do this instead.
-            if (!in_grid && ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst,
-                                                        temp, dev_status, B, s) != cudaSuccess)
-                return PPD_ERR_CUDA;
+            if (!in_grid) {
+                const int narrow = narrow_argmax_grid(L, B, H, T, D, V, S_max);
+                const cudaError_t e =
+                    narrow > 0 ? ppd::launch_argmax_narrow(logits, rows, V, wl.splits, narrow, pv, pi, pst,
+                                                           temp, dev_status, B, s)
+                               : ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temp,
+                                                             dev_status, B, s);
+                if (e != cudaSuccess) return PPD_ERR_CUDA;
+            }
             // 2. attention over every layer, overlapping step 1; its side warps combine
             //    the argmax, decide acceptance and compact the accepted rows
             ppd::FusedStep f{};
@@ -377,6 +435,8 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
             if (in_grid) {
                 f.in_grid = 1;
                 f.chunk = argmax_chunk(V, wl.splits);
+            }
+            if (in_grid) {
                 f.vec = argmax_vec(logits, V);
                 f.stat_k = 1.4426950408889634f / temp;
                 f.epoch = reinterpret_cast<unsigned long long *>(ws + wl.sync);
@@ -428,14 +488,29 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
                                               prefix_len, L, B, H, T, D, S_max, eb, s));
 }
 
+int ppd_verify_step_form(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt)
+{
+    if (!attn_dims_ok(L, B, H, T, D, S_max, dt) || V < 1) return -1;
+    if (B > ppd::kFusedMaxB) return kFormGrids;
+    return choose_form(L, B, H, T, D, V, S_max);
+}
+
+int ppd_set_verify_step_form(int form)
+{
+    if (form != -1 && form != kFormTwoGrids && form != kFormSide) return -2;
+    return g_forced_form.exchange(form);
+}
+
 int ppd_verify_step_launches(int L, int B, int H, int T, int D, int V, int S_max, ppd_dtype dt,
                              int typical)
 {
     (void)typical;   // both acceptance rules launch the same number of kernels
-    if (!attn_dims_ok(L, B, H, T, D, S_max, dt) || V < 1) return -1;
+    const int form = ppd_verify_step_form(L, B, H, T, D, V, S_max, dt);
+    if (form < 0) return -1;
     const int round = dt == PPD_F32 ? 5 : 0;   // fp32 -> bf16 copies of Q, K/V tree, K/V cache
     const int attn = attention_splits(L, B, H, T, S_max) ? 2 : 1;   // + the merge grid
-    if (B <= ppd::kFusedMaxB) return (in_grid_argmax_pays(L, B, H, T, D, V, S_max) ? 0 : 1) + round + attn;
+    if (form == kFormTwoGrids) return 1 + round + attn;
+    if (form == kFormSide) return round + attn;
     // partial maxima, combine (or statistics), acceptance, attention, compaction
     return 3 + round + attn + 1;
 }

@@ -491,10 +491,37 @@ static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const W
         }
         for (int r = lane; r < T; r += 32) {
             const size_t base = ((size_t)b * T + r) * S;
-            float bv = __ldcg(f.part_val + base);
-            int bi = __ldcg(f.part_idx + base);
+            float bv = -INFINITY;
+            int bi = INT_MAX;
+            if ((S & 3) == 0) {
+                // 16-byte loads, up to 16 partials in flight (the arrays are 256-byte
+                // aligned and a row's partials start at a multiple of 4)
+                const float4 *v4 = reinterpret_cast<const float4 *>(f.part_val + base);
+                const int4 *i4 = reinterpret_cast<const int4 *>(f.part_idx + base);
+                for (int k0 = 0; k0 < S / 4; k0 += 4) {
+                    float4 v[4];
+                    int4 ix[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        if (k0 + j < S / 4) {
+                            v[j] = __ldcg(v4 + k0 + j);
+                            ix[j] = __ldcg(i4 + k0 + j);
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        if (k0 + j < S / 4) {
+                            consider(v[j].x, ix[j].x, bv, bi);
+                            consider(v[j].y, ix[j].y, bv, bi);
+                            consider(v[j].z, ix[j].z, bv, bi);
+                            consider(v[j].w, ix[j].w, bv, bi);
+                        }
+                    }
+                }
+            } else {
 #pragma unroll 8
-            for (int k = 1; k < S; ++k) consider(__ldcg(f.part_val + base + k), __ldcg(f.part_idx + base + k), bv, bi);
+                for (int k = 0; k < S; ++k) consider(__ldcg(f.part_val + base + k), __ldcg(f.part_idx + base + k), bv, bi);
+            }
             top[r] = bi;
             if (designated) f.argmax_out[(size_t)b * T + r] = bi;
             if (f.typical) stats_finish(combine_stats(f.part_stats, (int64_t)b * T + r, S), s_lse[r], s_ent[r]);
@@ -528,15 +555,29 @@ static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const W
             owns_first_tile([&](int u) {
                 const int lbh = u / p.n_qb;
                 if (u % p.n_qb != 0 || ((lbh / p.H) % B) != b) return false;
-                for (int w = lane; w < n * chunks; w += 32) {
-                    const int j = w / chunks, c = w - j * chunks;
-                    const int src = path[j];
-                    const size_t so = ((size_t)lbh * T + src) * f.row_bytes + (size_t)c * 16;
-                    const size_t dof = ((size_t)lbh * p.S_max + P + j) * f.row_bytes + (size_t)c * 16;
-                    const uint4 kx = __ldg(reinterpret_cast<const uint4 *>(f.k_tree + so));
-                    const uint4 vx = __ldg(reinterpret_cast<const uint4 *>(f.v_tree + so));
-                    *reinterpret_cast<uint4 *>(f.k_cache + dof) = kx;
-                    *reinterpret_cast<uint4 *>(f.v_cache + dof) = vx;
+                // four 16-byte pieces of K and of V per lane loaded before any is
+                // stored, so a slice's rows cost one round trip
+                for (int w0 = 0; w0 < n * chunks; w0 += 4 * 32) {
+                    uint4 kx[4], vx[4];
+                    size_t dof[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int w = w0 + u * 32 + lane;
+                        if (w < n * chunks) {
+                            const int j = w / chunks, c = w - j * chunks;
+                            const size_t so = ((size_t)lbh * T + path[j]) * f.row_bytes + (size_t)c * 16;
+                            dof[u] = ((size_t)lbh * p.S_max + P + j) * f.row_bytes + (size_t)c * 16;
+                            kx[u] = __ldg(reinterpret_cast<const uint4 *>(f.k_tree + so));
+                            vx[u] = __ldg(reinterpret_cast<const uint4 *>(f.v_tree + so));
+                        }
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        if (w0 + u * 32 + lane < n * chunks) {
+                            *reinterpret_cast<uint4 *>(f.k_cache + dof[u]) = kx[u];
+                            *reinterpret_cast<uint4 *>(f.v_cache + dof[u]) = vx[u];
+                        }
+                    }
                 }
                 return false;
             });

@@ -23,12 +23,14 @@ struct FusedStep {
     float *part_val;             // [B*T*splits] partial maxima
     int32_t *part_idx;
     int splits;
-    // in_grid != 0: no preceding grid.  Chunk c of the [B*T][splits] partial
-    // grid is computed by CTA c mod grid; a CTA publishes ready[cta] = tag once
-    // its chunks are written, where tag = *epoch + 1 read at its start.  CTA 0
-    // waits until every flag equals tag, then sets *epoch = tag and
-    // *all_ready = tag; the other CTAs read partials once *all_ready equals
-    // their tag.  Every call has a fresh tag, so no flag needs zeroing.
+    // in_grid != 0: no preceding grid; the side warps compute the partial
+    // maxima themselves while the other warps stream K/V.  Chunk c of the
+    // [B*T][splits] partial grid is computed by CTA c mod grid; a CTA
+    // publishes ready[cta] = tag once its chunks are written, where tag =
+    // *epoch + 1 read at its start.  CTA 0 waits until every flag equals tag,
+    // then sets *epoch = tag and *all_ready = tag; the other CTAs read
+    // partials once *all_ready equals their tag.  Every call has a fresh tag,
+    // so no flag needs zeroing.
     int in_grid;
     int chunk;                   // logits per chunk (multiple of 4 when vec)
     int vec;                     // 16-byte loads of the logits
@@ -152,6 +154,13 @@ cudaError_t launch_argmax_partials(const float *logits, int64_t rows, int V, int
                                    float *part_val, int32_t *part_idx, float *part_stats,
                                    float temperature, int32_t *zero_status, int n_zero,
                                    cudaStream_t stream);
+// The same partials from `grid` blocks of 512 threads (one warp per chunk at a
+// time): the fused step's argmax grid on the SMs of its attention grid's last,
+// partial round.
+cudaError_t launch_argmax_narrow(const float *logits, int64_t rows, int V, int splits, int grid,
+                                 float *part_val, int32_t *part_idx, float *part_stats,
+                                 float temperature, int32_t *zero_status, int n_zero,
+                                 cudaStream_t stream);
 cudaError_t launch_argmax_combine(const float *part_val, const int32_t *part_idx, int64_t rows,
                                   int splits, int32_t *argmax_out, cudaStream_t stream);
 

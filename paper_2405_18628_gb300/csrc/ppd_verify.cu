@@ -159,6 +159,65 @@ cudaError_t launch_argmax_partials(const float *logits, int64_t rows, int V, int
     return cudaGetLastError();
 }
 
+// The same partial maxima from a narrow grid: `gridDim.x` blocks of 512
+// threads, each warp scanning (row, split) chunks c = warp, warp + all warps,
+// ... with sixteen 16-byte loads per lane in flight.  The fused step launches
+// it on as few SMs as hold the last, partial round of its attention grid, so
+// the attention CTAs that must wait for those SMs are ones with a slice to
+// spare.  Block 0 also zeroes `zero_status`; a grid launched after this one
+// with programmatic stream serialization may start right away.
+template <bool kStats>
+__global__ void __launch_bounds__(512)
+argmax_narrow_kernel(const float *__restrict__ logits, int V, int splits, int chunk, int vec,
+                     int64_t n_chunks, float *part_val, int32_t *part_idx, float *part_stats,
+                     float stat_k, int32_t *zero_status, int n_zero)
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (zero_status && blockIdx.x == 0)
+        for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_status[i] = 0;
+    const int lane = threadIdx.x & 31;
+    const int64_t n_warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t c = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); c < n_chunks;
+         c += n_warps) {
+        const int64_t row = c / splits;
+        const int lo = (int)(c - row * splits) * chunk;
+        const int hi = min(V, lo + chunk);
+        float bv;
+        int bi;
+        SoftStats st;
+        warp_logit_span<kStats, 16>(logits + row * (int64_t)V, lo, hi, vec != 0, stat_k, lane, bv, bi, st);
+        if (lane == 0) {
+            part_val[c] = bv;
+            part_idx[c] = bi;
+            if (kStats) {
+                part_stats[3 * c] = st.m;
+                part_stats[3 * c + 1] = st.s;
+                part_stats[3 * c + 2] = st.t;
+            }
+        }
+    }
+}
+
+cudaError_t launch_argmax_narrow(const float *logits, int64_t rows, int V, int splits, int grid,
+                                 float *part_val, int32_t *part_idx, float *part_stats,
+                                 float temperature, int32_t *zero_status, int n_zero,
+                                 cudaStream_t stream)
+{
+    const int vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
+    const int chunk = (((V + splits - 1) / splits) + 3) & ~3;
+    const int64_t n_chunks = rows * splits;
+    if (part_stats)
+        argmax_narrow_kernel<true><<<grid, 512, 0, stream>>>(logits, V, splits, chunk, vec, n_chunks,
+                                                             part_val, part_idx, part_stats,
+                                                             1.4426950408889634f / temperature,
+                                                             zero_status, n_zero);
+    else
+        argmax_narrow_kernel<false><<<grid, 512, 0, stream>>>(logits, V, splits, chunk, vec, n_chunks,
+                                                              part_val, part_idx, nullptr, 0.f,
+                                                              zero_status, n_zero);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_argmax_combine(const float *part_val, const int32_t *part_idx, int64_t rows,
                                   int splits, int32_t *argmax_out, cudaStream_t stream)
 {

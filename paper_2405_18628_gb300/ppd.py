@@ -43,6 +43,8 @@ def load() -> ctypes.CDLL:
         sig = {
             "ppd_workspace_bytes": ([i32] * 7 + [i32], sz),
             "ppd_verify_step_launches": ([i32] * 7 + [i32, i32], i32),
+            "ppd_verify_step_form": ([i32] * 7 + [i32], i32),
+            "ppd_set_verify_step_form": ([i32], i32),
             "ppd_status_string": ([i32], ctypes.c_char_p),
             "ppd_tree_attention": ([vp] * 7 + [i32] * 7 + [f32, vp, vp, vp, vp, sz, vp], i32),
             "ppd_node_argmax": ([vp, i32, i32, i32, vp, vp, sz, vp], i32),
@@ -107,6 +109,19 @@ def ppd_workspace_bytes(L, B, H, T, D, V, S_max, dtype=PPD_BF16) -> int:
 def ppd_verify_step_launches(L, B, H, T, D, V, S_max, dtype=PPD_BF16, typical=False) -> int:
     """Kernels one ppd_verify_step (or ppd_verify_step_typical) call enqueues."""
     return int(load().ppd_verify_step_launches(L, B, H, T, D, V, S_max, dtype, int(typical)))
+
+
+def ppd_verify_step_form(L, B, H, T, D, V, S_max, dtype=PPD_BF16) -> int:
+    """Form of the fused step for these sizes: 0 separate grids, 1 argmax grid
+    then attention grid, 2 one grid with the argmax in the side warps, 3 one
+    grid with the argmax in the CTAs of the last, partial round."""
+    return int(load().ppd_verify_step_form(L, B, H, T, D, V, S_max, dtype))
+
+
+def ppd_set_verify_step_form(form: int) -> int:
+    """Force the fused step's form (1, 2 or 3; -1 = automatic); returns the
+    previous setting."""
+    return int(load().ppd_set_verify_step_form(int(form)))
 
 
 def workspace(L, B, H, T, D, V, S_max, dtype=PPD_BF16, device="cuda") -> torch.Tensor:

@@ -67,6 +67,33 @@ def test_verify_step_launch_counts(lib):
     assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 0, 176) == -1
 
 
+def test_verify_step_forms(lib):
+    """The fused step's form: separate grids above 64 sequences, an argmax grid
+    first when the logits weigh more than 1/64 of the K/V bytes (the tiny
+    shapes), the argmax in the attention grid's side warps otherwise (the
+    Vicuna-7B shapes), -1 for rejected sizes.  A forced form applies to every
+    fused size until it is reset, and other values are refused."""
+    from paper_2405_18628_gb300 import ppd
+    assert ppd.ppd_verify_step_form(1, 65, 2, 16, 64, 300, 56) == 0
+    assert ppd.ppd_verify_step_form(1, 1, 4, 48, 64, 1024, 176) == 1
+    assert ppd.ppd_verify_step_form(32, 1, 32, 64, 128, 32000, 2112) == 2
+    assert ppd.ppd_verify_step_form(1, 1, 4, 48, 96, 1024, 176) == -1
+    prev = ppd.ppd_set_verify_step_form(2)
+    try:
+        assert prev == -1
+        assert ppd.ppd_verify_step_form(1, 1, 4, 48, 64, 1024, 176) == 2
+        assert ppd.ppd_verify_step_form(1, 65, 2, 16, 64, 300, 56) == 0
+        assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 1024, 176) == 1
+        assert ppd.ppd_set_verify_step_form(1) == 2
+        assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112) == 2
+        for bad in (0, 3, 4):
+            assert ppd.ppd_set_verify_step_form(bad) == -2
+        assert ppd.ppd_verify_step_form(1, 1, 4, 48, 64, 1024, 176) == 1
+    finally:
+        ppd.ppd_set_verify_step_form(-1)
+    assert ppd.ppd_verify_step_form(32, 1, 32, 64, 128, 32000, 2112) == 2
+
+
 def test_host_argument_checks(lib):
     """Invalid sizes and null pointers are rejected with PPD_ERR_INVALID_ARG
     (or UNSUPPORTED) without launching anything."""

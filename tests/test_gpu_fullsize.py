@@ -95,10 +95,11 @@ def test_full_size_step(cuda_device, name):
     assert err <= ATOL and rel <= RTOL_L2, (layers, err, rel)
 
 
-def _plant_ties(logits, chunk):
-    """Rows of one sequence's logits rewritten with ties, NaNs, infinities and
-    signed zeros, many of them straddling the boundaries of the argmax's
-    per-row chunks (columns k*chunk - 1 | k*chunk)."""
+def _plant_ties(logits, chunk, r0=0):
+    """Rows r0.. of one sequence's logits rewritten with ties, NaNs,
+    infinities and signed zeros, many of them straddling the boundaries of the
+    argmax's per-row column spans (columns k*chunk - 1 | k*chunk)."""
+    logits = logits[r0:]
     T, V = logits.shape
     n_b = max(1, (V - 1) // chunk)
     for r in range(min(T, 7)):                           # max tied across a boundary
@@ -125,15 +126,18 @@ def _plant_ties(logits, chunk):
 
 @pytest.mark.parametrize("name", ["mobilellama", "vicuna7b"])
 def test_full_size_step_argmax_ties(cuda_device, name):
-    """The fused step at full size (its in-grid side-warp argmax at Vicuna-7B
-    shapes, the argmax grid at MobileLlama shapes) with ties, NaNs, +-inf and
-    signed zeros planted across the per-row argmax chunks: every index output
-    and the compacted cache rows bit for bit against the oracle."""
+    """The fused step at full size, in the form the benchmark times, with ties,
+    NaNs, +-inf and signed zeros planted across the column chunks of both
+    in-grid argmax forms (the side warps' chunks of 4000 logits, rows 0..24;
+    the softmax warps' chunks of 1000, rows 25..49): every index output and
+    the compacted cache rows bit for bit against the oracle."""
     w = W.WORKLOADS[name]
+    assert ppd.ppd_verify_step_form(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max) in (1, 2, 3)
     s = W.make_step_inputs(w)
     lg = s.logits.copy()
     for b in range(w.B):
         _plant_ties(lg[b], 4000)
+        _plant_ties(lg[b], 1000, r0=25)
     am = oracle.node_argmax(lg)
     # candidates that copied their parent's planted top token now copy the new argmax
     cand = s.cand_tokens.copy()
