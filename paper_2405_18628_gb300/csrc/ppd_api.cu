@@ -254,7 +254,8 @@ ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, cons
                              const void *vt, const int32_t *prefix_len, const int32_t *parent,
                              int L, int B, int H, int T, int D, int S_max, float scale, float *out,
                              float *lse, int32_t *dev_status, uint8_t *ws, const WsLayout *wl,
-                             const ppd::FusedStep *fused, bool programmatic, cudaStream_t stream)
+                             const ppd::FusedStep *fused, bool programmatic, bool chained,
+                             cudaStream_t stream)
 {
     const int T_pad = (T + 31) & ~31;
     const uint64_t lbh = (uint64_t)L * B * H;
@@ -292,7 +293,9 @@ ppd_status enqueue_attention(const void *q, const void *kc, const void *vc, cons
     }
     p.fused = fused != nullptr;
     if (fused) p.fs = *fused;
-    return cuda_status(ppd::launch_tree_attention(m, p, D, split_grid(), programmatic, stream));
+    p.pdl_wait = chained ? 1 : 0;
+    return cuda_status(ppd::launch_tree_attention(m, p, D, split_grid(), programmatic || chained,
+                                                  stream));
 }
 
 // fp32 operands: round to bf16 copies in the workspace first.
@@ -301,14 +304,16 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
                                  int L, int B, int H, int T, int D, int S_max, ppd_dtype dt,
                                  float scale, float *out, float *lse, int32_t *dev_status,
                                  uint8_t *ws, const WsLayout &wl, const ppd::FusedStep *fused,
-                                 cudaStream_t stream)
+                                 cudaStream_t stream, bool chained = false)
 {
     // With bf16 operands the attention grid only reads caller inputs before its end
     // phase, so it may overlap the preceding (argmax) grid -- when there is one.
+    // `chained`: the grid follows a status reset launched as a programmatic
+    // dependent, and waits for it (and so for whatever preceded it) itself.
     if (dt == PPD_BF16)
         return enqueue_attention(q, kc, vc, kt, vt, prefix_len, parent, L, B, H, T, D, S_max, scale,
                                  out, lse, dev_status, ws, ws ? &wl : nullptr, fused,
-                                 fused != nullptr && !fused->in_grid, stream);
+                                 fused != nullptr && !fused->in_grid, chained, stream);
     const int64_t lbh = (int64_t)L * B * H;
     const int64_t n_t = lbh * T * D, n_c = lbh * (int64_t)S_max * D;
     uint16_t *bq = reinterpret_cast<uint16_t *>(ws + wl.conv);
@@ -323,7 +328,7 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
         ppd::launch_round_bf16((const float *)vc, bvc, n_c, stream) != cudaSuccess)
         return PPD_ERR_CUDA;
     return enqueue_attention(bq, bkc, bvc, bkt, bvt, prefix_len, parent, L, B, H, T, D, S_max,
-                             scale, out, lse, dev_status, ws, &wl, fused, false, stream);
+                             scale, out, lse, dev_status, ws, &wl, fused, false, false, stream);
 }
 
 // Blocks of the fused step's narrow argmax grid (0: use the wide grid).  When
@@ -562,11 +567,17 @@ ppd_status ppd_tree_attention(const void *q, const void *k_cache, const void *v_
     const bool ws_ok = workspace && ws_bytes >= wl.total && aligned(workspace, kAlign);
     if (dt == PPD_F32 && !ws_ok) return PPD_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (cudaMemsetAsync(dev_status, 0, (size_t)B * 4, s) != cudaSuccess) return PPD_ERR_CUDA;
+    // dev_status is reset by a one-block grid launched as a programmatic
+    // dependent (it waits for the preceding grid before writing); the attention
+    // grid is its programmatic dependent in turn, so a sequence of calls (one
+    // per layer, as a model runs them) launches each grid while the previous
+    // one still runs and only the setup that reads no input runs early
+    if (ppd::launch_zero_status(dev_status, B, s) != cudaSuccess) return PPD_ERR_CUDA;
     // a bf16 call without a full workspace runs unsplit
     return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B, H,
                                  T, D, S_max, dt, scale, out, lse, dev_status,
-                                 ws_ok ? static_cast<uint8_t *>(workspace) : nullptr, wl, nullptr, s);
+                                 ws_ok ? static_cast<uint8_t *>(workspace) : nullptr, wl, nullptr, s,
+                                 true);
 }
 
 ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *argmax_out,

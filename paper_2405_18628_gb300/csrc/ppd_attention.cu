@@ -160,6 +160,21 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
         tmem_alloc(tmem_ptr, Lay::TMEM_COLS);
         tmem_relinquish();
     }
+    if (warp == 8 && lane == 0) {
+        // the tensor maps are kernel parameters: fetch them before any wait
+        tma_prefetch_map(&map_q);
+        tma_prefetch_map(&map_kc);
+        tma_prefetch_map(&map_vc);
+        tma_prefetch_map(&map_kt);
+        tma_prefetch_map(&map_vt);
+    }
+    // in a chain of programmatic launches the inputs may come from the preceding
+    // grid: everything above overlapped it, nothing below reads before it is done
+    // (the first K/V tiles are only asked of L2 before)
+    if (p.pdl_wait) {
+        if (warp == 8) prefetch_first_tiles<SPLIT>(p, lane, &map_kc, &map_vc, Lay::DCH, 3);
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+    }
     WorkRange *wr_s = reinterpret_cast<WorkRange *>(smem + Lay::OFF_RANGE);
     if (warp == 8) {
         const WorkRange w = plan_range(p, lane);   // whole units round-robin without p.split
@@ -168,9 +183,9 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
             if (SPLIT) p.split_rec[blockIdx.x].u = -1;   // no cut unit recorded yet
         }
     }
-    // the merge of cut units (a dependent launch) may be scheduled now; it waits
-    // for this grid to complete
-    if (SPLIT) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // the merge of cut units, or the next call of a chain (a dependent launch),
+    // may be scheduled now; it waits for this grid to complete
+    if (SPLIT || p.pdl_wait) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -183,11 +198,6 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
     } else if (warp == 8) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            tma_prefetch_map(&map_q);
-            tma_prefetch_map(&map_kc);
-            tma_prefetch_map(&map_vc);
-            tma_prefetch_map(&map_kt);
-            tma_prefetch_map(&map_vt);
             const uint64_t pol = l2_policy_evict_first();
             const uint32_t q_tx = (uint32_t)T_pad * 128u * Lay::DCH;
             int g = 0, k = 0;
@@ -773,6 +783,9 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
 // once the attention grid has completed.
 __global__ void __launch_bounds__(256) split_merge_kernel(const AttnParams p, int D)
 {
+    // a next grid launched as a programmatic dependent may start at once; it
+    // waits for this grid to complete before it reads or writes anything
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const SplitRecord r = p.split_rec[blockIdx.x];
     if (r.u < 0) return;

@@ -64,7 +64,10 @@ PPD_DEV int split_cta_of(long long x, long long N, int G) { return (int)(((x + 1
 
 // This CTA's work, computed by one whole warp (every lane gets the result).
 // The tiles of one layer's block of sequence b number H * n_qb * (n_pref(b) +
-// n_tt); lanes hold sequences b = lane and lane + 32.
+// n_tt); lanes hold sequences b = lane and lane + 32.  kHint: the prefix
+// lengths are read through L2 because they may still be changing (a plan
+// made before the wait of a chained launch, used for prefetch hints only).
+template <bool kHint = false>
 PPD_DEV WorkRange plan_range(const AttnParams &p, int lane)
 {
     WorkRange w{};
@@ -78,7 +81,8 @@ PPD_DEV WorkRange plan_range(const AttnParams &p, int lane)
     const unsigned full = 0xffffffffu;
     const int per_b = p.H * p.n_qb;
     auto nt_of = [&](int b) {
-        const int P = min(max(__ldg(p.prefix_len + b), 0), p.S_max);
+        const int P = min(max(kHint ? ld_relaxed_gpu_s32(p.prefix_len + b) : __ldg(p.prefix_len + b), 0),
+                          p.S_max);
         return ((P + 127) >> 7) + p.n_tt;
     };
     const int w0 = lane < p.B ? per_b * nt_of(lane) : 0;
@@ -139,6 +143,40 @@ PPD_DEV WorkRange plan_range(const AttnParams &p, int lane)
         locate(base + ge - 1, w.u_last, jl);
     }
     return w;
+}
+
+// Before the wait of a chained launch (one warp, all lanes): ask L2 for the
+// first `n` K and V prefix tiles this CTA will stream, from a plan made with
+// prefix lengths that may still be changing.  Only a hint -- nothing is
+// written to shared memory and nothing waits on it; the real loads follow the
+// wait with the plan remade -- so the preceding grid's work overlaps the
+// first tiles' trip from HBM.  Tree tiles are skipped (in a model the
+// preceding grids write them).
+template <bool SPLIT>
+PPD_DEV void prefetch_first_tiles(const AttnParams &p, int lane, const CUtensorMap *kc,
+                                  const CUtensorMap *vc, int dch, int n)
+{
+    const WorkRange w = plan_range<true>(p, lane);
+    if (lane != 0) return;
+    int u = SPLIT ? w.u_first : (int)blockIdx.x;
+    int j = SPLIT ? w.j_first : 0;
+    int left = SPLIT ? w.n_tiles : n;
+    for (int k = 0; k < n && left > 0 && u < p.n_units; ++k, --left) {
+        const int lbh = u / p.n_qb;
+        const int b = (lbh / p.H) % p.B;
+        const int P = min(max(ld_relaxed_gpu_s32(p.prefix_len + b), 0), p.S_max);
+        const int n_pref = (P + 127) >> 7;
+        if (j < n_pref) {
+            for (int c = 0; c < dch; ++c) {
+                tma_prefetch_l2_3d(kc, c * 64, j * 128, lbh);
+                tma_prefetch_l2_3d(vc, c * 64, j * 128, lbh);
+            }
+            ++j;
+        } else {   // the unit's tree tiles: on to the next unit
+            u = SPLIT ? u + 1 : u + (int)gridDim.x;
+            j = 0;
+        }
+    }
 }
 
 // One stretch of a unit's tiles [j0, j1) processed by this CTA.

@@ -119,6 +119,21 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
         tmem_alloc(tmem_ptr, Lay::TMEM_COLS);
         tmem_relinquish();
     }
+    if (warp == 8 && lane == 0) {
+        // the tensor maps are kernel parameters: fetch them before any wait
+        tma_prefetch_map(&map_q);
+        tma_prefetch_map(&map_kc);
+        tma_prefetch_map(&map_vc);
+        tma_prefetch_map(&map_kt);
+        tma_prefetch_map(&map_vt);
+    }
+    // in a chain of programmatic launches the inputs may come from the preceding
+    // grid: everything above overlapped it, nothing below reads before it is done
+    // (the first K/V tiles are only asked of L2 before)
+    if (p.pdl_wait) {
+        if (warp == 8) prefetch_first_tiles<SPLIT>(p, lane, &map_kc, &map_vc, Lay::DCH, 3);
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+    }
     WorkRange *wr_s = reinterpret_cast<WorkRange *>(smem + Lay::OFF_RANGE);
     if (warp == 8) {
         const WorkRange w = plan_range(p, lane);   // whole units round-robin without p.split
@@ -127,9 +142,9 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
             if (SPLIT) p.split_rec[blockIdx.x].u = -1;   // no cut unit recorded yet
         }
     }
-    // the merge of cut units (a dependent launch) may be scheduled now; it waits
-    // for this grid to complete
-    if (SPLIT) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // the merge of cut units, or the next call of a chain (a dependent launch),
+    // may be scheduled now; it waits for this grid to complete
+    if (SPLIT || p.pdl_wait) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -147,11 +162,6 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
         // roughly in issue order, so a V tile queued ahead of its turn would
         // hold back the K tile the next score product waits for, and vice versa.
         if (lane == 0) {
-            tma_prefetch_map(&map_q);
-            tma_prefetch_map(&map_kc);
-            tma_prefetch_map(&map_kt);
-            tma_prefetch_map(&map_vc);
-            tma_prefetch_map(&map_vt);
             const uint64_t pol = l2_policy_evict_first();
             constexpr int LAG = 2;
             int v_row[LAG + 1], v_lbh[LAG + 1];

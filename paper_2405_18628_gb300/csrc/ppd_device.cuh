@@ -136,6 +136,14 @@ PPD_DEV unsigned long long ld_acquire_gpu(const unsigned long long *p)
     return v;
 }
 
+// A 32-bit load served by L2 (never a stale L1 or texture-cache line).
+PPD_DEV int ld_relaxed_gpu_s32(const int *p)
+{
+    int v;
+    asm volatile("ld.relaxed.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
 PPD_DEV void st_release_gpu(unsigned long long *p, unsigned long long v)
 {
     asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
@@ -193,6 +201,15 @@ PPD_DEV void tma_load_3d(void *dst, const CUtensorMap *map, uint64_t *bar, int x
         ".L2::cache_hint [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(smem_addr(dst)),
         "l"(map), "r"(smem_addr(bar)), "r"(x), "r"(y), "r"(z), "l"(policy)
         : "memory");
+}
+
+// Fetch a 3-D tile of a tensor map into L2 only (a hint: no shared memory, no
+// completion to wait for).  x must be 16-byte aligned as for tma_load_3d.
+PPD_DEV void tma_prefetch_l2_3d(const CUtensorMap *map, int x, int y, int z)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(map),
+                 "r"(x), "r"(y), "r"(z)
+                 : "memory");
 }
 
 PPD_DEV void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar, int x, int y)

@@ -87,6 +87,10 @@ struct AttnParams {
     struct SplitRecord *split_rec;   // [grid]
     int fused;                  // run the end phase below
     FusedStep fs;
+    // Launched as a programmatic dependent of the preceding grid (a chain of
+    // ppd_tree_attention calls): the setup that reads no input overlaps that
+    // grid, then every thread waits for it before reading any input.
+    int pdl_wait;
 };
 
 // Work split limits: batch size (the per-CTA range search holds the batch in
@@ -209,6 +213,10 @@ cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const i
                              cudaStream_t stream);
 
 cudaError_t launch_round_bf16(const float *src, uint16_t *dst, int64_t n, cudaStream_t stream);
+
+// Zero `n` status words once the preceding grid has completed, as a
+// programmatic dependent launch that lets the next grid launch at once.
+cudaError_t launch_zero_status(int32_t *status, int n, cudaStream_t stream);
 
 cudaError_t launch_selftest_umma(const CUtensorMap &ma, const CUtensorMap &mb, const void *a_raw,
                                  const void *b_raw, float *d, int mode, int N, cudaStream_t stream);

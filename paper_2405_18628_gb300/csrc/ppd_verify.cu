@@ -355,6 +355,29 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_tree,
     return cudaGetLastError();
 }
 
+// ------------------------------------------------------------------ status reset
+
+__global__ void zero_status_kernel(int32_t *status, int n)
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    for (int i = threadIdx.x; i < n; i += blockDim.x) status[i] = 0;
+}
+
+cudaError_t launch_zero_status(int32_t *status, int n, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(128);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, zero_status_kernel, status, n);
+}
+
 // ------------------------------------------------------------------ fp32 -> bf16
 
 __global__ void round_bf16_kernel(const float *__restrict__ src, uint16_t *__restrict__ dst,
