@@ -74,3 +74,15 @@ def test_packed_buffer_layout():
     assert buf.numel() == 512 + 256 + 256
     v["parent"].copy_(torch.arange(4, dtype=torch.int32))
     assert buf[768:784].view(torch.int32).tolist() == [0, 1, 2, 3]
+
+
+def test_e2e_layer_groups():
+    """The pipelined end-to-end leg's layer groups cover every layer once, the
+    last group no larger than the first."""
+    sys.path.insert(0, ROOT)
+    import bench
+    for L in (1, 2, 4, 24, 32, 40, 80):
+        g = bench.e2e_groups(L)
+        assert sum(g) == L and all(n >= 1 for n in g)
+        assert g[-1] <= g[0]
+    assert bench.e2e_groups(32) == [14, 10, 6, 2]
