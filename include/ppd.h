@@ -333,6 +333,19 @@ int ppd_verify_step_form(int L, int B, int H, int T, int D, int V, int S_max, pp
  */
 int ppd_set_verify_step_form(int form);
 
+/*
+ * Diagnostics of the device-side timeout (no paper counterpart; for tests).
+ * In the one-grid form (2) of every later fused step of this process, the
+ * grid-wide wait for the argmax partials gives up after `limit_ns`
+ * nanoseconds instead of 4 s (0 restores 4 s), and CTA `withhold_cta` never
+ * publishes that its partials are ready (-1: every CTA does), so that a test
+ * can make the wait run out: the step then reports PPD_ERR_TIMEOUT in
+ * dev_status for every sequence, writes no cache row, and (as after any
+ * timeout) its workspace must be zeroed before the next call.  Returns
+ * PPD_ERR_INVALID_ARG for withhold_cta < -1.
+ */
+ppd_status ppd_debug_grid_wait(unsigned long long limit_ns, int withhold_cta);
+
 /* Human-readable name of a status code (static string). */
 const char *ppd_status_string(ppd_status s);
 

@@ -97,6 +97,12 @@ enum FusedForm { kFormGrids = 0, kFormTwoGrids = 1, kFormSide = 2 };
 // A form forced by ppd_set_verify_step_form (-1: chosen by the rules below).
 std::atomic<int> g_forced_form{-1};
 
+// The in-grid argmax's grid-wide wait: its limit in ns (0: the default of the
+// device-side waits) and a CTA that withholds its flag (-1: none); set only by
+// ppd_debug_grid_wait, for tests of the timeout path.
+std::atomic<unsigned long long> g_grid_wait_ns{0};
+std::atomic<int> g_withhold_cta{-1};
+
 int narrow_argmax_grid(int L, int B, int H, int T, int D, int V, int S_max);
 
 // The form of a fused step (B <= kFusedMaxB) of these sizes: an argmax grid
@@ -442,6 +448,12 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
                 f.chunk = argmax_chunk(V, wl.splits);
             }
             if (in_grid) {
+                // no argmax grid to zero the status first: a one-block reset does,
+                // so that every status write can be an atomic maximum
+                if (ppd::launch_zero_status(dev_status, B, s) != cudaSuccess) return PPD_ERR_CUDA;
+                const unsigned long long lim = g_grid_wait_ns.load(std::memory_order_relaxed);
+                f.wait_limit_ns = lim ? lim : ppd::kWaitLimitNs;
+                f.withhold_cta = g_withhold_cta.load(std::memory_order_relaxed);
                 f.vec = argmax_vec(logits, V);
                 f.stat_k = 1.4426950408889634f / temp;
                 f.epoch = reinterpret_cast<unsigned long long *>(ws + wl.sync);
@@ -500,6 +512,14 @@ int ppd_verify_step_form(int L, int B, int H, int T, int D, int V, int S_max, pp
     return choose_form(L, B, H, T, D, V, S_max);
 }
 
+ppd_status ppd_debug_grid_wait(unsigned long long limit_ns, int withhold_cta)
+{
+    if (withhold_cta < -1) return PPD_ERR_INVALID_ARG;
+    g_grid_wait_ns.store(limit_ns);
+    g_withhold_cta.store(withhold_cta);
+    return PPD_OK;
+}
+
 int ppd_set_verify_step_form(int form)
 {
     if (form != -1 && form != kFormTwoGrids && form != kFormSide) return -2;
@@ -515,7 +535,7 @@ int ppd_verify_step_launches(int L, int B, int H, int T, int D, int V, int S_max
     const int round = dt == PPD_F32 ? 5 : 0;   // fp32 -> bf16 copies of Q, K/V tree, K/V cache
     const int attn = attention_splits(L, B, H, T, S_max) ? 2 : 1;   // + the merge grid
     if (form == kFormTwoGrids) return 1 + round + attn;
-    if (form == kFormSide) return round + attn;
+    if (form == kFormSide) return 1 + round + attn;   // the status reset, then one grid
     // partial maxima, combine (or statistics), acceptance, attention, compaction
     return 3 + round + attn + 1;
 }

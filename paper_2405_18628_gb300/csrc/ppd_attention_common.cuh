@@ -431,11 +431,11 @@ PPD_DEV void side_argmax_chunks(const AttnParams &p, unsigned long long tag, int
     }
     __threadfence();
     __syncwarp();
-    if (lane == 0) st_release_gpu(f.ready + blockIdx.x, tag);
+    if (lane == 0 && (int)blockIdx.x != f.withhold_cta) st_release_gpu(f.ready + blockIdx.x, tag);
 }
 
 // Wait until every CTA of the grid has published `tag` (bounded: raises the
-// CTA's abort flag and returns false after kWaitLimitNs, or at once when the
+// CTA's abort flag and returns false after f.wait_limit_ns, or at once when the
 // flag is already up; lane 0 takes that decision for the whole warp, so no
 // lane leaves while others still shuffle).  Only CTA 0 reads the per-CTA flags; once all are up
 // it advances the epoch for the next call and publishes `tag` in all_ready,
@@ -458,7 +458,7 @@ PPD_DEV bool side_wait_all(const AttnParams &p, unsigned long long tag, int lane
         }
         if (done) break;
         const bool give_up = __shfl_sync(
-            0xffffffffu, lane == 0 && (*abort_flag || global_timer() - t0 > kWaitLimitNs), 0);
+            0xffffffffu, lane == 0 && (*abort_flag || global_timer() - t0 > f.wait_limit_ns), 0);
         if (give_up) {
             if (lane == 0) *abort_flag = 1;
             return false;
@@ -581,8 +581,7 @@ static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const W
                 f.accept_len[b] = res.n_acc;
                 f.next_token[b] = res.next_token;
                 f.new_prefix_len[b] = res.new_prefix_len;
-                if (f.in_grid) f.status[b] = res.status;
-                else atomicMax(f.status + b, res.status);
+                atomicMax(f.status + b, res.status);
             }
         }
         if (has_unit && res.n_acc > 0) {

@@ -4,6 +4,8 @@
 // descriptors of the 5th-generation tensor cores, written as inline PTX.
 #pragma once
 
+#include "ppd_kernels.h"
+
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cstdint>
@@ -16,8 +18,6 @@ namespace ppd {
 enum : int { kOk = 0, kErrInvalidArg = 1, kErrUnsupported = 2, kErrTree = 3,
              kErrCapacity = 4, kErrCuda = 5, kErrTimeout = 6 };
 
-// A bounded wait gives up after this many nanoseconds of %globaltimer.
-constexpr uint64_t kWaitLimitNs = 4000000000ull;
 
 PPD_DEV uint32_t smem_addr(const void *p)
 {

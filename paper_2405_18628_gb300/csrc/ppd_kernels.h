@@ -8,6 +8,9 @@
 
 namespace ppd {
 
+// A bounded device-side wait gives up after this many nanoseconds of %globaltimer.
+constexpr uint64_t kWaitLimitNs = 4000000000ull;
+
 // Tensor maps of the attention operands (bf16, 128-byte swizzle, boxes of
 // 64 columns): Q [LBH][T][D] (box rows T_pad), cache K/V [LBH][S_max][D] and
 // tree K/V [LBH][T][D] (box rows 128).
@@ -32,6 +35,8 @@ struct FusedStep {
     // partials once *all_ready equals their tag.  Every call has a fresh tag,
     // so no flag needs zeroing.
     int in_grid;
+    unsigned long long wait_limit_ns;   // the grid-wide wait gives up after this long
+    int withhold_cta;            // diagnostics: this CTA never publishes its flag (-1: none)
     int chunk;                   // logits per chunk (multiple of 4 when vec)
     int vec;                     // 16-byte loads of the logits
     float stat_k;                // log2(e) / temperature (typical acceptance)
@@ -44,8 +49,8 @@ struct FusedStep {
     int32_t *path;               // [B,T]
     int32_t *next_token;         // [B]
     int32_t *new_prefix_len;     // [B]
-    int32_t *status;             // [B]: zeroed by the argmax grid and raised with atomicMax;
-                                 // with in_grid written by the sequence's designated CTA
+    int32_t *status;             // [B]: zeroed by the grid before (the argmax grid, or with
+                                 // in_grid a one-block reset), then raised with atomicMax
     uint8_t *k_cache, *v_cache;  // raw cache storage
     const uint8_t *k_tree, *v_tree;
     int row_bytes;               // D * element size

@@ -45,6 +45,7 @@ def load() -> ctypes.CDLL:
             "ppd_verify_step_launches": ([i32] * 7 + [i32, i32], i32),
             "ppd_verify_step_form": ([i32] * 7 + [i32], i32),
             "ppd_set_verify_step_form": ([i32], i32),
+            "ppd_debug_grid_wait": ([ctypes.c_ulonglong, i32], i32),
             "ppd_status_string": ([i32], ctypes.c_char_p),
             "ppd_tree_attention": ([vp] * 7 + [i32] * 7 + [f32, vp, vp, vp, vp, sz, vp], i32),
             "ppd_node_argmax": ([vp, i32, i32, i32, vp, vp, sz, vp], i32),
@@ -122,6 +123,13 @@ def ppd_set_verify_step_form(form: int) -> int:
     """Force the fused step's form (1, 2 or 3; -1 = automatic); returns the
     previous setting."""
     return int(load().ppd_set_verify_step_form(int(form)))
+
+
+def ppd_debug_grid_wait(limit_ns: int, withhold_cta: int = -1) -> None:
+    """Tests of the timeout path: the one-grid step's grid-wide wait gives up
+    after limit_ns (0: the default 4 s) and CTA withhold_cta never publishes
+    its flag (-1: none)."""
+    _check(load().ppd_debug_grid_wait(int(limit_ns), int(withhold_cta)), "ppd_debug_grid_wait")
 
 
 def workspace(L, B, H, T, D, V, S_max, dtype=PPD_BF16, device="cuda") -> torch.Tensor:

@@ -52,14 +52,15 @@ def test_workspace_bytes(lib):
 
 
 def test_verify_step_launch_counts(lib):
-    """Kernels per verification step: one grid when the argmax runs inside the
-    attention grid (Vicuna-7B shapes: 8 MB of logits against 1.1 GB of K/V), an
+    """Kernels per verification step: a one-block status reset and one grid
+    when the argmax runs inside the attention grid (Vicuna-7B shapes on a
+    device of unknown SM count: 8 MB of logits against 1.1 GB of K/V), an
     argmax grid first when the logits weigh more (48 x 1024 logits against a
     128-token prefix), five grids above 64 sequences, five fp32 rounding grids
     in front for fp32 operands, and -1 for sizes the step rejects."""
     from paper_2405_18628_gb300 import ppd
-    assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112) == 1
-    assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112, typical=True) == 1
+    assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112) == 2
+    assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112, typical=True) == 2
     assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 1024, 176) == 2
     assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 1024, 176, ppd.PPD_F32) == 7
     assert ppd.ppd_verify_step_launches(1, 65, 2, 16, 64, 300, 56) == 5
@@ -83,7 +84,7 @@ def test_verify_step_forms(lib):
         assert prev == -1
         assert ppd.ppd_verify_step_form(1, 1, 4, 48, 64, 1024, 176) == 2
         assert ppd.ppd_verify_step_form(1, 65, 2, 16, 64, 300, 56) == 0
-        assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 1024, 176) == 1
+        assert ppd.ppd_verify_step_launches(1, 1, 4, 48, 64, 1024, 176) == 2
         assert ppd.ppd_set_verify_step_form(1) == 2
         assert ppd.ppd_verify_step_launches(32, 1, 32, 64, 128, 32000, 2112) == 2
         for bad in (0, 3, 4):
@@ -102,6 +103,9 @@ def test_host_argument_checks(lib):
     null = None
     s = vp(0)
     INVALID = 1
+    # the timeout diagnostics reject a negative CTA other than -1, and restore cleanly
+    assert lib.ppd_debug_grid_wait(ctypes.c_ulonglong(0), -2) == INVALID
+    assert lib.ppd_debug_grid_wait(ctypes.c_ulonglong(0), -1) == 0
     # T > 512
     assert lib.ppd_tree_attention(fake, fake, fake, fake, fake, fake, fake, 1, 1, 1, 513, 64, 200,
                                   0, 0.0, fake, null, fake, null, 0, s) == INVALID
