@@ -64,16 +64,17 @@ REFERENCE_BUDGET_S = 180.0
 # DRAM traffic of one launch of the roofline kernel (dram__bytes_read.sum +
 # dram__bytes_write.sum), keyed by workload, with the hash of the attention
 # sources it was taken on: a stale entry reports null.  The captures ran the
-# same shapes with 19 layers (608 / 760 units: whole rounds of 152 CTAs) and
-# are scaled to the full layer count, since traffic grows with the units
-# (the logits, read once per step, are not scaled).  Writes still held in L2
-# when the kernel ends are not in the count, so this is the reads plus the
-# part of the writes that reached DRAM during the launch.
+# attention alone (ppd_tree_attention, the roofline kernel whenever the step
+# is more than one launch) at the same shapes with 19 layers (608 / 760 units:
+# whole rounds of 152 CTAs) and are scaled to the full layer count, since the
+# traffic grows with the units.  Writes still held in L2 when the kernel ends
+# are not in the count, so this is the reads plus the part of the writes that
+# reached DRAM during the launch.
 MEASURED_TRAFFIC = {
-    # whole fused step: 685,382,912 B at 19 layers; slices x 32/19, logits once
-    "vicuna7b": {"bytes_per_launch": 1_148_724_062, "src": "34ce1a8dc4edf4e2"},
-    # whole fused step: 1,672,942,592 B at 19 layers; slices x 40/19, logits once
-    "vicuna13b": {"bytes_per_launch": 3_508_402_931, "src": "34ce1a8dc4edf4e2"},
+    # 675,924,224 B at 19 layers (reads 667,973,120), x 32/19
+    "vicuna7b": {"bytes_per_launch": 1_138_398_693, "src": "6cc40380e523c3a7"},
+    # 1,658,914,816 B at 19 layers (reads 1,650,980,352), x 40/19
+    "vicuna13b": {"bytes_per_launch": 3_492_452_244, "src": "6cc40380e523c3a7"},
 }
 
 
