@@ -216,6 +216,102 @@ PPD_DEV AcceptResult accept_warp_pass(TopLoad top, Pass pass, const int32_t *par
     return r;
 }
 
+// ------------------------------------------------------------------ trees of up to 64 nodes
+//
+// The same acceptance with the tree in registers: node i's values live in lane
+// i % 32, slot i / 32, of a two-slot array, and a node's value is fetched with
+// two warp shuffles (every lane takes part; n < 64).  No scratch memory: in
+// the fused step's side warp, where a round trip to L2 costs about a
+// microsecond while the other warps stream K/V, the walk up the tree then
+// costs shuffles instead of dependent loads.
+template <class V2>
+PPD_DEV auto node_value(const V2 (&v)[2], int n) -> V2
+{
+    const V2 a = __shfl_sync(0xffffffffu, v[0], n & 31);
+    const V2 b = __shfl_sync(0xffffffffu, v[1], n & 31);
+    return n < 32 ? a : b;
+}
+
+// Acceptance of one sequence of T <= 64 nodes by one warp (all lanes call it;
+// the rule and the result are those of accept_warp_pass).
+//   top    node i's top-1 token in lane i % 32, slot i / 32
+//   pass   pass(i, parent, token), called by every lane at once (it may fetch
+//          node values); lanes with no node pass parent 0 and token 0
+//   path   out: accepted node j (depth order) in lane j % 32, slot j / 32; -1
+//          from n_acc on
+template <class Pass>
+PPD_DEV AcceptResult accept_warp_small(const int (&top)[2], Pass pass, const int32_t *par,
+                                       const int32_t *tok, int P, int T, int V, int S_max, int lane,
+                                       int (&path)[2])
+{
+    int pa[2], tk[2];
+    bool bad = false;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int i = lane + 32 * k;
+        pa[k] = -1;
+        tk[k] = -1;
+        if (i < T) {
+            pa[k] = __ldg(par + i);
+            tk[k] = __ldg(tok + i);
+            if (i == 0)
+                bad |= (pa[k] != -1) || tk[k] < 0 || tk[k] >= V;
+            else
+                bad |= pa[k] < 0 || pa[k] >= i || tk[k] < -1 || tk[k] >= V;
+        }
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    int err = bad ? kErrTree : ((P < 0 || P > S_max) ? kErrCapacity : kOk);
+
+    uint32_t okw[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int i = lane + 32 * k;
+        const bool cand = i > 0 && i < T && err == kOk && tk[k] >= 0;
+        const bool ps = pass(i, cand ? pa[k] : 0, cand ? tk[k] : 0);
+        okw[k] = __ballot_sync(0xffffffffu, (i == 0 && err == kOk) || (cand && ps));
+    }
+
+    int best_key = -1;   // (depth << 10) | (1023 - node): deepest, then smallest index
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int i = lane + 32 * k;
+        const bool mine = i < T && err == kOk;
+        int n = mine ? i : 0, depth = 0;
+        bool good = true;
+        // a valid tree's parents precede their children: every walk ends at 0
+        while (__any_sync(0xffffffffu, n > 0)) {
+            const int up = node_value(pa, n);
+            if (n > 0) {
+                good &= (((n >> 5) ? okw[1] : okw[0]) >> (n & 31) & 1u) != 0;
+                n = up;
+                ++depth;
+            }
+        }
+        if (mine && good) best_key = max(best_key, (depth << 10) | (1023 - i));
+    }
+    best_key = __reduce_max_sync(0xffffffffu, best_key);
+    const int best = 1023 - (best_key & 1023);
+    const int n_acc = (best_key >> 10) + 1;
+    if (err == kOk && (long long)P + n_acc > S_max) err = kErrCapacity;
+    const int n_out = (err == kOk) ? n_acc : 0;
+
+    path[0] = -1;
+    path[1] = -1;
+    int n = best;
+    for (int j = n_out - 1; j >= 0; --j) {   // warp-uniform trip count
+        if (lane == (j & 31)) path[j >> 5 ? 1 : 0] = n;
+        n = node_value(pa, n);
+    }
+    AcceptResult r;
+    r.n_acc = n_out;
+    const int nt = node_value(top, err == kOk ? best : 0);
+    r.next_token = (err == kOk) ? nt : -1;
+    r.new_prefix_len = (err == kOk) ? P + n_acc : P;
+    r.status = err;
+    return r;
+}
+
 // Exact matching (Section 3 step (2)): a candidate passes when it equals the
 // top-1 token predicted at its parent.
 template <class TopLoad>

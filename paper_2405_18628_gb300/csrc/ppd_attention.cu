@@ -194,7 +194,7 @@ tree_attention_kernel(const __grid_constant__ CUtensorMap map_q,
 
     if (warp == 10) {
         // ------------------------------------------------------------ fused-step side work
-        if (p.fused) fused_side_warp(p, wr, lane, abort_flag);
+        if (p.fused) fused_side_warp<true>(p, wr, lane, abort_flag);
     } else if (warp == 8) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {

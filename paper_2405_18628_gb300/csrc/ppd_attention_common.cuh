@@ -486,6 +486,7 @@ PPD_DEV bool side_wait_all(const AttnParams &p, unsigned long long tag, int lane
 // so the copies never race with it.  Scratch (parent copies, top-1 tokens,
 // path) lives in a per-CTA slice of the workspace.  Kept out of line so that
 // its code does not reshape the register allocation of the attention loops.
+template <bool kSmallTree>
 static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const WorkRange &wr, int lane,
                                                     volatile int *abort_flag)
 {
@@ -527,7 +528,9 @@ static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const W
             if (!side_wait_all(p, tag, lane, abort_flag)) return;
             have_all = true;
         }
-        for (int r = lane; r < T; r += 32) {
+        // node r's top-1 token from its partials (with typical acceptance also its
+        // log-sum-exp and entropy)
+        auto row_top = [&](int r, float &lse_r, float &ent_r) {
             const size_t base = ((size_t)b * T + r) * S;
             float bv = -INFINITY;
             int bi = INT_MAX;
@@ -560,33 +563,71 @@ static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const W
 #pragma unroll 8
                 for (int k = 0; k < S; ++k) consider(__ldcg(f.part_val + base + k), __ldcg(f.part_idx + base + k), bv, bi);
             }
-            top[r] = bi;
-            if (designated) f.argmax_out[(size_t)b * T + r] = bi;
-            if (f.typical) stats_finish(combine_stats(f.part_stats, (int64_t)b * T + r, S), s_lse[r], s_ent[r]);
-        }
-        __syncwarp();
-        const auto top_of = [&](int n) { return top[n]; };
-        const AcceptResult res =
-            f.typical
-                ? accept_warp_typical(top_of, f.logits + (size_t)b * T * f.V,
-                                      [&](int n) { return s_lse[n]; }, [&](int n) { return s_ent[n]; },
-                                      f.inv_temp, f.epsilon, f.delta, p.parent + (size_t)b * T,
-                                      f.cand_tokens + (size_t)b * T, __ldg(p.prefix_len + b), T, f.V,
-                                      p.S_max, lane, s_par, path)
-                : accept_warp(top_of, p.parent + (size_t)b * T, f.cand_tokens + (size_t)b * T,
-                              __ldg(p.prefix_len + b), T, f.V, p.S_max, lane, s_par, path);
-        if (designated) {
-            for (int i = lane; i < T; i += 32) f.path[(size_t)b * T + i] = path[i];
-            if (lane == 0) {
-                f.accept_len[b] = res.n_acc;
-                f.next_token[b] = res.next_token;
-                f.new_prefix_len[b] = res.new_prefix_len;
-                atomicMax(f.status + b, res.status);
+            if (f.typical) stats_finish(combine_stats(f.part_stats, (int64_t)b * T + r, S), lse_r, ent_r);
+            return bi;
+        };
+        const int32_t *par_b = p.parent + (size_t)b * T;
+        const int32_t *tok_b = f.cand_tokens + (size_t)b * T;
+        const int P = __ldg(p.prefix_len + b);
+        AcceptResult res;
+        // the accepted path: in registers (lane j % 32, slot j / 32) for trees of up
+        // to 64 nodes, else in the scratch
+        int path_r[2] = {-1, -1};
+        constexpr bool small = kSmallTree;   // the key-row kernel's trees: T <= 64
+        if constexpr (small) {
+            int top_r[2] = {0, 0};
+            float lse_r[2] = {0.f, 0.f}, ent_r[2] = {0.f, 0.f};
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int r = lane + 32 * k;
+                if (r < T) {
+                    top_r[k] = row_top(r, lse_r[k], ent_r[k]);
+                    if (designated) f.argmax_out[(size_t)b * T + r] = top_r[k];
+                }
             }
+            if (f.typical) {
+                const float *x = f.logits + (size_t)b * T * f.V;
+                res = accept_warp_small(
+                    top_r,
+                    [&](int, int pa, int tk) {
+                        const float pt = expf(__ldg(x + (size_t)pa * f.V + tk) * f.inv_temp - node_value(lse_r, pa));
+                        return pt > fminf(f.epsilon, f.delta * expf(-node_value(ent_r, pa)));
+                    },
+                    par_b, tok_b, P, T, f.V, p.S_max, lane, path_r);
+            } else {
+                res = accept_warp_small(
+                    top_r, [&](int, int pa, int tk) { return tk == node_value(top_r, pa); }, par_b, tok_b, P,
+                    T, f.V, p.S_max, lane, path_r);
+            }
+            if (designated) {
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    if (lane + 32 * k < T) f.path[(size_t)b * T + lane + 32 * k] = path_r[k];
+            }
+        } else {
+            for (int r = lane; r < T; r += 32) {
+                top[r] = row_top(r, s_lse[r], s_ent[r]);
+                if (designated) f.argmax_out[(size_t)b * T + r] = top[r];
+            }
+            __syncwarp();
+            const auto top_of = [&](int n) { return top[n]; };
+            res = f.typical
+                      ? accept_warp_typical(top_of, f.logits + (size_t)b * T * f.V,
+                                            [&](int n) { return s_lse[n]; }, [&](int n) { return s_ent[n]; },
+                                            f.inv_temp, f.epsilon, f.delta, par_b, tok_b, P, T, f.V, p.S_max,
+                                            lane, s_par, path)
+                      : accept_warp(top_of, par_b, tok_b, P, T, f.V, p.S_max, lane, s_par, path);
+            if (designated)
+                for (int i = lane; i < T; i += 32) f.path[(size_t)b * T + i] = path[i];
+        }
+        if (designated && lane == 0) {
+            f.accept_len[b] = res.n_acc;
+            f.next_token[b] = res.next_token;
+            f.new_prefix_len[b] = res.new_prefix_len;
+            atomicMax(f.status + b, res.status);
         }
         if (has_unit && res.n_acc > 0) {
             // cache rows [P_b, P_b + n_acc) <- the accepted tree rows
-            const int P = __ldg(p.prefix_len + b);
             const int n = res.n_acc;
             // each slice once: by the CTA holding the first tile of its first query block
             owns_first_tile([&](int u) {
@@ -600,9 +641,11 @@ static __device__ __noinline__ void fused_side_warp(const AttnParams &p, const W
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
                         const int w = w0 + u * 32 + lane;
-                        if (w < n * chunks) {
-                            const int j = w / chunks, c = w - j * chunks;
-                            const size_t so = ((size_t)lbh * T + path[j]) * f.row_bytes + (size_t)c * 16;
+                        const bool in = w < n * chunks;
+                        const int j = in ? w / chunks : 0, c = w - j * chunks;
+                        const int src = small ? node_value(path_r, j) : (in ? path[j] : 0);
+                        if (in) {
+                            const size_t so = ((size_t)lbh * T + src) * f.row_bytes + (size_t)c * 16;
                             dof[u] = ((size_t)lbh * p.S_max + P + j) * f.row_bytes + (size_t)c * 16;
                             kx[u] = __ldg(reinterpret_cast<const uint4 *>(f.k_tree + so));
                             vx[u] = __ldg(reinterpret_cast<const uint4 *>(f.v_tree + so));

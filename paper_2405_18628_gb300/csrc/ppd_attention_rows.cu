@@ -153,7 +153,7 @@ tree_attention_rows_kernel(const __grid_constant__ CUtensorMap map_q,
 
     if (warp == 10) {
         // ------------------------------------------------------------ fused-step side work
-        if (p.fused) fused_side_warp(p, wr, lane, abort_flag);
+        if (p.fused) fused_side_warp<false>(p, wr, lane, abort_flag);
     } else if (warp == 8) {
         // ------------------------------------------------------------ TMA producer
         // One queue of copies in the order the MMA issuer consumes them -- S(g)
