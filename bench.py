@@ -581,33 +581,37 @@ def copy_bandwidth(n_bytes, dev, reps=20):
 
 
 def e2e_groups(L):
-    """Layer groups of the pipelined end-to-end step, largest first in the
-    proportions 7 : 5 : 3 : 1 (14, 10, 6, 2 of 32 layers): the first group's
-    copy cannot overlap any compute, the last group's compute and copy back
-    cannot overlap any copy in, so the last group is the smallest.  Measured
-    at Vicuna-7B shapes: 0.435 ms per step against 0.482 for four equal
-    groups and 0.653 with one copy each way around the fused step."""
-    if L < 4:
+    """Layer groups of the pipelined end-to-end step, in the proportions
+    3 : 4 : 4 : 3 : 2 (6, 8, 8, 6, 4 of 32 layers): the first group's copy in
+    overlaps no compute and the last group's compute and copy back overlap no
+    copy in, so both are smaller; a group of a few layers is latency-bound
+    (one call streams few tiles per SM), so neither is tiny.  Measured at
+    Vicuna-7B shapes (device span of one graph replay): 424 us against 434
+    for 8 / 8 / 8 / 8 and 443 for 14 / 10 / 6 / 2."""
+    if L < 8:
         return [L]
-    parts = [7, 5, 3, 1]
+    parts = [3, 4, 4, 3, 2]
     sizes = [max(1, (p * L) // 16) for p in parts]
-    sizes[0] += L - sum(sizes)
+    sizes[1] += L - sum(sizes)
     return [n for n in sizes if n > 0]
 
 
-def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, in_streams=1):
+def e2e_pipelined(w, t, st, K, groups, dev, check_against=None):
     """The step end to end from pinned host buffers through the public C ABI,
-    with the copies overlapping the compute: the layers go in `groups` groups;
-    each group's Q / tree K / tree V are copied in on one copy stream, and its
-    attention (ppd_tree_attention) starts as soon as they have landed while
-    the next group's copy runs; the last group runs ppd_verify_step (node
-    argmax, acceptance, its layers' attention and compaction) once the logits
-    and index arrays are in too, then ppd_kv_compact writes the other groups'
-    accepted rows; every group's output is copied back on a second copy
-    stream as soon as it is done, and the index outputs last.  A step ends
-    with every result in host memory (stream synchronised).  Returns the
-    timing, the copied bytes and, with `check_against` (the device step's
-    outputs), the largest difference found."""
+    with the copies overlapping the compute.  The layers go in `groups` groups;
+    each group's Q / tree K / tree V are copied in on a copy stream, and its
+    attention (ppd_tree_attention) starts as soon as they have landed, on one
+    of two compute streams in turn (so one group's last, partial round of
+    slices overlaps the next group's first), while the next group's copy
+    runs; each group's output is copied back on a third stream as soon as it
+    is done.  The logits and index arrays are copied in last: node argmax
+    (ppd_node_argmax), acceptance (ppd_accept_path) and the compaction of
+    every layer's accepted rows (ppd_kv_compact) need no attention output, so
+    they run while the last groups' outputs are copied back, and the index
+    outputs follow.  A step ends with every result in host memory (stream
+    synchronised).  Returns the timing, the copied bytes and, with
+    `check_against` (the device step's outputs), the largest difference
+    found."""
     import torch
 
     from paper_2405_18628_gb300 import ppd
@@ -639,52 +643,51 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, in_streams=1):
     d_idx, di = packed({k: (shapes[k], torch.int32) for k in names}, dev)
     h_idx, hi = packed({k: (shapes[k], torch.int32) for k in names}, "cpu")
     st_grp = torch.zeros(groups, w.B, dtype=torch.int32, device=dev)
-    ws = st.bufs.workspace
-    s_ins = [torch.cuda.Stream() for _ in range(in_streams)]
-    s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    # one workspace per compute stream (a call's work split keeps its partial
+    # states there until its merge grid has run)
+    ws = [st.bufs.workspace, torch.zeros_like(st.bufs.workspace)]
+    s_in = torch.cuda.Stream()
+    s_cmp = [torch.cuda.Stream(), torch.cuda.Stream()]
+    s_out = torch.cuda.Stream()
     kc, vc = t["k_cache"], t["v_cache"]
 
     def one_step():
-        ev_in = [[torch.cuda.Event() for _ in s_ins] for _ in range(groups)]
+        ev_in = [torch.cuda.Event() for _ in range(groups)]
         ev_small = torch.cuda.Event()
         ev_done = [torch.cuda.Event() for _ in range(groups)]
         ev_idx = torch.cuda.Event()
-        # a group's three tensors spread over the copy streams (round-robin)
-        for g in range(groups):
-            a, b = bounds[g], bounds[g + 1]
-            if g == groups - 1:
-                with torch.cuda.stream(s_ins[0]):
-                    d_small.copy_(h_small, non_blocking=True)
-                    ev_small.record(s_ins[0])
-            for i, k in enumerate(("q", "k_tree", "v_tree")):
-                with torch.cuda.stream(s_ins[i % len(s_ins)]):
+        with torch.cuda.stream(s_in):
+            for g in range(groups):
+                a, b = bounds[g], bounds[g + 1]
+                for k in ("q", "k_tree", "v_tree"):
                     d[k][a:b].copy_(h[k][a:b], non_blocking=True)
-            for j, sj in enumerate(s_ins):
-                ev_in[g][j].record(sj)
+                ev_in[g].record(s_in)
+            d_small.copy_(h_small, non_blocking=True)
+            ev_small.record(s_in)
         for g in range(groups):
             a, b = bounds[g], bounds[g + 1]
-            for e in ev_in[g]:
-                s_cmp.wait_event(e)
+            sc = s_cmp[g % 2]
+            sc.wait_event(ev_in[g])
             sl = lambda x: x[a:b]
-            if g < groups - 1:
-                ppd.ppd_tree_attention(sl(d["q"]), sl(kc), sl(vc), sl(d["k_tree"]), sl(d["v_tree"]),
-                                       ds["prefix"], ds["parent"], sl(out), st_grp[g], workspace=ws,
-                                       stream=s_cmp)
-            else:
-                s_cmp.wait_event(ev_small)
-                ppd.ppd_verify_step(sl(d["q"]), sl(kc), sl(vc), sl(d["k_tree"]), sl(d["v_tree"]),
-                                    ds["prefix"], ds["parent"], ds["cand"], ds["logits"], sl(out),
-                                    di["argmax"], di["accept_len"], di["path"], di["next_token"],
-                                    di["new_prefix_len"], di["dev_status"], ws, stream=s_cmp)
-            ev_done[g].record(s_cmp)
+            ppd.ppd_tree_attention(sl(d["q"]), sl(kc), sl(vc), sl(d["k_tree"]), sl(d["v_tree"]),
+                                   ds["prefix"], ds["parent"], sl(out), st_grp[g], workspace=ws[g % 2],
+                                   stream=sc)
+            ev_done[g].record(sc)
             s_out.wait_event(ev_done[g])
             with torch.cuda.stream(s_out):
                 h_out[a:b].copy_(out[a:b], non_blocking=True)
-        if groups > 1:
-            b0 = bounds[groups - 1]
-            ppd.ppd_kv_compact(kc[:b0], vc[:b0], d["k_tree"][:b0], d["v_tree"][:b0], di["path"],
-                               di["accept_len"], ds["prefix"], stream=s_cmp)
-        ev_idx.record(s_cmp)
+        # argmax, acceptance and compaction once the logits are in and both
+        # compute streams are done with the attention
+        sc = s_cmp[groups % 2]
+        sc.wait_event(ev_small)
+        sc.wait_stream(s_cmp[(groups + 1) % 2])
+        ppd.ppd_node_argmax(ds["logits"], di["argmax"], workspace=ws[groups % 2], stream=sc)
+        ppd.ppd_accept_path(di["argmax"], ds["cand"], ds["parent"], ds["prefix"], w.V, w.S_max,
+                            di["accept_len"], di["path"], di["next_token"], di["new_prefix_len"],
+                            di["dev_status"], stream=sc)
+        ev_idx.record(sc)
+        ppd.ppd_kv_compact(kc, vc, d["k_tree"], d["v_tree"], di["path"], di["accept_len"],
+                           ds["prefix"], stream=sc)
         s_out.wait_event(ev_idx)
         with torch.cuda.stream(s_out):
             h_idx.copy_(d_idx, non_blocking=True)
@@ -699,10 +702,10 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, in_streams=1):
     cap = torch.cuda.Stream()
     cap.wait_stream(torch.cuda.current_stream())
     with torch.cuda.graph(graph, stream=cap):
-        for x in (*s_ins, s_cmp, s_out):
+        for x in (s_in, *s_cmp, s_out):
             x.wait_stream(cap)
         one_step()
-        for x in (*s_ins, s_cmp, s_out):
+        for x in (s_in, *s_cmp, s_out):
             cap.wait_stream(x)
     torch.cuda.synchronize()
     for _ in range(3):
@@ -953,13 +956,14 @@ def main(argv=None):
                          "matches_device_step": ok, "max_abs_diff_out": pip["max_abs_diff_out"],
                          "note": "KV cache resident on the device; the layers in groups of "
                                  + "/".join(str(n) for n in e2e_groups(w.L)) + ", each "
-                                 "group's tree tensors copied in on one stream while the previous "
-                                 "group's attention runs (ppd_tree_attention; the last group "
-                                 "ppd_verify_step with the logits and index arrays, then "
-                                 "ppd_kv_compact for the other groups' accepted rows), each "
-                                 "group's output copied back on another stream as soon as it is "
-                                 "done; the copies and calls of a step captured once in a CUDA "
-                                 "graph and replayed once per step"}
+                                 "group's tree tensors copied in on one stream and its attention "
+                                 "(ppd_tree_attention) run as soon as they have landed, on two "
+                                 "compute streams in turn, its output copied back on a third as "
+                                 "soon as it is done; the logits and index arrays copied in last, "
+                                 "then ppd_node_argmax, ppd_accept_path and ppd_kv_compact (all "
+                                 "layers) and the index outputs copied back; the copies and calls "
+                                 "of a step captured once in a CUDA graph and replayed once per "
+                                 "step"}
             if ok:
                 e2e = dict(pipelined)
                 e2e["serial"] = serial
