@@ -71,10 +71,12 @@ REFERENCE_BUDGET_S = 180.0
 # are not in the count, so this is the reads plus the part of the writes that
 # reached DRAM during the launch.
 MEASURED_TRAFFIC = {
-    # 675,924,224 B at 19 layers (reads 667,973,120), x 32/19
-    "vicuna7b": {"bytes_per_launch": 1_138_398_693, "src": "6cc40380e523c3a7"},
-    # 1,658,914,816 B at 19 layers (reads 1,650,980,352), x 40/19
-    "vicuna13b": {"bytes_per_launch": 3_492_452_244, "src": "6cc40380e523c3a7"},
+    # 676,180,992 B at 19 layers (reads 667,975,936), x 32/19
+    "vicuna7b": {"bytes_per_launch": 1_138_831_144, "src": "028eaf175014bde9"},
+    # 1,658,903,808 B at 19 layers (reads 1,650,978,560), x 40/19
+    "vicuna13b": {"bytes_per_launch": 3_492_429_069, "src": "028eaf175014bde9"},
+    # 123,361,024 B, a fused-step launch at the full 24 layers (reads 119,708,928)
+    "mobilellama": {"bytes_per_launch": 123_361_024, "src": "028eaf175014bde9"},
 }
 
 
