@@ -68,6 +68,9 @@ def measure_step_latency(w: W.Workload, steps: int = 30, warmup: int = 5, device
           for _ in range(steps)]
     torch.cuda.synchronize()
     with (timed if timed is not None else contextlib.nullcontext()):
+        # a ~1 ms spin first, outside the events, so that the host has queued the
+        # first steps before the GPU reaches them
+        torch.cuda._sleep(2_000_000)
         for a, b in ev:
             if flush is not None:
                 flush.zero_()
