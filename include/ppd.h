@@ -346,6 +346,12 @@ int ppd_set_verify_step_form(int form);
  */
 ppd_status ppd_debug_grid_wait(unsigned long long limit_ns, int withhold_cta);
 
+/*
+ * Name of the CUDA error behind the most recent PPD_ERR_CUDA returned in this
+ * process ("cudaSuccess" if none; static string; diagnostics).
+ */
+const char *ppd_last_cuda_error(void);
+
 /* Human-readable name of a status code (static string). */
 const char *ppd_status_string(ppd_status s);
 

@@ -207,7 +207,27 @@ bool encode_2d(CUtensorMap *m, const void *base, uint64_t inner, uint64_t rows, 
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-ppd_status cuda_status(cudaError_t e) { return e == cudaSuccess ? PPD_OK : PPD_ERR_CUDA; }
+// The CUDA error behind the latest PPD_ERR_CUDA of this process (diagnostics).
+std::atomic<int> g_last_cuda_error{cudaSuccess};
+
+// A launch reported failed through the runtime's last error (kernels launched
+// with <<< >>>): record it and clear it.
+ppd_status cuda_failed()
+{
+    const cudaError_t e = cudaGetLastError();
+    g_last_cuda_error.store((int)(e != cudaSuccess ? e : cudaErrorUnknown), std::memory_order_relaxed);
+    return PPD_ERR_CUDA;
+}
+
+// A failed call clears the runtime's last-error state (errors that do not
+// break the context), so it cannot surface as the status of a later call.
+ppd_status cuda_status(cudaError_t e)
+{
+    if (e == cudaSuccess) return PPD_OK;
+    g_last_cuda_error.store((int)e, std::memory_order_relaxed);
+    (void)cudaGetLastError();
+    return PPD_ERR_CUDA;
+}
 
 // ------------------------------------------------------------------ shared checks
 
@@ -332,7 +352,7 @@ ppd_status enqueue_attention_any(const void *q, const void *kc, const void *vc, 
         ppd::launch_round_bf16((const float *)vt, bvt, n_t, stream) != cudaSuccess ||
         ppd::launch_round_bf16((const float *)kc, bkc, n_c, stream) != cudaSuccess ||
         ppd::launch_round_bf16((const float *)vc, bvc, n_c, stream) != cudaSuccess)
-        return PPD_ERR_CUDA;
+        return cuda_failed();
     return enqueue_attention(bq, bkc, bvc, bkt, bvt, prefix_len, parent, L, B, H, T, D, S_max,
                              scale, out, lse, dev_status, ws, &wl, fused, false, false, stream);
 }
@@ -420,7 +440,7 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
                                                            temp, dev_status, B, s)
                                : ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temp,
                                                              dev_status, B, s);
-                if (e != cudaSuccess) return PPD_ERR_CUDA;
+                if (e != cudaSuccess) return cuda_status(e);
             }
             // 2. attention over every layer, overlapping step 1; its side warps combine
             //    the argmax, decide acceptance and compact the accepted rows
@@ -450,7 +470,7 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
             if (in_grid) {
                 // no argmax grid to zero the status first: a one-block reset does,
                 // so that every status write can be an atomic maximum
-                if (ppd::launch_zero_status(dev_status, B, s) != cudaSuccess) return PPD_ERR_CUDA;
+                if (ppd::launch_zero_status(dev_status, B, s) != cudaSuccess) return cuda_failed();
                 const unsigned long long lim = g_grid_wait_ns.load(std::memory_order_relaxed);
                 f.wait_limit_ns = lim ? lim : ppd::kWaitLimitNs;
                 f.withhold_cta = g_withhold_cta.load(std::memory_order_relaxed);
@@ -473,7 +493,8 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
             if (st == PPD_OK || !in_grid) return st;
             // the cooperative launch could not have every CTA resident (SMs taken by
             // other work): clear its error and run the argmax as its own grid
-            if (cudaGetLastError() != cudaErrorCooperativeLaunchTooLarge) return st;
+            if (g_last_cuda_error.load(std::memory_order_relaxed) != cudaErrorCooperativeLaunchTooLarge)
+                return st;
             in_grid = false;
         }
     }
@@ -483,7 +504,7 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
                  dev_status, T, V, S_max};
     if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temp, nullptr, 0, s) !=
         cudaSuccess)
-        return PPD_ERR_CUDA;
+        return cuda_failed();
     if (typ) {
         float *nl = reinterpret_cast<float *>(ws + wl.node_lse);
         float *ne = reinterpret_cast<float *>(ws + wl.node_ent);
@@ -491,11 +512,11 @@ static ppd_status verify_step_impl(const void *q, void *k_cache, void *v_cache,
                 cudaSuccess ||
             ppd::launch_typical_accept(logits, nl, ne, argmax_out, a, B, typ->temperature,
                                        typ->epsilon, typ->delta, s) != cudaSuccess)
-            return PPD_ERR_CUDA;
+            return cuda_failed();
     } else {
         if (ppd::launch_argmax_combine(pv, pi, rows, wl.splits, argmax_out, s) != cudaSuccess ||
             ppd::launch_accept_path(argmax_out, a, B, s) != cudaSuccess)
-            return PPD_ERR_CUDA;
+            return cuda_failed();
     }
     ppd_status st = enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent,
                                           L, B, H, T, D, S_max, dt, scale, out, lse, dev_status,
@@ -555,6 +576,11 @@ size_t ppd_workspace_bytes(int L, int B, int H, int T, int D, int V, int S_max, 
 }
 
 
+const char *ppd_last_cuda_error(void)
+{
+    return cudaGetErrorName((cudaError_t)g_last_cuda_error.load(std::memory_order_relaxed));
+}
+
 const char *ppd_status_string(ppd_status s)
 {
     switch (s) {
@@ -592,7 +618,7 @@ ppd_status ppd_tree_attention(const void *q, const void *k_cache, const void *v_
     // grid is its programmatic dependent in turn, so a sequence of calls (one
     // per layer, as a model runs them) launches each grid while the previous
     // one still runs and only the setup that reads no input runs early
-    if (ppd::launch_zero_status(dev_status, B, s) != cudaSuccess) return PPD_ERR_CUDA;
+    if (ppd::launch_zero_status(dev_status, B, s) != cudaSuccess) return cuda_failed();
     // a bf16 call without a full workspace runs unsplit
     return enqueue_attention_any(q, k_cache, v_cache, k_tree, v_tree, prefix_len, parent, L, B, H,
                                  T, D, S_max, dt, scale, out, lse, dev_status,
@@ -614,7 +640,7 @@ ppd_status ppd_node_argmax(const float *logits, int B, int T, int V, int32_t *ar
     const int64_t rows = (int64_t)B * T;
     if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, nullptr, 1.f, nullptr, 0, s) !=
         cudaSuccess)
-        return PPD_ERR_CUDA;
+        return cuda_failed();
     return cuda_status(ppd::launch_argmax_combine(pv, pi, rows, wl.splits, argmax_out, s));
 }
 
@@ -711,7 +737,7 @@ ppd_status ppd_node_stats(const float *logits, int B, int T, int V, float temper
     const int64_t rows = (int64_t)B * T;
     if (ppd::launch_argmax_partials(logits, rows, V, wl.splits, pv, pi, pst, temperature, nullptr, 0,
                                     s) != cudaSuccess)
-        return PPD_ERR_CUDA;
+        return cuda_failed();
     return cuda_status(ppd::launch_node_stats_combine(pv, pi, pst, rows, wl.splits, argmax_out,
                                                       lse_out, entropy_out, s));
 }

@@ -26,7 +26,10 @@ _lib = None
 
 class PPDError(RuntimeError):
     def __init__(self, status: int, where: str):
-        super().__init__(f"{where}: {status_string(status)} (status {status})")
+        msg = f"{where}: {status_string(status)} (status {status})"
+        if status == PPD_ERR_CUDA and _lib is not None:
+            msg += f", {_lib.ppd_last_cuda_error().decode()}"
+        super().__init__(msg)
         self.status = status
 
 
@@ -47,6 +50,8 @@ def load() -> ctypes.CDLL:
             "ppd_set_verify_step_form": ([i32], i32),
             "ppd_debug_grid_wait": ([ctypes.c_ulonglong, i32], i32),
             "ppd_status_string": ([i32], ctypes.c_char_p),
+            "ppd_last_cuda_error": ([], ctypes.c_char_p),
+            "ppd_last_cuda_error": ([], ctypes.c_char_p),
             "ppd_tree_attention": ([vp] * 7 + [i32] * 7 + [f32, vp, vp, vp, vp, sz, vp], i32),
             "ppd_node_argmax": ([vp, i32, i32, i32, vp, vp, sz, vp], i32),
             "ppd_accept_path": ([vp] * 4 + [i32] * 4 + [vp] * 5 + [vp], i32),

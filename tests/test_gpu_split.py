@@ -118,3 +118,25 @@ def test_workspace_contents_do_not_matter(cuda_device):
         out, _, st = _attend(t_dev, pl, parent, cuda_device, ws)
         assert (st == 0).all()
         assert_attn_close(out.reshape(ref.shape), ref, f"workspace filled with {fill:#x}")
+
+
+def test_split_status_per_call(cuda_device):
+    """Per-sequence status on the split path: a malformed tree and a prefix
+    beyond the cache are reported over a status array holding junk, and the
+    next call on the same workspace, with clean inputs, reports neither and
+    matches the oracle."""
+    L, B, H, T, D, S_max = 1, 3, 2, 48, 64, 2048
+    t, pl, parent = _case(L, B, H, T, D, [2000, 1500, 2000], S_max, seed=11)
+    t_dev = {k: v.to(cuda_device) for k, v in t.items()}
+    ws = ppd.workspace(L, B, H, T, D, 1, S_max, device=cuda_device)
+    bad_parent = parent.copy()
+    bad_parent[1, 5] = 7            # not before its child
+    bad_pl = pl.copy()
+    bad_pl[2] = t["k_cache"].shape[3] + 1   # beyond the cache
+    _, _, st = _attend(t_dev, bad_pl, bad_parent, cuda_device, ws)
+    assert st.tolist() == [0, ppd.PPD_ERR_TREE, ppd.PPD_ERR_CAPACITY]
+    ref, _, _, _ = oracle.tree_attention(t["q"], t["k_cache"], t["v_cache"], t["k_tree"],
+                                         t["v_tree"], pl, parent)
+    out, _, st = _attend(t_dev, pl, parent, cuda_device, ws)
+    assert (st == 0).all(), st
+    assert_attn_close(out.reshape(ref.shape), ref, "clean call after a failed one")
