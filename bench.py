@@ -610,7 +610,7 @@ def e2e_groups(L):
     return [n for n in sizes if n > 0]
 
 
-def e2e_pipelined(w, t, st, K, groups, dev, check_against=None):
+def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, n_cmp=2):
     """The step end to end from pinned host buffers through the public C ABI,
     with the copies overlapping the compute.  The layers go in `groups` groups;
     each group's Q / tree K / tree V are copied in on a copy stream, and its
@@ -659,9 +659,9 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None):
     st_grp = torch.zeros(groups, w.B, dtype=torch.int32, device=dev)
     # one workspace per compute stream (a call's work split keeps its partial
     # states there until its merge grid has run)
-    ws = [st.bufs.workspace, torch.zeros_like(st.bufs.workspace)]
+    ws = [st.bufs.workspace] + [torch.zeros_like(st.bufs.workspace) for _ in range(n_cmp - 1)]
     s_in = torch.cuda.Stream()
-    s_cmp = [torch.cuda.Stream(), torch.cuda.Stream()]
+    s_cmp = [torch.cuda.Stream() for _ in range(n_cmp)]
     s_out = torch.cuda.Stream()
     kc, vc = t["k_cache"], t["v_cache"]
 
@@ -680,11 +680,11 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None):
             ev_small.record(s_in)
         for g in range(groups):
             a, b = bounds[g], bounds[g + 1]
-            sc = s_cmp[g % 2]
+            sc = s_cmp[g % n_cmp]
             sc.wait_event(ev_in[g])
             sl = lambda x: x[a:b]
             ppd.ppd_tree_attention(sl(d["q"]), sl(kc), sl(vc), sl(d["k_tree"]), sl(d["v_tree"]),
-                                   ds["prefix"], ds["parent"], sl(out), st_grp[g], workspace=ws[g % 2],
+                                   ds["prefix"], ds["parent"], sl(out), st_grp[g], workspace=ws[g % n_cmp],
                                    stream=sc)
             ev_done[g].record(sc)
             s_out.wait_event(ev_done[g])
@@ -692,10 +692,12 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None):
                 h_out[a:b].copy_(out[a:b], non_blocking=True)
         # argmax, acceptance and compaction once the logits are in and both
         # compute streams are done with the attention
-        sc = s_cmp[groups % 2]
+        sc = s_cmp[groups % n_cmp]
         sc.wait_event(ev_small)
-        sc.wait_stream(s_cmp[(groups + 1) % 2])
-        ppd.ppd_node_argmax(ds["logits"], di["argmax"], workspace=ws[groups % 2], stream=sc)
+        for other in s_cmp:
+            if other is not sc:
+                sc.wait_stream(other)
+        ppd.ppd_node_argmax(ds["logits"], di["argmax"], workspace=ws[groups % n_cmp], stream=sc)
         ppd.ppd_accept_path(di["argmax"], ds["cand"], ds["parent"], ds["prefix"], w.V, w.S_max,
                             di["accept_len"], di["path"], di["next_token"], di["new_prefix_len"],
                             di["dev_status"], stream=sc)
