@@ -83,6 +83,10 @@ def _load():
                                          c_int, c_int, i32p, i32p, c_int, c_int, i32p, i32p, i32p,
                                          i32p]
         lib.oracle_next_tree.restype = c_int
+        lib.oracle_next_tree_ept.argtypes = [vp, i32p, i32p, i32p, i32p, i32p, c_int, c_int, c_int,
+                                             c_int, c_int, i32p, i32p, c_int, c_int, c_int, i32p,
+                                             i32p, i32p, i32p]
+        lib.oracle_next_tree_ept.restype = c_int
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = c_int
         _lib = lib
@@ -258,11 +262,14 @@ def topk(logits, K: int) -> np.ndarray:
 
 
 def next_tree(logits, parent, cand_tokens, path, accept_len, next_token, tmpl_parent, tmpl_rank,
-              K: int, n_ept: int = 1):
+              K: int, n_ept: int = 1, ept_mean: str = "logits"):
     """Next-step candidate tree.  logits [B,T,V]; parent, cand_tokens, path
     [B,T]; accept_len, next_token [B]; tmpl_parent, tmpl_rank [n_states,
-    T_next]; n_ept ensemble prompt tokens per position.  Returns dict of
-    next_parent, next_cand [B,T_next], next_state, status [B]."""
+    T_next]; n_ept ensemble prompt tokens per position, whose logits
+    (ept_mean="logits") or probabilities (ept_mean="probs") are averaged.
+    Returns dict of next_parent, next_cand [B,T_next], next_state, status [B]."""
+    if ept_mean not in ("logits", "probs"):
+        raise ValueError(f"ept_mean must be 'logits' or 'probs', not {ept_mean!r}")
     lg, _ = _host(logits)
     lg = np.ascontiguousarray(lg, dtype=np.float32)
     par, cd, pth, al, nt = (_i32(x) for x in (parent, cand_tokens, path, accept_len, next_token))
@@ -273,9 +280,10 @@ def next_tree(logits, parent, cand_tokens, path, accept_len, next_token, tmpl_pa
     res = {"next_parent": np.empty((B, T_next), np.int32), "next_cand": np.empty((B, T_next), np.int32),
            "next_state": np.empty(B, np.int32), "status": np.empty(B, np.int32)}
     p = lambda a: _ptr(a, ctypes.c_int32)
-    rc = _load().oracle_next_tree(_ptr(lg), p(par), p(cd), p(pth), p(al), p(nt), B, T, V, n_states,
-                                  T_next, p(tp), p(tr), int(K), int(n_ept), p(res["next_parent"]),
-                                  p(res["next_cand"]), p(res["next_state"]), p(res["status"]))
+    rc = _load().oracle_next_tree_ept(_ptr(lg), p(par), p(cd), p(pth), p(al), p(nt), B, T, V,
+                                      n_states, T_next, p(tp), p(tr), int(K), int(n_ept),
+                                      int(ept_mean == "probs"), p(res["next_parent"]),
+                                      p(res["next_cand"]), p(res["next_state"]), p(res["status"]))
     if rc != 0:
         raise ValueError(f"oracle_next_tree rejected its arguments (code {rc})")
     return res

@@ -29,6 +29,9 @@
  *   oracle_next_tree       next-step candidate tree from the accepted node's
  *                          prompt tokens (Section 3 step (1); Appendix,
  *                          tree states T_k)
+ *   oracle_next_tree_ept   the same with the ensemble chains' probabilities
+ *                          averaged instead of their logits (the formula of
+ *                          Section 3, "Ensemble Prompt Tokens")
  *
  * Status codes (per sequence): 0 ok, 3 malformed tree, 4 capacity / prefix
  * length out of range.  Whole-call argument errors return 1.
@@ -499,6 +502,51 @@ void oracle_topk(const float *logits, int64_t rows, int64_t V, int K, int32_t *o
     free(taken);
 }
 
+/* The K best of x[0..V) in ranking order (NaN first, then larger, then lower index). */
+static int ranks_before_d(double av, int64_t ai, double bv, int64_t bi)
+{
+    int an = isnan(av), bn = isnan(bv);
+    if (an || bn)
+        return an && bn ? ai < bi : an;
+    if (av != bv)
+        return av > bv;
+    return ai < bi;
+}
+
+static void topk_d(const double *x, int64_t V, int K, int32_t *out, char *taken)
+{
+    memset(taken, 0, (size_t)V);
+    for (int k = 0; k < K; ++k) {
+        int64_t best = -1;
+        for (int64_t v = 0; v < V; ++v)
+            if (!taken[v] && (best < 0 || ranks_before_d(x[v], v, x[best], best)))
+                best = v;
+        taken[best] = 1;
+        out[k] = (int32_t)best;
+    }
+}
+
+/* ln sum_v exp(x[v]) in fp64, shifted by the row's maximum: NaN if the row
+ * holds a NaN, or if its maximum is +inf or -inf (so every probability of
+ * such a row is NaN). */
+static double row_lse(const float *x, int64_t V)
+{
+    double m = -INFINITY;
+    int nan_seen = 0;
+    for (int64_t v = 0; v < V; ++v) {
+        if (isnan(x[v]))
+            nan_seen = 1;
+        else if ((double)x[v] > m)
+            m = (double)x[v];
+    }
+    if (nan_seen)
+        return NAN;
+    double sum = 0.0;
+    for (int64_t v = 0; v < V; ++v)
+        sum += exp((double)x[v] - m);
+    return m + log(sum);
+}
+
 /*
  * Next-step candidate tree of each sequence (Section 3 step (1): the prompt
  * tokens appended to a guess token predict the tokens after it; Appendix,
@@ -525,14 +573,28 @@ void oracle_topk(const float *logits, int64_t rows, int64_t V, int K, int32_t *o
  * template k is not a tree in topological order, has a candidate below a
  * prompt node, a candidate deeper than k, or a rank outside [0, K).
  */
-int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *cand,
-                     const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
-                     int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
-                     const int32_t *tmpl_rank, int K, int n_ept, int32_t *next_parent,
-                     int32_t *next_cand, int32_t *next_state, int32_t *status)
+/*
+ * ept_mean = 1 (oracle_next_tree_ept): with n_ept > 1 the guesses for depth d
+ * are instead the K best tokens of the mean of the chains' probabilities at
+ * position d, p(v) = (1/n_ept) sum_j exp(x_j[v] - lse_j), lse_j = ln sum_v
+ * exp(x_j[v]), all in fp64 (row_lse: a chain row holding a NaN or a +-inf
+ * maximum makes every p NaN); ranked like the logits (NaN first, then larger,
+ * then lower index).  n_ept = 1 ranks the plain logits, which order the
+ * tokens as their probabilities do.  ept_mean = 0 is oracle_next_tree.
+ */
+int oracle_next_tree_ept(const float *logits, const int32_t *parent, const int32_t *cand,
+                         const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
+                         int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
+                         const int32_t *tmpl_rank, int K, int n_ept, int ept_mean,
+                         int32_t *next_parent, int32_t *next_cand, int32_t *next_state,
+                         int32_t *status)
 {
-    if (B < 1 || T < 1 || V < 1 || n_states < 1 || T_next < 1 || K < 1 || K > V || n_ept < 1)
+    if (B < 1 || T < 1 || V < 1 || n_states < 1 || T_next < 1 || K < 1 || K > V || n_ept < 1 ||
+        ept_mean < 0 || ept_mean > 1)
         return ORC_ERR_INVALID_ARG;
+    double *pmean = (double *)malloc(sizeof(double) * (size_t)V);
+    double *lse = (double *)malloc(sizeof(double) * (size_t)n_ept);
+    char *taken = (char *)malloc((size_t)V);
     int32_t *top = (int32_t *)malloc(sizeof(int32_t) * (size_t)K);
     int *cdepth = (int *)malloc(sizeof(int) * (size_t)T_next);
     int *chain = (int *)malloc(sizeof(int) * (size_t)(T + 1) * (size_t)n_ept);
@@ -602,13 +664,26 @@ int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *
                 }
                 nc[0] = next_token[b];
                 for (int d = 1; d <= k; ++d) {
-                    for (int64_t v = 0; v < V; ++v) {
-                        float sum = logits[((int64_t)b * T + chain[d - 1]) * V + v];
-                        for (int j = 1; j < n_ept; ++j)
-                            sum += logits[((int64_t)b * T + chain[(int64_t)j * (T + 1) + d - 1]) * V + v];
-                        avg[v] = sum / (float)n_ept;
+                    if (ept_mean == 1 && n_ept > 1) {
+                        /* the chains' probabilities at position d, averaged */
+                        for (int j = 0; j < n_ept; ++j)
+                            lse[j] = row_lse(logits + ((int64_t)b * T + chain[(int64_t)j * (T + 1) + d - 1]) * V, V);
+                        for (int64_t v = 0; v < V; ++v) {
+                            double sum = 0.0;
+                            for (int j = 0; j < n_ept; ++j)
+                                sum += exp((double)logits[((int64_t)b * T + chain[(int64_t)j * (T + 1) + d - 1]) * V + v] - lse[j]);
+                            pmean[v] = sum / (double)n_ept;
+                        }
+                        topk_d(pmean, V, K, top, taken);
+                    } else {
+                        for (int64_t v = 0; v < V; ++v) {
+                            float sum = logits[((int64_t)b * T + chain[d - 1]) * V + v];
+                            for (int j = 1; j < n_ept; ++j)
+                                sum += logits[((int64_t)b * T + chain[(int64_t)j * (T + 1) + d - 1]) * V + v];
+                            avg[v] = sum / (float)n_ept;
+                        }
+                        oracle_topk(avg, 1, V, K, top);
                     }
-                    oracle_topk(avg, 1, V, K, top);
                     for (int i = 1; i < T_next; ++i)
                         if (tr[i] >= 0 && cdepth[i] == d)
                             nc[i] = top[tr[i]];
@@ -629,7 +704,21 @@ int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *
     free(cdepth);
     free(chain);
     free(avg);
+    free(pmean);
+    free(lse);
+    free(taken);
     return ORC_OK;
+}
+
+int oracle_next_tree(const float *logits, const int32_t *parent, const int32_t *cand,
+                     const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
+                     int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
+                     const int32_t *tmpl_rank, int K, int n_ept, int32_t *next_parent,
+                     int32_t *next_cand, int32_t *next_state, int32_t *status)
+{
+    return oracle_next_tree_ept(logits, parent, cand, path, accept_len, next_token, B, T, V,
+                                n_states, T_next, tmpl_parent, tmpl_rank, K, n_ept, 0, next_parent,
+                                next_cand, next_state, status);
 }
 
 /* ------------------------------------------------------------------ compaction */

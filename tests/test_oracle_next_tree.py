@@ -65,11 +65,23 @@ def test_hand_worked_example():
     assert r["next_cand"][0].tolist() == [4, 2, 3, 5, -1, -1]
 
 
-def _independent(logits, parent, cand, path, accept_len, next_token, tp, tr, K, n_ept=1):
+def _softmax_rows(x):
+    """fp64 softmax of each row, written out: a row holding a NaN, or whose
+    largest entry is +inf or -inf, gives NaN everywhere (numpy's inf - inf)."""
+    x = np.asarray(x, np.float64)
+    m = np.where(np.isnan(x).any(-1), np.nan, np.max(np.where(np.isnan(x), -np.inf, x), -1))
+    with np.errstate(invalid="ignore"):
+        lse = m + np.log(np.exp(x - m[..., None]).sum(-1))
+        return np.exp(x - lse[..., None])
+
+
+def _independent(logits, parent, cand, path, accept_len, next_token, tp, tr, K, n_ept=1,
+                 ept_mean="logits"):
     """Restatement: per-node lists of prompt children (lowest index first); the
     end node's first n_ept prompt children head the chains, each continued
     through first children; the average over the chains is an explicit fp32
-    loop; ranks come from numpy."""
+    loop over logits, or (ept_mean="probs", n_ept > 1) the fp64 mean of the
+    chains' softmax rows; ranks come from numpy."""
     B, T = parent.shape
     n_states, T_next = tp.shape
     out_p = np.full((B, T_next), -1)
@@ -90,10 +102,13 @@ def _independent(logits, parent, cand, path, accept_len, next_token, tp, tr, K, 
         k = min(k, n_states - 1)
         ranks = []
         for d in range(k):
-            acc = np.array(logits[b, chains[0][d]], np.float32)
-            for c in chains[1:]:
-                acc = (acc + logits[b, c[d]]).astype(np.float32)
-            avg = (acc / np.float32(n_ept)).astype(np.float32)
+            if ept_mean == "probs" and n_ept > 1:
+                avg = _softmax_rows(np.stack([logits[b, c[d]] for c in chains])).mean(0)
+            else:
+                acc = np.array(logits[b, chains[0][d]], np.float32)
+                for c in chains[1:]:
+                    acc = (acc + logits[b, c[d]]).astype(np.float32)
+                avg = (acc / np.float32(n_ept)).astype(np.float32)
             nan = np.isnan(avg)          # NaN ranks first; numpy would sort it last
             ranks.append(np.lexsort((np.arange(logits.shape[2]), -np.where(nan, 0, avg), ~nan))[:K])
         depth = {0: 0}
@@ -165,6 +180,46 @@ def test_ept_hand_worked_example():
     assert r3["next_state"].tolist() == [0] and r3["next_cand"][0].tolist() == [7, -1, -1, -1, -1]
 
 
+def test_ept_probability_mean_hand_worked_example():
+    """The same tree with the chains' probabilities averaged (softmax by hand):
+    position 1 -> mean [0.4615, 0.5026, 0.0262, 0.0097], ranking 1, 0, 2, 3;
+    position 2 -> chain 1 softmax [0.0170, 0.9304, 0.0063, 0.0463], chain 2
+    [0.7052, 0.0002, 0.0351, 0.2594], mean [0.3611, 0.4653, 0.0207, 0.1529],
+    ranking 1, 0, 3, 2 -- where the logit average ranks 0, 3 first."""
+    logits, parent, cand, path, alen, nt, tp, tr = _ept_hand_tree()
+    r = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=2,
+                         ept_mean="probs")
+    assert r["status"].tolist() == [0] and r["next_state"].tolist() == [2]
+    assert r["next_parent"][0].tolist() == [-1, 0, 1, 1, 0]
+    assert r["next_cand"][0].tolist() == [7, 1, 1, 0, -1]
+    # one ensemble token: the probabilities rank as the logits do
+    for n in (1, 3):
+        rp = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=n,
+                              ept_mean="probs")
+        rl = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=n)
+        for k in rp:
+            np.testing.assert_array_equal(rp[k], rl[k], err_msg=k)
+    with pytest.raises(ValueError):
+        oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=2,
+                         ept_mean="mean")
+
+
+def test_ept_probability_mean_is_shift_invariant():
+    """Softmax ignores a constant added to a row: shifting one chain's logits by
+    a large constant leaves the probability-mean guesses unchanged.  Averaging
+    unnormalised exp(x) instead would let the shifted chain decide alone
+    (guesses 7, 1, 0, 3)."""
+    logits, parent, cand, path, alen, nt, tp, tr = _ept_hand_tree()
+    a = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=2,
+                         ept_mean="probs")
+    for c in (40.0, -60.0):
+        shifted = logits.copy()
+        shifted[0, [3, 5]] += c         # chain 2, both positions
+        b = oracle.next_tree(shifted, parent, cand, path, alen, nt, tp, tr, K=2, n_ept=2,
+                             ept_mean="probs")
+        np.testing.assert_array_equal(a["next_cand"], b["next_cand"])
+
+
 def test_ept_state_is_the_shortest_chain():
     logits, parent, cand, path, alen, nt, tp, tr = _ept_hand_tree()
     parent = parent.copy()
@@ -201,13 +256,18 @@ def test_ept_identical_chains_match_one_chain(n_ept):
                          acc["next_token"], tp, tr, 4, n_ept=n_ept)
     r1 = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
                           acc["next_token"], tp, tr, 4, n_ept=1)
+    # the probabilities of n_ept equal rows average (fp64, 2^j of them) to one row's
+    rp = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                          acc["next_token"], tp, tr, 4, n_ept=n_ept, ept_mean="probs")
     assert (r["status"] == 0).all()
     for k in ("next_parent", "next_cand", "next_state"):
         np.testing.assert_array_equal(r[k], r1[k], err_msg=k)
+        np.testing.assert_array_equal(rp[k], r1[k], err_msg=k)
 
 
+@pytest.mark.parametrize("ept_mean", ["logits", "probs"])
 @pytest.mark.parametrize("seed,n_ept", [(0, 2), (1, 3), (2, 2), (3, 5)])
-def test_ept_random_cases_match_independent_restatement(seed, n_ept):
+def test_ept_random_cases_match_independent_restatement(seed, n_ept, ept_mean):
     rng = np.random.default_rng(100 + seed)
     c = 1 + seed % 3
     w = W.scaled(W.WORKLOADS["tiny"], B=4, V=257, T=12 * (1 + n_ept * c), n_cand=12,
@@ -221,9 +281,10 @@ def test_ept_random_cases_match_independent_restatement(seed, n_ept):
     n_states, K = 4, 5
     tp, tr = W.make_tree_templates(n_states, 48, K, rng, n_ept=n_ept)
     r = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
-                         acc["next_token"], tp, tr, K, n_ept=n_ept)
+                         acc["next_token"], tp, tr, K, n_ept=n_ept, ept_mean=ept_mean)
     ref_p, ref_c, ref_s = _independent(logits, s.parent, s.cand_tokens, acc["path"],
-                                       acc["accept_len"], acc["next_token"], tp, tr, K, n_ept)
+                                       acc["accept_len"], acc["next_token"], tp, tr, K, n_ept,
+                                       ept_mean)
     assert (r["status"] == 0).all()
     np.testing.assert_array_equal(r["next_state"], ref_s)
     np.testing.assert_array_equal(r["next_parent"], ref_p)
