@@ -248,7 +248,13 @@ ppd_status ppd_verify_step_typical(const void *q, void *k_cache, void *v_cache,
  *   the K best tokens (ranking: NaN first, then larger value, then lower index)
  *   of the fp32 average of the chains' logits at position d: summed in chain
  *   order, then divided by n_ept with IEEE rounding.  n_ept = 1: one chain,
- *   plain logits.
+ *   plain logits.  ppd_next_tree_ept with ept_mean = 1 ranks instead the mean
+ *   of the chains' probabilities (the section's formula):
+ *   sum_j exp(x_j[v] - lse_j), lse_j = ln sum_v exp(x_j[v]), fp32, summed in
+ *   chain order (the 1/n_ept scale, which changes no ranking, left out); a
+ *   chain row holding a NaN or +inf, or only -inf, makes every score NaN.
+ *   Tokens whose mean probabilities differ by less than a few fp32 roundings
+ *   may rank either way.  ept_mean = 0 is ppd_next_tree.
  *   tmpl_parent, tmpl_rank int32 [n_states][T_next] (device): the next tree of
  *   each state; node 0 is the root (parent -1), rank r >= 0 marks a candidate
  *   taking guess r at its depth, -1 a prompt node.
@@ -259,7 +265,8 @@ ppd_status ppd_verify_step_typical(const void *q, void *k_cache, void *v_cache,
  * next_token[b] < 0, or template k is not a tree in topological order, has a
  * candidate below a prompt node, a candidate deeper than k or a rank >= K.
  * logits, parent, cand_tokens, path as for the verification step that just ran.
- * 1 <= K <= 16, K <= V; 1 <= n_ept <= 128; n_states <= 128; T_next <= 512.
+ * 1 <= K <= 16, K <= V; 1 <= n_ept <= 128; ept_mean 0 or 1; n_states <= 128;
+ * T_next <= 512.
  * Workspace:
  * ppd_next_tree_workspace_bytes(B, n_states, K) bytes.
  */
@@ -271,6 +278,13 @@ ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32
                          int32_t *next_cand, int32_t *next_state, int32_t *dev_status,
                          void *workspace, size_t ws_bytes,
                          void *stream);
+ppd_status ppd_next_tree_ept(const float *logits, const int32_t *parent,
+                             const int32_t *cand_tokens, const int32_t *path,
+                             const int32_t *accept_len, const int32_t *next_token, int B, int T,
+                             int V, int n_states, int T_next, const int32_t *tmpl_parent,
+                             const int32_t *tmpl_rank, int K, int n_ept, int ept_mean,
+                             int32_t *next_parent, int32_t *next_cand, int32_t *next_state,
+                             int32_t *dev_status, void *workspace, size_t ws_bytes, void *stream);
 
 /*
  * Node argmax without a workspace (no paper counterpart; an interface for

@@ -767,18 +767,19 @@ size_t ppd_next_tree_workspace_bytes(int B, int n_states, int K)
     return align_up(align_up((size_t)B * n_states * K * sizeof(int32_t)) + (size_t)B * sizeof(int32_t));
 }
 
-ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32_t *cand_tokens,
-                         const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
-                         int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
-                         const int32_t *tmpl_rank, int K, int n_ept, int32_t *next_parent,
-                         int32_t *next_cand, int32_t *next_state, int32_t *dev_status,
-                         void *workspace, size_t ws_bytes, void *stream)
+ppd_status ppd_next_tree_ept(const float *logits, const int32_t *parent,
+                             const int32_t *cand_tokens, const int32_t *path,
+                             const int32_t *accept_len, const int32_t *next_token, int B, int T,
+                             int V, int n_states, int T_next, const int32_t *tmpl_parent,
+                             const int32_t *tmpl_rank, int K, int n_ept, int ept_mean,
+                             int32_t *next_parent, int32_t *next_cand, int32_t *next_state,
+                             int32_t *dev_status, void *workspace, size_t ws_bytes, void *stream)
 {
     if (!logits || !parent || !cand_tokens || !path || !accept_len || !next_token || !tmpl_parent ||
         !tmpl_rank || !next_parent || !next_cand || !next_state || !dev_status || !workspace)
         return PPD_ERR_INVALID_ARG;
     if (B < 1 || T < 1 || T > kMaxT || V < 1 || n_states < 1 || n_states > 128 || T_next < 1 ||
-        T_next > kMaxT || K < 1 || K > V || n_ept < 1)
+        T_next > kMaxT || K < 1 || K > V || n_ept < 1 || ept_mean < 0 || ept_mean > 1)
         return PPD_ERR_INVALID_ARG;
     if (K > ppd::kNextMaxK || n_ept > ppd::kNextMaxEpt) return PPD_ERR_UNSUPPORTED;
     if ((double)B * T * V > 9.0e15) return PPD_ERR_INVALID_ARG;
@@ -789,8 +790,20 @@ ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32
                                                   align_up((size_t)B * n_states * K * sizeof(int32_t)));
     return cuda_status(ppd::launch_next_tree(
         logits, parent, cand_tokens, path, accept_len, next_token, B, T, V, n_states, T_next,
-        tmpl_parent, tmpl_rank, K, n_ept, topk, kstate, next_parent, next_cand, next_state,
-        dev_status, static_cast<cudaStream_t>(stream)));
+        tmpl_parent, tmpl_rank, K, n_ept, ept_mean, topk, kstate, next_parent, next_cand,
+        next_state, dev_status, static_cast<cudaStream_t>(stream)));
+}
+
+ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32_t *cand_tokens,
+                         const int32_t *path, const int32_t *accept_len, const int32_t *next_token,
+                         int B, int T, int V, int n_states, int T_next, const int32_t *tmpl_parent,
+                         const int32_t *tmpl_rank, int K, int n_ept, int32_t *next_parent,
+                         int32_t *next_cand, int32_t *next_state, int32_t *dev_status,
+                         void *workspace, size_t ws_bytes, void *stream)
+{
+    return ppd_next_tree_ept(logits, parent, cand_tokens, path, accept_len, next_token, B, T, V,
+                             n_states, T_next, tmpl_parent, tmpl_rank, K, n_ept, 0, next_parent,
+                             next_cand, next_state, dev_status, workspace, ws_bytes, stream);
 }
 
 ppd_status ppd_selftest_umma(const void *a, const void *b, float *d, int mode, int N, void *stream)

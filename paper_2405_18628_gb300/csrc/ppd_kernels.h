@@ -213,9 +213,9 @@ cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const i
                              const int32_t *path, const int32_t *accept_len,
                              const int32_t *next_token, int B, int T, int V, int n_states,
                              int T_next, const int32_t *tmpl_parent, const int32_t *tmpl_rank, int K,
-                             int n_ept, int32_t *topk, int32_t *kstate, int32_t *next_parent,
-                             int32_t *next_cand, int32_t *next_state, int32_t *status,
-                             cudaStream_t stream);
+                             int n_ept, int ept_mean, int32_t *topk, int32_t *kstate,
+                             int32_t *next_parent, int32_t *next_cand, int32_t *next_state,
+                             int32_t *status, cudaStream_t stream);
 
 cudaError_t launch_round_bf16(const float *src, uint16_t *dst, int64_t n, cudaStream_t stream);
 

@@ -2,7 +2,8 @@
 // Section 3 step (1): the prompt tokens appended to a guess token predict the
 // tokens that follow it; Section 3, Ensemble Prompt Tokens: each prompt
 // position holds n_ept tokens, the j-th seeing only the j-th of the positions
-// before it, and the guess comes from the average of their logits; Appendix,
+// before it, and the guess comes from the average of their logits -- or, in
+// the formula the section gives, of their probabilities; Appendix,
 // Definition of tree states: the next tree takes state T_k, whose candidate
 // subtree is at most k deep, k being the number of prompt positions left
 // below the accepted token).
@@ -10,9 +11,12 @@
 // Kernel 1, one block per (sequence, chain position d): finds the n_ept
 // prompt chains below the accepted end node (warp ballots over the parent
 // array, one warp per chain) and, if d is within the state, the K best tokens
-// of the chains' averaged logits at position d -- every thread keeps its own
-// top-K over a strided slice of the row, then K rounds of a block-wide
-// best-of-heads merge.  Kernel 2, one warp per sequence: fills the state's
+// of the chains' averaged logits (or probabilities) at position d -- every
+// thread keeps its own top-K over a strided slice of the row, then K rounds of
+// a block-wide best-of-heads merge.  The probability mode first takes each
+// chain row's log-sum-exp (one warp a row, an online maximum and sum), then
+// ranks sum_j exp(x_j - lse_j): the mean without its 1/n_ept, which no
+// ranking sees.  Kernel 2, one warp per sequence: fills the state's
 // template with the root token and the guesses.
 #include "ppd.h"
 #include "ppd_accept.cuh"
@@ -36,16 +40,53 @@ PPD_DEV int next_prompt_child(const int32_t *par, const int32_t *tok, int T, int
     return -1;
 }
 
-// Top-K (K <= kNextMaxK) of the averaged logits at chain position d (1-based)
-// of sequence b, written to topk[(b * (n_states - 1) + d - 1) * K ...] in
-// ranking order (NaN first, then larger value, then lower index).  The blocks
-// of position 1 also write the state k of their sequence to kstate[b].
+// ln sum_v exp(x[v]) of one row, by one warp: NaN if the row holds a NaN or
+// +inf, or if every entry is -inf (each probability of such a row is NaN).
+// -inf entries add nothing; every exponent is a difference <= 0, so nothing
+// overflows.
+PPD_DEV float row_lse_warp(const float *x, int V, int lane)
+{
+    constexpr float kLog2e = 1.4426950408889634f;
+    float m = -INFINITY, s = 0.f;
+    bool bad = false;
+    for (int v = lane; v < V; v += 32) {
+        const float xv = __ldg(x + v);
+        if (isnan(xv) || xv == INFINITY) {
+            bad = true;
+        } else if (xv > m) {
+            s = s * exp2f((m - xv) * kLog2e) + 1.f;
+            m = xv;
+        } else if (xv > -INFINITY) {
+            s += exp2f((xv - m) * kLog2e);
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float om = __shfl_xor_sync(0xffffffffu, m, off);
+        const float os = __shfl_xor_sync(0xffffffffu, s, off);
+        const float nm = fmaxf(m, om);
+        if (nm > -INFINITY)
+            s = (m > -INFINITY ? s * exp2f((m - nm) * kLog2e) : 0.f) +
+                (om > -INFINITY ? os * exp2f((om - nm) * kLog2e) : 0.f);
+        m = nm;
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    return (bad || m == -INFINITY) ? NAN : m + logf(s);
+}
+
+// Top-K (K <= kNextMaxK) of the averaged logits (ept_mean 0) or probabilities
+// (ept_mean 1) at chain position d (1-based) of sequence b, written to
+// topk[(b * (n_states - 1) + d - 1) * K ...] in ranking order (NaN first, then
+// larger value, then lower index).  The blocks of position 1 also write the
+// state k of their sequence to kstate[b].
 __global__ void __launch_bounds__(256)
 next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const int32_t *cand,
                  const int32_t *path, const int32_t *accept_len, int T, int V, int n_states, int K,
-                 int n_ept, int32_t *topk, int32_t *kstate)
+                 int n_ept, int ept_mean, int32_t *topk, int32_t *kstate)
 {
+    constexpr float kLog2e = 1.4426950408889634f;
     __shared__ int s_head[kNextMaxEpt];
+    __shared__ float s_lse[kNextMaxEpt];
     __shared__ int s_len[kNextMaxEpt];
     __shared__ int s_node[kNextMaxEpt];
     __shared__ int s_nh, s_k;
@@ -107,6 +148,14 @@ next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const 
     if (d > s_k) return;   // uniform over the block
     const float *x0 = logits + ((size_t)b * T + s_node[0]) * V;
     const float n_f = (float)n_ept;
+    const bool probs = ept_mean == 1 && n_ept > 1;
+    if (probs) {
+        for (int j = warp; j < n_ept; j += 8) {
+            const float l = row_lse_warp(logits + ((size_t)b * T + s_node[j]) * V, V, lane);
+            if (lane == 0) s_lse[j] = l;
+        }
+        __syncthreads();
+    }
 
     // this thread's best K over its slice, best first
     float hv[kNextMaxK];
@@ -119,11 +168,19 @@ next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const 
     float tv = -INFINITY;   // the K-th best so far (the entry a new token must beat)
     int ti = INT_MAX;
     for (int v = threadIdx.x; v < V; v += 256) {
-        float xv = __ldcs(x0 + v);
-        if (n_ept > 1) {
+        float xv;
+        if (probs) {
+            // sum_j p_j(v), chain order; a NaN lse_j makes every score NaN
+            xv = 0.f;
+            for (int j = 0; j < n_ept; ++j)
+                xv += exp2f((__ldcs(logits + ((size_t)b * T + s_node[j]) * V + v) - s_lse[j]) * kLog2e);
+        } else if (n_ept > 1) {
+            xv = __ldcs(x0 + v);
             // the EPT average: summed in chain order, then one IEEE division
             for (int j = 1; j < n_ept; ++j) xv += __ldcs(logits + ((size_t)b * T + s_node[j]) * V + v);
             xv = xv / n_f;
+        } else {
+            xv = __ldcs(x0 + v);
         }
         if (!ranks_before(xv, v, tv, ti)) continue;
         // insert, shifting worse entries down (slots K.. stay unused)
@@ -273,13 +330,14 @@ cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const i
                              const int32_t *path, const int32_t *accept_len,
                              const int32_t *next_token, int B, int T, int V, int n_states,
                              int T_next, const int32_t *tmpl_parent, const int32_t *tmpl_rank, int K,
-                             int n_ept, int32_t *topk, int32_t *kstate, int32_t *next_parent,
-                             int32_t *next_cand, int32_t *next_state, int32_t *status,
-                             cudaStream_t stream)
+                             int n_ept, int ept_mean, int32_t *topk, int32_t *kstate,
+                             int32_t *next_parent, int32_t *next_cand, int32_t *next_state,
+                             int32_t *status, cudaStream_t stream)
 {
     if (n_states > 1) {
         next_topk_kernel<<<dim3((unsigned)B, (unsigned)(n_states - 1)), 256, 0, stream>>>(
-            logits, parent, cand, path, accept_len, T, V, n_states, K, n_ept, topk, kstate);
+            logits, parent, cand, path, accept_len, T, V, n_states, K, n_ept, ept_mean, topk,
+            kstate);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }

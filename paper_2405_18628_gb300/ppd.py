@@ -62,6 +62,8 @@ def load() -> ctypes.CDLL:
             "ppd_node_stats": ([vp, i32, i32, i32, f32, vp, vp, vp, vp, sz, vp], i32),
             "ppd_typical_accept": ([vp] * 7 + [i32] * 4 + [f32] * 3 + [vp] * 5 + [vp], i32),
             "ppd_next_tree_workspace_bytes": ([i32, i32, i32], sz),
+            "ppd_next_tree_ept": ([vp] * 6 + [i32] * 5 + [vp, vp, i32, i32, i32] + [vp] * 4 +
+                                  [vp, sz, vp], i32),
             "ppd_next_tree": ([vp] * 6 + [i32] * 5 + [vp, vp, i32, i32] + [vp] * 4 + [vp, sz, vp],
                               i32),
             "ppd_verify_step_typical": ([vp] * 9 + [i32] * 8 + [f32] * 4 + [vp] * 8 +
@@ -248,23 +250,26 @@ def ppd_verify_step_typical(q, k_cache, v_cache, k_tree, v_tree, prefix_len, par
 
 def ppd_next_tree(logits, parent, cand_tokens, path, accept_len, next_token, tmpl_parent,
                   tmpl_rank, K: int, next_parent, next_cand, next_state, dev_status,
-                  workspace=None, stream=None, n_ept: int = 1):
+                  workspace=None, stream=None, n_ept: int = 1, ept_mean: str = "logits"):
     """Next-step candidate tree.  logits [B,T,V]; parent, cand_tokens, path
     [B,T]; accept_len, next_token [B]; tmpl_parent, tmpl_rank [n_states,
-    T_next] (device int32); n_ept ensemble prompt tokens per prompt position;
+    T_next] (device int32); n_ept ensemble prompt tokens per prompt position,
+    whose logits (ept_mean="logits") or probabilities ("probs") are averaged;
     outputs next_parent, next_cand [B,T_next], next_state, dev_status [B].  A
     workspace is allocated if none is given."""
+    if ept_mean not in ("logits", "probs"):
+        raise ValueError(f"ept_mean must be 'logits' or 'probs', not {ept_mean!r}")
     B, T, V = logits.shape
     n_states, T_next = tmpl_parent.shape
     need = int(load().ppd_next_tree_workspace_bytes(B, n_states, int(K)))
     if workspace is None:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=logits.device)
-    st = load().ppd_next_tree(_ptr(logits), _ptr(parent), _ptr(cand_tokens), _ptr(path),
-                              _ptr(accept_len), _ptr(next_token), B, T, V, n_states, T_next,
-                              _ptr(tmpl_parent), _ptr(tmpl_rank), int(K), int(n_ept),
-                              _ptr(next_parent),
-                              _ptr(next_cand), _ptr(next_state), _ptr(dev_status), _ptr(workspace),
-                              workspace.numel(), _stream(stream))
+    st = load().ppd_next_tree_ept(_ptr(logits), _ptr(parent), _ptr(cand_tokens), _ptr(path),
+                                  _ptr(accept_len), _ptr(next_token), B, T, V, n_states, T_next,
+                                  _ptr(tmpl_parent), _ptr(tmpl_rank), int(K), int(n_ept),
+                                  int(ept_mean == "probs"), _ptr(next_parent), _ptr(next_cand),
+                                  _ptr(next_state), _ptr(dev_status), _ptr(workspace),
+                                  workspace.numel(), _stream(stream))
     _check(st, "ppd_next_tree")
 
 

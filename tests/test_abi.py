@@ -190,3 +190,12 @@ def test_next_tree_host_checks(lib):
     need = lib.ppd_next_tree_workspace_bytes(2, 4, 4)
     assert need >= 2 * 4 * 4 * 4 + 2 * 4
     assert call(ws_bytes=need - 1) == ppd.PPD_ERR_INVALID_ARG
+
+    def call_ept(ept_mean, n_ept=2, K=4):
+        return lib.ppd_next_tree_ept(*[fake] * 6, 2, 16, 100, 4, 32, fake, fake, K, n_ept,
+                                     ept_mean, *[fake] * 4, fake, ws, s)
+
+    assert call_ept(2) == ppd.PPD_ERR_INVALID_ARG
+    assert call_ept(-1) == ppd.PPD_ERR_INVALID_ARG
+    assert call_ept(1, n_ept=129) == ppd.PPD_ERR_UNSUPPORTED
+    assert call_ept(1, K=17) == ppd.PPD_ERR_UNSUPPORTED
