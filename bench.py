@@ -612,20 +612,24 @@ def e2e_groups(L):
 
 def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, n_cmp=2):
     """The step end to end from pinned host buffers through the public C ABI,
-    with the copies overlapping the compute.  The layers go in `groups` groups;
-    each group's Q / tree K / tree V are copied in on a copy stream, and its
-    attention (ppd_tree_attention) starts as soon as they have landed, on one
-    of two compute streams in turn (so one group's last, partial round of
-    slices overlaps the next group's first), while the next group's copy
-    runs; each group's output is copied back on a third stream as soon as it
-    is done.  The logits and index arrays are copied in last: node argmax
-    (ppd_node_argmax), acceptance (ppd_accept_path) and the compaction of
-    every layer's accepted rows (ppd_kv_compact) need no attention output, so
-    they run while the last groups' outputs are copied back, and the index
-    outputs follow.  A step ends with every result in host memory (stream
-    synchronised).  Returns the timing, the copied bytes and, with
-    `check_against` (the device step's outputs), the largest difference
-    found."""
+    with the copies overlapping the compute.  The layers go in `groups` groups.
+    Each group's Q, tree K and tree V sit together in one pinned host buffer
+    and one device buffer (the tree's index arrays -- parents, candidate
+    tokens, prefix lengths -- ride in front of the first group's), so a group
+    is one copy in.  A group's attention (ppd_tree_attention) starts as soon
+    as its copy has landed, on one of `n_cmp` compute streams in turn (so one
+    group's last, partial round of slices overlaps the next group's first),
+    while the next group's copy runs; its output is copied back on another
+    stream as soon as it is done.  The logits come in last: node argmax
+    (ppd_node_argmax) and acceptance (ppd_accept_path) need no attention
+    output, so they run on a stream of their own once the logits have landed,
+    then the compaction of each group's accepted rows (ppd_kv_compact; it
+    writes cache rows at and past each prefix length, which no attention call
+    of the step reads), and the index outputs go back after the last group's
+    output.  A step ends with every
+    result in host memory (stream synchronised).  Returns the timing, the
+    copied bytes and, with `check_against` (the device step's outputs), the
+    largest difference found."""
     import torch
 
     from paper_2405_18628_gb300 import ppd
@@ -638,17 +642,28 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, n_cmp=2):
             bounds.append(bounds[-1] + n)
         assert bounds[-1] == L
         groups = len(groups)
-    pin = lambda x: x.cpu().pin_memory()
-    h = {k: pin(t[k]) for k in ("q", "k_tree", "v_tree")}
-    h_small, hs = packed({"logits": ((w.B, w.T, w.V), torch.float32),
-                          "parent": ((w.B, w.T), torch.int32), "cand": ((w.B, w.T), torch.int32),
-                          "prefix": ((w.B,), torch.int32)}, "cpu")
-    hs["logits"].copy_(st.logits.cpu())
-    hs["parent"].copy_(st.parent.cpu())
-    hs["cand"].copy_(st.cand.cpu())
-    hs["prefix"].copy_(st.prefix.cpu())
-    d = {k: torch.empty_like(t[k]) for k in ("q", "k_tree", "v_tree")}
-    d_small, ds = packed({k: (v.shape, v.dtype) for k, v in hs.items()}, dev)
+    tree_specs = {"parent": ((w.B, w.T), torch.int32), "cand": ((w.B, w.T), torch.int32),
+                  "prefix": ((w.B,), torch.int32)}
+    h_in, d_in, dv = [], [], []             # per group: host buffer, device buffer, views
+    for g in range(groups):
+        a, b = bounds[g], bounds[g + 1]
+        specs = dict(tree_specs) if g == 0 else {}
+        specs.update({k: ((b - a,) + tuple(t[k].shape[1:]), t[k].dtype)
+                      for k in ("q", "k_tree", "v_tree")})
+        hb, hvw = packed(specs, "cpu")
+        db, dvw = packed(specs, dev)
+        for k in ("q", "k_tree", "v_tree"):
+            hvw[k].copy_(t[k][a:b])
+        if g == 0:
+            tree_h, tree_d = hvw, dvw
+        h_in.append(hb)
+        d_in.append(db)
+        dv.append(dvw)
+    tree_h["parent"].copy_(st.parent.cpu())
+    tree_h["cand"].copy_(st.cand.cpu())
+    tree_h["prefix"].copy_(st.prefix.cpu())
+    h_logits = st.logits.cpu().pin_memory()
+    d_logits = torch.empty_like(h_logits, device=dev)
     out = torch.empty(L, w.B, w.H, w.T, w.D, dtype=torch.float32, device=dev)
     h_out = torch.empty(out.shape, dtype=torch.float32, pin_memory=True)
     names = ["argmax", "accept_len", "path", "next_token", "new_prefix_len", "dev_status"]
@@ -658,52 +673,49 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, n_cmp=2):
     h_idx, hi = packed({k: (shapes[k], torch.int32) for k in names}, "cpu")
     st_grp = torch.zeros(groups, w.B, dtype=torch.int32, device=dev)
     # one workspace per compute stream (a call's work split keeps its partial
-    # states there until its merge grid has run)
-    ws = [st.bufs.workspace] + [torch.zeros_like(st.bufs.workspace) for _ in range(n_cmp - 1)]
+    # states there until its merge grid has run), one for the argmax
+    ws = [st.bufs.workspace] + [torch.zeros_like(st.bufs.workspace) for _ in range(n_cmp)]
     s_in = torch.cuda.Stream()
     s_cmp = [torch.cuda.Stream() for _ in range(n_cmp)]
     s_out = torch.cuda.Stream()
+    s_idx = torch.cuda.Stream()
     kc, vc = t["k_cache"], t["v_cache"]
 
     def one_step():
         ev_in = [torch.cuda.Event() for _ in range(groups)]
-        ev_small = torch.cuda.Event()
+        ev_logits = torch.cuda.Event()
         ev_done = [torch.cuda.Event() for _ in range(groups)]
         ev_idx = torch.cuda.Event()
         with torch.cuda.stream(s_in):
             for g in range(groups):
-                a, b = bounds[g], bounds[g + 1]
-                for k in ("q", "k_tree", "v_tree"):
-                    d[k][a:b].copy_(h[k][a:b], non_blocking=True)
+                d_in[g].copy_(h_in[g], non_blocking=True)
                 ev_in[g].record(s_in)
-            d_small.copy_(h_small, non_blocking=True)
-            ev_small.record(s_in)
+            d_logits.copy_(h_logits, non_blocking=True)
+            ev_logits.record(s_in)
+
+        # argmax and acceptance once the logits are in, then the compaction
+        with torch.cuda.stream(s_idx):
+            s_idx.wait_event(ev_logits)
+            ppd.ppd_node_argmax(d_logits, di["argmax"], workspace=ws[n_cmp], stream=s_idx)
+            ppd.ppd_accept_path(di["argmax"], tree_d["cand"], tree_d["parent"], tree_d["prefix"],
+                                w.V, w.S_max, di["accept_len"], di["path"], di["next_token"],
+                                di["new_prefix_len"], di["dev_status"], stream=s_idx)
+            ev_idx.record(s_idx)
+            for g in range(groups):
+                a, b = bounds[g], bounds[g + 1]
+                ppd.ppd_kv_compact(kc[a:b], vc[a:b], dv[g]["k_tree"], dv[g]["v_tree"], di["path"],
+                                   di["accept_len"], tree_d["prefix"], stream=s_idx)
         for g in range(groups):
             a, b = bounds[g], bounds[g + 1]
             sc = s_cmp[g % n_cmp]
             sc.wait_event(ev_in[g])
-            sl = lambda x: x[a:b]
-            ppd.ppd_tree_attention(sl(d["q"]), sl(kc), sl(vc), sl(d["k_tree"]), sl(d["v_tree"]),
-                                   ds["prefix"], ds["parent"], sl(out), st_grp[g], workspace=ws[g % n_cmp],
-                                   stream=sc)
+            ppd.ppd_tree_attention(dv[g]["q"], kc[a:b], vc[a:b], dv[g]["k_tree"], dv[g]["v_tree"],
+                                   tree_d["prefix"], tree_d["parent"], out[a:b], st_grp[g],
+                                   workspace=ws[g % n_cmp], stream=sc)
             ev_done[g].record(sc)
             s_out.wait_event(ev_done[g])
             with torch.cuda.stream(s_out):
                 h_out[a:b].copy_(out[a:b], non_blocking=True)
-        # argmax, acceptance and compaction once the logits are in and both
-        # compute streams are done with the attention
-        sc = s_cmp[groups % n_cmp]
-        sc.wait_event(ev_small)
-        for other in s_cmp:
-            if other is not sc:
-                sc.wait_stream(other)
-        ppd.ppd_node_argmax(ds["logits"], di["argmax"], workspace=ws[groups % n_cmp], stream=sc)
-        ppd.ppd_accept_path(di["argmax"], ds["cand"], ds["parent"], ds["prefix"], w.V, w.S_max,
-                            di["accept_len"], di["path"], di["next_token"], di["new_prefix_len"],
-                            di["dev_status"], stream=sc)
-        ev_idx.record(sc)
-        ppd.ppd_kv_compact(kc, vc, d["k_tree"], d["v_tree"], di["path"], di["accept_len"],
-                           ds["prefix"], stream=sc)
         s_out.wait_event(ev_idx)
         with torch.cuda.stream(s_out):
             h_idx.copy_(d_idx, non_blocking=True)
@@ -718,10 +730,10 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, n_cmp=2):
     cap = torch.cuda.Stream()
     cap.wait_stream(torch.cuda.current_stream())
     with torch.cuda.graph(graph, stream=cap):
-        for x in (s_in, *s_cmp, s_out):
+        for x in (s_in, *s_cmp, s_out, s_idx):
             x.wait_stream(cap)
         one_step()
-        for x in (s_in, *s_cmp, s_out):
+        for x in (s_in, *s_cmp, s_out, s_idx):
             cap.wait_stream(x)
     torch.cuda.synchronize()
     for _ in range(3):
@@ -734,8 +746,7 @@ def e2e_pipelined(w, t, st, K, groups, dev, check_against=None, n_cmp=2):
         graph.replay()                            # on the current stream
         torch.cuda.current_stream().synchronize()
         ms.append((time.perf_counter() - t0) * 1e3)
-    res = {"ms": ms, "h2d_bytes": int(sum(v.numel() * v.element_size() for v in h.values())
-                                      + h_small.numel()),
+    res = {"ms": ms, "h2d_bytes": int(sum(x.numel() for x in h_in) + h_logits.numel() * 4),
            "d2h_bytes": int(h_out.numel() * 4 + h_idx.numel()), "groups": groups}
     if check_against is not None:
         ref_out, ref_idx = check_against
@@ -973,14 +984,15 @@ def main(argv=None):
                          "matches_device_step": ok, "max_abs_diff_out": pip["max_abs_diff_out"],
                          "note": "KV cache resident on the device; the layers in groups of "
                                  + "/".join(str(n) for n in e2e_groups(w.L)) + ", each "
-                                 "group's tree tensors copied in on one stream and its attention "
-                                 "(ppd_tree_attention) run as soon as they have landed, on two "
-                                 "compute streams in turn, its output copied back on a third as "
-                                 "soon as it is done; the logits and index arrays copied in last, "
-                                 "then ppd_node_argmax, ppd_accept_path and ppd_kv_compact (all "
-                                 "layers) and the index outputs copied back; the copies and calls "
-                                 "of a step captured once in a CUDA graph and replayed once per "
-                                 "step"}
+                                 "group's Q and tree K/V in one pinned buffer (the tree's index "
+                                 "arrays in front of the first), copied in as one copy on one "
+                                 "stream, its attention (ppd_tree_attention) run as soon as it "
+                                 "has landed, on two compute streams in turn, its output copied "
+                                 "back on a third as soon as it is done; the logits copied in "
+                                 "last, then ppd_node_argmax, ppd_accept_path and ppd_kv_compact "
+                                 "on a fourth stream and the index outputs copied back; the "
+                                 "copies and calls of a step captured once in a CUDA graph and "
+                                 "replayed once per step"}
             if ok:
                 e2e = dict(pipelined)
                 e2e["serial"] = serial
