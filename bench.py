@@ -71,12 +71,12 @@ REFERENCE_BUDGET_S = 180.0
 # are not in the count, so this is the reads plus the part of the writes that
 # reached DRAM during the launch.
 MEASURED_TRAFFIC = {
-    # 676,180,992 B at 19 layers (reads 667,975,936), x 32/19
-    "vicuna7b": {"bytes_per_launch": 1_138_831_144, "src": "028eaf175014bde9"},
-    # 1,658,903,808 B at 19 layers (reads 1,650,978,560), x 40/19
-    "vicuna13b": {"bytes_per_launch": 3_492_429_069, "src": "028eaf175014bde9"},
-    # 123,361,024 B, a fused-step launch at the full 24 layers (reads 119,708,928)
-    "mobilellama": {"bytes_per_launch": 123_361_024, "src": "028eaf175014bde9"},
+    # 676,500,480 B at 19 layers (reads 667,940,352), x 32/19
+    "vicuna7b": {"bytes_per_launch": 1_139_369_229, "src": "7004aad6620e17ff"},
+    # 1,659,106,304 B at 19 layers (reads 1,650,952,704), x 40/19
+    "vicuna13b": {"bytes_per_launch": 3_492_855_376, "src": "7004aad6620e17ff"},
+    # 123,587,072 B, a fused-step launch at the full 24 layers (reads 119,713,792)
+    "mobilellama": {"bytes_per_launch": 123_587_072, "src": "7004aad6620e17ff"},
 }
 
 
