@@ -255,3 +255,33 @@ def test_next_tree_probability_mean(cuda_device, n_ept, c, T_next, K):
             assert n_diff <= 2
         else:
             _compare(got, ref)
+
+
+@pytest.mark.parametrize("ept_mean", ["logits", "probs"])
+def test_next_tree_128_ensemble_chains(cuda_device, ept_mean):
+    """The largest ensemble the API takes: 128 prompt chains of two tokens
+    under the accepted candidate (nodes 2..129 the heads, 130..257 their
+    children), K = 16 guesses per depth; every chain's block of warps runs."""
+    n_ept, T, V, K = 128, 258, 1000, 16
+    parent = np.zeros((1, T), np.int32)
+    parent[0, 0] = -1
+    parent[0, 1] = 0
+    parent[0, 2:130] = 1
+    parent[0, 130:258] = np.arange(2, 130)
+    cand = np.full((1, T), -1, np.int32)
+    cand[0, :2] = [5, 6]
+    path = np.full((1, T), -1, np.int32)
+    path[0, :2] = [0, 1]
+    rng = np.random.default_rng(128)
+    logits = (2.0 * rng.standard_normal((1, T, V))).astype(np.float32)
+    alen, nt = np.array([2], np.int32), np.array([9], np.int32)
+    tp, tr = W.make_tree_templates(3, 40, K, rng)
+    ref = oracle.next_tree(logits, parent, cand, path, alen, nt, tp, tr, K, n_ept=n_ept,
+                           ept_mean=ept_mean)
+    assert ref["status"].tolist() == [0] and ref["next_state"].tolist() == [2]
+    got = _run(cuda_device, logits, parent, cand, path, alen, nt, tp, tr, K, n_ept=n_ept,
+               ept_mean=ept_mean)
+    if ept_mean == "logits":
+        _compare(got, ref)
+    else:
+        assert _compare_probs(got, ref, logits, parent, cand, path, alen, tp, tr, n_ept) <= 2
