@@ -18,9 +18,12 @@ and the batch-8 / prefix-16384 tree-size sweep) under "workloads", the
 attention as a model calls it (one call per layer) under
 "per_layer_attention", and the step latency against the tree size (the
 hardware half of the paper's hardware-aware tree size) under
-"tree_size_profile".  GPU clocks are sampled from before the first warm-up
-step to after the last timed loop; "clocks" summarises the samples taken
-inside timed loops.
+"tree_size_profile", and the steps after the verification path: the step
+with typical acceptance under "typical_step" and next-step candidate
+generation under "next_tree" (on the headline trees, and on trees of four
+ensemble chains with the chains' logits or probabilities averaged).  GPU
+clocks are sampled from before the first warm-up step to after the last
+timed loop; "clocks" summarises the samples taken inside timed loops.
 
 Under torchrun (N > 1) each rank runs an independent replica of the headline
 workload on its own GPU (weak scaling: the sequences of different ranks are
@@ -509,6 +512,67 @@ def time_loop(fn, K, warmup, stream, flush, windows):
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
     return [a.elapsed_time(b) for a, b in ev], wall
+
+
+def next_tree_ept(w, dev, stream, K, n_ept=4, chain=3, B=4):
+    """Next-step candidate generation on trees whose every candidate carries
+    n_ept ensemble chains of `chain` prompt tokens (the headline workload's
+    vocabulary), with the chains' logits and then their probabilities
+    averaged.  Acceptance comes from the library's argmax and acceptance
+    calls.  Times each mode with CUDA events (median of K calls).  Algorithmic
+    bytes: for every sequence, state k times n_ept logits rows of V fp32 (the
+    rows ranked; the probability mode reads them a second time, from L2)."""
+    import torch
+
+    from paper_2405_18628_gb300 import ppd
+    from paper_2405_18628_gb300 import workloads as W
+    we = W.scaled(w, B=B, T=16 * (1 + n_ept * chain), n_cand=16, chains=f"ept{n_ept}x{chain}")
+    s = W.make_step_inputs(we, seed=we.seed)
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
+    logits = torch.from_numpy(s.logits).to(dev)
+    parent, cand, prefix = i32(s.parent), i32(s.cand_tokens), i32(s.prefix_len)
+    o = {k: torch.empty(shape, dtype=torch.int32, device=dev) for k, shape in
+         (("argmax", (we.B, we.T)), ("accept_len", (we.B,)), ("path", (we.B, we.T)),
+          ("next_token", (we.B,)), ("new_prefix_len", (we.B,)), ("status", (we.B,)))}
+    ws = ppd.workspace(1, we.B, 1, we.T, we.D, we.V, we.S_max, device=dev)
+    ppd.ppd_node_argmax(logits, o["argmax"], workspace=ws, stream=stream)
+    ppd.ppd_accept_path(o["argmax"], cand, parent, prefix, we.V, we.S_max, o["accept_len"],
+                        o["path"], o["next_token"], o["new_prefix_len"], o["status"],
+                        stream=stream)
+    n_states, K_guess, T_next = chain + 1, 8, 64
+    tp, trk = W.make_tree_templates(n_states, T_next, K_guess, np.random.default_rng(we.seed),
+                                    n_ept=n_ept)
+    tp_d, tr_d = i32(tp), i32(trk)
+    nx = {k: torch.empty(shape, dtype=torch.int32, device=dev) for k, shape in
+          (("parent", (we.B, T_next)), ("cand", (we.B, T_next)), ("state", (we.B,)),
+           ("status", (we.B,)))}
+    ws_nt = torch.empty(max(256, ppd.load().ppd_next_tree_workspace_bytes(we.B, n_states, K_guess)),
+                        dtype=torch.uint8, device=dev)
+    res = {"batch": we.B, "tree_tokens": we.T, "n_ept": n_ept, "chain_tokens": chain,
+           "states": n_states, "guesses_per_depth": K_guess}
+    for mode in ("logits", "probs"):
+        call = lambda: ppd.ppd_next_tree(logits, parent, cand, o["path"], o["accept_len"],
+                                         o["next_token"], tp_d, tr_d, K_guess, nx["parent"],
+                                         nx["cand"], nx["state"], nx["status"], workspace=ws_nt,
+                                         stream=stream, n_ept=n_ept, ept_mean=mode)
+        for _ in range(3):
+            call()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
+        head_start(stream)
+        for a, b in ev:
+            a.record(stream)
+            call()
+            b.record(stream)
+        torch.cuda.synchronize()
+        if (o["status"].cpu().numpy() != 0).any() or (nx["status"].cpu().numpy() != 0).any():
+            raise SystemExit("ensemble next-tree generation reported an error")
+        us = statistics.median(a.elapsed_time(b) for a, b in ev) * 1e3
+        states = nx["state"].cpu().numpy()
+        nbytes = int(states.sum()) * n_ept * we.V * 4
+        res[mode] = {"us": us, "state_histogram": np.bincount(states, minlength=n_states).tolist(),
+                     "bytes": nbytes, "gbs": nbytes / (us * 1e-6) / 1e9}
+    return res
 
 
 def per_layer_attention(w, t, prefix, parent, out, dev, reps, windows):
@@ -1002,7 +1066,7 @@ def main(argv=None):
 
     # ---------------------------------------------------------------- next-step candidates
     next_tree = None
-    if args.next_tree:
+    if args.next_tree or extras:
         from paper_2405_18628_gb300 import workloads as W
         i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
         n_states, K_guess = 5, 8
@@ -1032,9 +1096,28 @@ def main(argv=None):
         if (nxt["status"].cpu().numpy() != 0).any():
             raise SystemExit("next-step candidate generation reported an error")
         nt_ms = statistics.median(a.elapsed_time(b) for a, b in ev4)
+        nt_states = nxt["state"].cpu().numpy()
+        nt_bytes = int(nt_states.sum()) * w.V * 4
         next_tree = {"us": nt_ms * 1e3, "states": n_states, "guesses_per_depth": K_guess,
-                     "state_histogram": np.bincount(nxt["state"].cpu().numpy(),
-                                                    minlength=n_states).tolist()}
+                     "state_histogram": np.bincount(nt_states, minlength=n_states).tolist(),
+                     "bytes": nt_bytes, "gbs": nt_bytes / (nt_ms * 1e-3) / 1e9}
+        if extras:
+            next_tree["ensemble"] = next_tree_ept(w, dev, stream, K4)
+
+    # ---------------------------------------------------------------- typical acceptance
+    typical = None
+    if extras and args.accept == "exact":
+        st_t = Step(w, dev, w.seed, "typical")
+        ms_t, _ = time_loop(lambda: st_t(stream), min(K, 300), args.warmup, stream,
+                            flush if do_flush else None, windows)
+        n_acc_t = st_t.check()
+        typical = summarize(w, ms_t, n_acc_t, peak,
+                            ppd.ppd_verify_step_launches(w.L, w.B, w.H, w.T, w.D, w.V, w.S_max,
+                                                         typical=True))
+        typical["temperature_epsilon_delta"] = list(TYPICAL)
+        typical["accepted_tokens"] = n_acc_t
+        del st_t
+        torch.cuda.empty_cache()
 
     # ---------------------------------------------------------------- per-layer attention
     per_layer = None
@@ -1131,6 +1214,8 @@ def main(argv=None):
             line["tree_size_profile"] = profile
         if next_tree is not None:
             line["next_tree"] = next_tree
+        if typical is not None:
+            line["typical_step"] = typical
         print(json.dumps(line), flush=True)
     if pg:
         pg.barrier()

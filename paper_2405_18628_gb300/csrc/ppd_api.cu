@@ -761,10 +761,20 @@ ppd_status ppd_typical_accept(const float *logits, const float *lse, const float
                                                   epsilon, delta, static_cast<cudaStream_t>(stream)));
 }
 
+// topk [B][n_states][K] int32, kstate [B] int32, then the partial lists
+// (values fp32, indices int32) [B][n_states][kNextMaxSplit][K] each, then the
+// chain rows' log-sum-exps fp32 [B][n_states][kNextMaxEpt].
+static size_t next_part_bytes(int B, int n_states, int K)
+{
+    return align_up((size_t)B * n_states * ppd::kNextMaxSplit * K * sizeof(int32_t));
+}
+
 size_t ppd_next_tree_workspace_bytes(int B, int n_states, int K)
 {
     if (B < 1 || n_states < 1 || K < 1) return 0;
-    return align_up(align_up((size_t)B * n_states * K * sizeof(int32_t)) + (size_t)B * sizeof(int32_t));
+    return align_up(align_up((size_t)B * n_states * K * sizeof(int32_t)) + (size_t)B * sizeof(int32_t)) +
+           2 * next_part_bytes(B, n_states, K) +
+           align_up((size_t)B * n_states * ppd::kNextMaxEpt * sizeof(float));
 }
 
 ppd_status ppd_next_tree_ept(const float *logits, const int32_t *parent,
@@ -788,10 +798,15 @@ ppd_status ppd_next_tree_ept(const float *logits, const int32_t *parent,
     int32_t *topk = static_cast<int32_t *>(workspace);
     int32_t *kstate = reinterpret_cast<int32_t *>(static_cast<char *>(workspace) +
                                                   align_up((size_t)B * n_states * K * sizeof(int32_t)));
+    char *parts = static_cast<char *>(workspace) +
+                  align_up(align_up((size_t)B * n_states * K * sizeof(int32_t)) + (size_t)B * sizeof(int32_t));
+    float *part_val = reinterpret_cast<float *>(parts);
+    int32_t *part_idx = reinterpret_cast<int32_t *>(parts + next_part_bytes(B, n_states, K));
+    float *lse = reinterpret_cast<float *>(parts + 2 * next_part_bytes(B, n_states, K));
     return cuda_status(ppd::launch_next_tree(
         logits, parent, cand_tokens, path, accept_len, next_token, B, T, V, n_states, T_next,
-        tmpl_parent, tmpl_rank, K, n_ept, ept_mean, topk, kstate, next_parent, next_cand,
-        next_state, dev_status, static_cast<cudaStream_t>(stream)));
+        tmpl_parent, tmpl_rank, K, n_ept, ept_mean, topk, kstate, part_val, part_idx, lse, num_sms(),
+        next_parent, next_cand, next_state, dev_status, static_cast<cudaStream_t>(stream)));
 }
 
 ppd_status ppd_next_tree(const float *logits, const int32_t *parent, const int32_t *cand_tokens,

@@ -208,12 +208,14 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_tree,
 // Next-step candidate tree: at most this many guesses per depth.
 constexpr int kNextMaxK = 16;
 constexpr int kNextMaxEpt = 128;
+constexpr int kNextMaxSplit = 16;   // blocks sharing one row's columns
 
 cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const int32_t *cand,
                              const int32_t *path, const int32_t *accept_len,
                              const int32_t *next_token, int B, int T, int V, int n_states,
                              int T_next, const int32_t *tmpl_parent, const int32_t *tmpl_rank, int K,
                              int n_ept, int ept_mean, int32_t *topk, int32_t *kstate,
+                             float *part_val, int32_t *part_idx, float *lse, int num_sms,
                              int32_t *next_parent, int32_t *next_cand, int32_t *next_state,
                              int32_t *status, cudaStream_t stream);
 

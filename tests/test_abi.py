@@ -71,13 +71,18 @@ def test_verify_step_launch_counts(lib):
 def test_verify_step_forms(lib):
     """The fused step's form: separate grids above 64 sequences, an argmax grid
     first when the logits weigh more than 1/64 of the K/V bytes (the tiny
-    shapes), the argmax in the attention grid's side warps otherwise (the
-    Vicuna-7B shapes), -1 for rejected sizes.  A forced form applies to every
-    fused size until it is reset, and other values are refused."""
+    shapes) or when a narrow argmax grid fits the SMs left idle by the last
+    round of slices (the Vicuna-7B shapes on 152 SMs), the argmax in the
+    attention grid's side warps otherwise, -1 for rejected sizes.  The
+    side-warp case uses 171 layers of the Vicuna-7B shapes: 5472 slices leave
+    fewer than 8 SMs of the last round idle on 148 SMs (the count assumed
+    without a GPU) and none on 152.  A forced form applies to every fused size
+    until it is reset, and other values are refused."""
     from paper_2405_18628_gb300 import ppd
     assert ppd.ppd_verify_step_form(1, 65, 2, 16, 64, 300, 56) == 0
     assert ppd.ppd_verify_step_form(1, 1, 4, 48, 64, 1024, 176) == 1
-    assert ppd.ppd_verify_step_form(32, 1, 32, 64, 128, 32000, 2112) == 2
+    assert ppd.ppd_verify_step_form(171, 1, 32, 64, 128, 32000, 2112) == 2
+    assert ppd.ppd_verify_step_form(32, 1, 32, 64, 128, 32000, 2112) in (1, 2)
     assert ppd.ppd_verify_step_form(1, 1, 4, 48, 96, 1024, 176) == -1
     prev = ppd.ppd_set_verify_step_form(2)
     try:
@@ -92,7 +97,7 @@ def test_verify_step_forms(lib):
         assert ppd.ppd_verify_step_form(1, 1, 4, 48, 64, 1024, 176) == 1
     finally:
         ppd.ppd_set_verify_step_form(-1)
-    assert ppd.ppd_verify_step_form(32, 1, 32, 64, 128, 32000, 2112) == 2
+    assert ppd.ppd_verify_step_form(171, 1, 32, 64, 128, 32000, 2112) == 2
 
 
 def test_host_argument_checks(lib):
