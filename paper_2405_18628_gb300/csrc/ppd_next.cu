@@ -36,6 +36,7 @@ constexpr int kTopkThreads = 512;                  // one tree node per thread (
 constexpr int kTopkWarps = kTopkThreads / 32;
 constexpr int kBatch = 4;                          // 16-byte loads in flight per row and thread
 constexpr float kLog2e = 1.4426950408889634f;
+static_assert(kMaxTree <= kTopkThreads, "find_chains takes one tree node per thread");
 
 // Running log-sum-exp of a row: maximum m, sum s of exp(x - m) over the finite
 // entries, and whether a NaN or +inf was seen.  -inf entries add nothing and
