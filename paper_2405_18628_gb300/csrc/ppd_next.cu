@@ -281,7 +281,6 @@ next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const 
     if (d > cs.k) return;   // uniform over the block
     auto row = [&](int j) { return logits + ((size_t)b * T + cs.node[j]) * V; };
     const bool probs = ept_mean == 1 && n_ept > 1;
-    const int V4 = V >> 2;
     const int c0 = (int)blockIdx.z * chunk, c1 = min(V, c0 + chunk);   // this block's columns
 
     // ---- probability mode: the chain rows' log-sum-exps (next_lse_kernel)
