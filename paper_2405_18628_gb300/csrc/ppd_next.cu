@@ -38,6 +38,15 @@ constexpr int kBatch = 4;                          // 16-byte loads in flight pe
 constexpr float kLog2e = 1.4426950408889634f;
 static_assert(kMaxTree <= kTopkThreads, "find_chains takes one tree node per thread");
 
+// The kernels of one call form a chain of programmatic launches: each lets
+// the next one launch at its entry, and the next does its setup from the
+// call's inputs (the chains, the template) before it waits for the previous
+// grid to complete and reads what that grid wrote.  The first kernel of a
+// call is launched in plain stream order, so the call's inputs are complete
+// before any of its kernels start.
+PPD_DEV void pdl_release() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+PPD_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Running log-sum-exp of a row: maximum m, sum s of exp(x - m) over the finite
 // entries, and whether a NaN or +inf was seen.  -inf entries add nothing and
 // every exponent is a difference <= 0, so nothing overflows.
@@ -214,6 +223,7 @@ next_lse_kernel(const float *__restrict__ logits, const int32_t *parent, const i
     __shared__ int s_b[kTopkWarps];
     const int b = blockIdx.x, d = blockIdx.y + 1, j = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    pdl_release();
     find_chains(cs, parent, cand, path, accept_len, b, d, T, n_states, n_ept);
     if (d > cs.k) return;   // uniform over the block
     const float *x = logits + ((size_t)b * T + cs.node[j]) * V;
@@ -276,7 +286,9 @@ next_topk_kernel(const float *__restrict__ logits, const int32_t *parent, const 
     const int d = blockIdx.y + 1;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
+    pdl_release();
     find_chains(cs, parent, cand, path, accept_len, b, d, T, n_states, n_ept);
+    pdl_wait();   // the log-sum-exps, and the previous call's readers of kstate and the lists
     if (tid == 0 && d == 1 && blockIdx.z == 0) kstate[b] = cs.k;
     if (d > cs.k) return;   // uniform over the block
     auto row = [&](int j) { return logits + ((size_t)b * T + cs.node[j]) * V; };
@@ -435,15 +447,17 @@ next_topk_merge_kernel(const float *part_val, const int32_t *part_idx, int n_sta
                        int n_split, const int32_t *kstate, int32_t *topk)
 {
     const int b = blockIdx.x, d = blockIdx.y + 1, lane = threadIdx.x;
-    if (d > __ldg(kstate + b)) return;   // uniform over the warp
+    pdl_release();
+    pdl_wait();   // the partial lists and the states
+    if (d > __ldcg(kstate + b)) return;   // uniform over the warp
     const size_t base = ((size_t)b * (n_states - 1) + d - 1) * n_split;
     int ptr = 0;
     for (int r = 0; r < K; ++r) {
         float bv = -INFINITY;
         int bi = INT_MAX, bl = lane;
         if (lane < n_split && ptr < K) {
-            bv = part_val[(base + lane) * K + ptr];
-            bi = part_idx[(base + lane) * K + ptr];
+            bv = __ldcg(part_val + (base + lane) * K + ptr);
+            bi = __ldcg(part_idx + (base + lane) * K + ptr);
         }
         warp_best(bv, bi, bl);
         if (lane == 0) topk[((size_t)b * (n_states - 1) + d - 1) * K + r] = bi;
@@ -465,11 +479,12 @@ next_assemble_kernel(const int32_t *parent, const int32_t *cand, const int32_t *
     const int n = __ldg(accept_len + b);
     const int nt = __ldg(next_token + b);
     bool bad = !(n >= 1 && n <= T && nt >= 0);
+    pdl_wait();   // the states and the guesses
     int k = 0;
     if (!bad) {
         const int e = __ldg(path + (size_t)b * T + n - 1);
         bad = !(e >= 0 && e < T);
-        if (!bad && n_states > 1) k = __ldg(kstate + b);
+        if (!bad && n_states > 1) k = __ldcg(kstate + b);
     }
     const int32_t *tp = tmpl_parent + (size_t)k * T_next;
     const int32_t *tr = tmpl_rank + (size_t)k * T_next;
@@ -504,7 +519,7 @@ next_assemble_kernel(const int32_t *parent, const int32_t *cand, const int32_t *
                 if (!ok || depth > k) {
                     tokv = INT_MIN;               // marks a bad template
                 } else {
-                    tokv = __ldg(topk + ((size_t)b * (n_states - 1) + depth - 1) * K + r);
+                    tokv = __ldcg(topk + ((size_t)b * (n_states - 1) + depth - 1) * K + r);
                 }
             }
             nc[i] = tokv;
@@ -527,6 +542,25 @@ next_assemble_kernel(const int32_t *parent, const int32_t *cand, const int32_t *
     }
 }
 
+// A kernel launch, as a programmatic dependent of the stream's previous grid
+// when `chained` (it may then start before that grid completes, and waits
+// for it with griddepcontrol.wait).
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_chained(void (*kern)(KArgs...), dim3 grid, dim3 block, bool chained,
+                                  cudaStream_t stream, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = chained ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const int32_t *cand,
                              const int32_t *path, const int32_t *accept_len,
                              const int32_t *next_token, int B, int T, int V, int n_states,
@@ -536,6 +570,7 @@ cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const i
                              int32_t *next_parent, int32_t *next_cand, int32_t *next_state,
                              int32_t *status, cudaStream_t stream)
 {
+    bool chained = false;   // the call's first kernel waits for the work before it
     if (n_states > 1) {
         const int vec = (V % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
         // each row shared by n_split blocks, about two blocks per SM in all
@@ -545,30 +580,30 @@ cudaError_t launch_next_tree(const float *logits, const int32_t *parent, const i
         int chunk = (V + n_split - 1) / n_split;
         chunk = (chunk + 3) & ~3;
         n_split = (V + chunk - 1) / chunk;
+        const unsigned cap = (unsigned)(n_states - 1);
+        cudaError_t e;
         if (ept_mean == 1 && n_ept > 1) {
-            next_lse_kernel<<<dim3((unsigned)B, (unsigned)(n_states - 1), (unsigned)n_ept),
-                              kTopkThreads, 0, stream>>>(logits, parent, cand, path, accept_len, T,
-                                                         V, n_states, n_ept, vec, lse);
-            const cudaError_t e = cudaGetLastError();
+            e = launch_chained(next_lse_kernel, dim3((unsigned)B, cap, (unsigned)n_ept),
+                               dim3(kTopkThreads), chained, stream, logits, parent, cand, path,
+                               accept_len, T, V, n_states, n_ept, vec, lse);
             if (e != cudaSuccess) return e;
+            chained = true;
         }
-        next_topk_kernel<<<dim3((unsigned)B, (unsigned)(n_states - 1), (unsigned)n_split),
-                           kTopkThreads, 0, stream>>>(logits, parent, cand, path, accept_len, T, V,
-                                                      n_states, K, n_ept, ept_mean, vec, chunk, lse,
-                                                      part_val, part_idx, kstate);
-        cudaError_t e = cudaGetLastError();
+        e = launch_chained(next_topk_kernel, dim3((unsigned)B, cap, (unsigned)n_split),
+                           dim3(kTopkThreads), chained, stream, logits, parent, cand, path,
+                           accept_len, T, V, n_states, K, n_ept, ept_mean, vec, chunk,
+                           (const float *)lse, part_val, part_idx, kstate);
         if (e != cudaSuccess) return e;
-        next_topk_merge_kernel<<<dim3((unsigned)B, (unsigned)(n_states - 1)), 32, 0, stream>>>(
-            part_val, part_idx, n_states, K, n_split, kstate, topk);
-        e = cudaGetLastError();
+        e = launch_chained(next_topk_merge_kernel, dim3((unsigned)B, cap), dim3(32), true, stream,
+                           (const float *)part_val, (const int32_t *)part_idx, n_states, K, n_split,
+                           (const int32_t *)kstate, topk);
         if (e != cudaSuccess) return e;
+        chained = true;
     }
-    next_assemble_kernel<<<(B + 3) / 4, 128, 0, stream>>>(parent, cand, path, accept_len, next_token,
-                                                          B, T, n_states, T_next, tmpl_parent,
-                                                          tmpl_rank, K, topk, kstate,
-                                                          next_parent, next_cand, next_state,
-                                                          status);
-    return cudaGetLastError();
+    return launch_chained(next_assemble_kernel, dim3((unsigned)((B + 3) / 4)), dim3(128), chained,
+                          stream, parent, cand, path, accept_len, next_token, B, T, n_states,
+                          T_next, tmpl_parent, tmpl_rank, K, (const int32_t *)topk,
+                          (const int32_t *)kstate, next_parent, next_cand, next_state, status);
 }
 
 }  // namespace ppd

@@ -285,3 +285,29 @@ def test_next_tree_128_ensemble_chains(cuda_device, ept_mean):
         _compare(got, ref)
     else:
         assert _compare_probs(got, ref, logits, parent, cand, path, alen, tp, tr, n_ept) <= 2
+
+
+@pytest.mark.parametrize("V,K", [(40, 16), (37, 5), (300, 16)])
+def test_next_tree_small_vocab_split_rows(cuda_device, V, K):
+    """Vocabularies so small that each of the blocks sharing a row holds fewer
+    columns than K (V = 40: ten blocks of four columns for sixteen guesses;
+    V = 37: no 16-byte loads), with ties and NaNs: the merged guesses are
+    still the oracle's, bit for bit, in both averaging modes."""
+    w = W.scaled(W.WORKLOADS["tiny"], B=2, V=V, T=16 * (1 + 2 * 3), n_cand=16, chains="ept2x3")
+    s = W.make_step_inputs(w, seed=V)
+    logits = np.round(s.logits * 2.0).astype(np.float32)   # many ties
+    logits[0, :, 3] = np.nan
+    acc = oracle.accept_path(oracle.node_argmax(logits), s.cand_tokens, s.parent, s.prefix_len,
+                             w.V, w.S_max)
+    tp, tr = W.make_tree_templates(4, 48, K, np.random.default_rng(V + K), n_ept=2)
+    for ne, mode in ((2, "logits"), (1, "logits"), (2, "probs")):
+        ref = oracle.next_tree(logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                               acc["next_token"], tp, tr, K, n_ept=ne, ept_mean=mode)
+        got = _run(cuda_device, logits, s.parent, s.cand_tokens, acc["path"], acc["accept_len"],
+                   acc["next_token"], tp, tr, K, n_ept=ne, ept_mean=mode)
+        if mode == "probs":
+            assert _compare_probs(got, ref, logits, s.parent, s.cand_tokens, acc["path"],
+                                  acc["accept_len"], tp, tr, ne) <= 4
+        else:
+            _compare(got, ref)
+        assert (ref["next_state"] > 0).any()
