@@ -74,12 +74,12 @@ REFERENCE_BUDGET_S = 180.0
 # are not in the count, so this is the reads plus the part of the writes that
 # reached DRAM during the launch.
 MEASURED_TRAFFIC = {
-    # 676,500,480 B at 19 layers (reads 667,940,352), x 32/19
-    "vicuna7b": {"bytes_per_launch": 1_139_369_229, "src": "7004aad6620e17ff"},
-    # 1,659,106,304 B at 19 layers (reads 1,650,952,704), x 40/19
-    "vicuna13b": {"bytes_per_launch": 3_492_855_376, "src": "7004aad6620e17ff"},
-    # 123,587,072 B, a fused-step launch at the full 24 layers (reads 119,713,792)
-    "mobilellama": {"bytes_per_launch": 123_587_072, "src": "7004aad6620e17ff"},
+    # 676,148,224 B at 19 layers (reads 667,937,280), x 32/19
+    "vicuna7b": {"bytes_per_launch": 1_138_775_956, "src": "2d25b5ff49083324"},
+    # 1,659,156,992 B at 19 layers (reads 1,650,976,000), x 40/19
+    "vicuna13b": {"bytes_per_launch": 3_492_962_088, "src": "2d25b5ff49083324"},
+    # 123,574,016 B, a fused-step launch at the full 24 layers (reads 119,720,448)
+    "mobilellama": {"bytes_per_launch": 123_574_016, "src": "2d25b5ff49083324"},
 }
 
 
