@@ -1101,6 +1101,10 @@ def main(argv=None):
         next_tree = {"us": nt_ms * 1e3, "states": n_states, "guesses_per_depth": K_guess,
                      "state_histogram": np.bincount(nt_states, minlength=n_states).tolist(),
                      "bytes": nt_bytes, "gbs": nt_bytes / (nt_ms * 1e-3) / 1e9}
+        if nt_bytes == 0:
+            next_tree["note"] = ("state 0 for every sequence: the accepted end node of this "
+                                 "workload's tree carries no prompt chain, so no guesses are "
+                                 "ranked (see \"ensemble\" for a case that ranks them)")
         if extras:
             next_tree["ensemble"] = next_tree_ept(w, dev, stream, K4)
 
